@@ -1,0 +1,200 @@
+"""Test infrastructure: the fp64 CPU oracle for Shift Sparse Block Attention.
+
+This package is NOT part of the product. Only ``tests/``, ``__graft_entry__.smoke()``
+and the CPU-baseline leg of ``bench.py`` may import it. It wraps ``ssba_oracle.c``
+(plain C loops in double precision, written from Sec. 2.2 and Algorithm 1 of the
+paper) through ctypes and shares no code with the CUDA library.
+
+Every function takes numpy arrays, widens them to float64 (bf16 and fp32 widen
+exactly) and returns numpy arrays.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "ssba_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "libssba_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+_I32P = np.ctypeslib.ndpointer(dtype=np.int32, flags="C_CONTIGUOUS")
+_F64P = np.ctypeslib.ndpointer(dtype=np.float64, flags="C_CONTIGUOUS")
+
+
+def build(force: bool = False) -> str:
+    """Compile ssba_oracle.c into libssba_oracle.so next to it (gcc, -O2, OpenMP)."""
+    if force or not os.path.exists(_LIB_PATH) or (
+        os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC)
+    ):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-fno-fast-math",
+               "-ffp-contract=off", _SRC, "-o", tmp, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        build()
+        lib = ctypes.CDLL(_LIB_PATH)
+        c_int, c_double = ctypes.c_int, ctypes.c_double
+        lib.ssba_oracle_drop_count.argtypes = [c_int, c_double]
+        lib.ssba_oracle_keep_count.argtypes = [c_int, c_double]
+        lib.ssba_oracle_partition.argtypes = [c_int, c_int, c_int, c_int, c_int, _I32P]
+        lib.ssba_oracle_pool.argtypes = [_F64P, c_int, c_int, _I32P, c_int, _F64P]
+        lib.ssba_oracle_affinity.argtypes = [_F64P, _F64P, c_int, c_int, _F64P]
+        lib.ssba_oracle_gate.argtypes = [_F64P, c_int, c_int, _I32P]
+        lib.ssba_oracle_attention.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, _I32P, c_int,
+                                              _I32P, c_int, c_double, _F64P, _F64P]
+        lib.ssba_oracle_dense_attention.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, c_double,
+                                                    _F64P, _F64P]
+        lib.ssba_oracle_build_mask_all.argtypes = [_F64P, _F64P, c_int, c_int, c_int, c_int, c_int,
+                                                   c_int, c_int, c_double, _I32P, _I32P,
+                                                   ctypes.c_void_p]
+        lib.ssba_oracle_forward_all.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, c_int, c_int,
+                                                c_int, c_int, c_int, _I32P, c_int, c_double,
+                                                _F64P, _F64P]
+        lib.ssba_oracle_dense_all.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, c_int, c_double,
+                                              _F64P, _F64P]
+        lib.ssba_oracle_set_threads.argtypes = [c_int]
+        lib.ssba_oracle_set_threads.restype = None
+        _lib = lib
+        return lib
+
+
+def _f64(x) -> np.ndarray:
+    if hasattr(x, "detach"):  # torch tensor: widen on the CPU, exactly
+        x = x.detach().to("cpu").double().numpy()
+    return np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+
+
+def _check(rc: int, what: str) -> None:
+    if rc != 0:
+        raise ValueError(f"oracle: {what} rejected its arguments")
+
+
+def max_threads() -> int:
+    return int(_load().ssba_oracle_max_threads())
+
+
+def set_threads(n: int) -> None:
+    _load().ssba_oracle_set_threads(int(n))
+
+
+def drop_count(Tb: int, rho: float) -> int:
+    """k = floor(Tb * rho), the number of key blocks dropped per query block."""
+    return int(_load().ssba_oracle_drop_count(int(Tb), float(rho)))
+
+
+def keep_count(Tb: int, rho: float) -> int:
+    return int(_load().ssba_oracle_keep_count(int(Tb), float(rho)))
+
+
+def partition(H: int, W: int, blk: int = 8, shift=(0, 0)) -> np.ndarray:
+    """Block label of every token of an H x W grid after the cyclic shift."""
+    out = np.empty(H * W, dtype=np.int32)
+    _check(_load().ssba_oracle_partition(H, W, blk, int(shift[0]), int(shift[1]), out),
+           "partition")
+    return out
+
+
+def pool(X, block_of: np.ndarray, Tb: int) -> np.ndarray:
+    X = _f64(X)
+    N, d = X.shape
+    out = np.empty((Tb, d), dtype=np.float64)
+    _check(_load().ssba_oracle_pool(X, N, d, np.ascontiguousarray(block_of, np.int32), Tb, out),
+           "pool")
+    return out
+
+
+def affinity(qb, kb) -> np.ndarray:
+    qb, kb = _f64(qb), _f64(kb)
+    Tb, d = qb.shape
+    out = np.empty((Tb, Tb), dtype=np.float64)
+    _check(_load().ssba_oracle_affinity(qb, kb, Tb, d, out), "affinity")
+    return out
+
+
+def gate(S, k_drop: int) -> np.ndarray:
+    """Kept key-block labels per row, ascending, after dropping the k_drop smallest."""
+    S = _f64(S)
+    Tb = S.shape[0]
+    out = np.empty((Tb, Tb - k_drop), dtype=np.int32)
+    _check(_load().ssba_oracle_gate(S, Tb, int(k_drop), out), "gate")
+    return out
+
+
+def attention(Q, K, V, block_of, idx, scale=None):
+    """Single-slice sparse attention; returns (O [N,d], lse [N])."""
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    N, d = Q.shape
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    Tb, keep = idx.shape
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    O = np.empty((N, d), dtype=np.float64)
+    lse = np.empty(N, dtype=np.float64)
+    _check(_load().ssba_oracle_attention(Q, K, V, N, d, np.ascontiguousarray(block_of, np.int32),
+                                         Tb, idx, keep, scale, O, lse), "attention")
+    return O, lse
+
+
+def dense_attention(Q, K, V, scale=None):
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    N, d = Q.shape
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    O = np.empty((N, d), dtype=np.float64)
+    lse = np.empty(N, dtype=np.float64)
+    _check(_load().ssba_oracle_dense_attention(Q, K, V, N, d, scale, O, lse), "dense_attention")
+    return O, lse
+
+
+def build_mask(Q, K, H: int, W: int, blk: int = 8, shift=(0, 0), rho: float = 0.0,
+               return_scores: bool = False):
+    """Whole-tensor mask build. Q, K: [B, heads, N, d]. Returns (idx, cnt[, S])."""
+    Q, K = _f64(Q), _f64(K)
+    B, h, N, d = Q.shape
+    if N != H * W:
+        raise ValueError("N must equal H*W")
+    Tb = N // (blk * blk)
+    keep = keep_count(Tb, rho)
+    idx = np.empty((B, h, Tb, keep), dtype=np.int32)
+    cnt = np.empty((B, h, Tb), dtype=np.int32)
+    S = np.empty((B, h, Tb, Tb), dtype=np.float64) if return_scores else None
+    _check(_load().ssba_oracle_build_mask_all(
+        Q, K, B * h, H, W, d, blk, int(shift[0]), int(shift[1]), float(rho), idx, cnt,
+        S.ctypes.data if S is not None else None), "build_mask")
+    return (idx, cnt, S) if return_scores else (idx, cnt)
+
+
+def forward(Q, K, V, idx, H: int, W: int, blk: int = 8, shift=(0, 0), scale=None):
+    """Whole-tensor sparse forward. Q, K, V: [B, heads, N, d]; idx [B, heads, Tb, keep]."""
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    B, h, N, d = Q.shape
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    keep = idx.shape[-1]
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    O = np.empty((B, h, N, d), dtype=np.float64)
+    lse = np.empty((B, h, N), dtype=np.float64)
+    _check(_load().ssba_oracle_forward_all(Q, K, V, B * h, H, W, d, blk, int(shift[0]),
+                                           int(shift[1]), idx, keep, scale, O, lse), "forward")
+    return O, lse
+
+
+def dense_forward(Q, K, V, scale=None):
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    B, h, N, d = Q.shape
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    O = np.empty((B, h, N, d), dtype=np.float64)
+    lse = np.empty((B, h, N), dtype=np.float64)
+    _check(_load().ssba_oracle_dense_all(Q, K, V, B * h, N, d, scale, O, lse), "dense_forward")
+    return O, lse

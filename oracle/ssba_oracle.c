@@ -1,0 +1,341 @@
+/*
+ * ssba_oracle.c -- TEST INFRASTRUCTURE, not part of the product.
+ *
+ * A plain, slow, obviously-correct CPU statement in fp64 of Shift Sparse Block
+ * Attention (SSBA) as the paper defines it (Sec. 2.2 "Sparse Block Attention",
+ * Eq. for q_b/k_b, the affinity S = q_b k_b^T, Top-k gating, Algorithm 1, and the
+ * "Window Shift Strategy" that follows it). Only the test-suite, the smoke check
+ * and the CPU-baseline leg of the benchmark may load this library; the CUDA
+ * library shares no code, header, table or helper with it.
+ *
+ * Every array is a single (batch, head) slice unless the name says "_all":
+ *   X        [N][d]   image tokens, token n = r*W + c on an H x W grid (row-major)
+ *   block_of [N]      block label of each token (Sec. 2.2 partition, shifted)
+ *   Xb       [Tb][d]  block means
+ *   S        [Tb][Tb] block affinity
+ *   idx      [Tb][keep] kept key-block labels per query block, ascending
+ *
+ * Readings of the paper taken here (the paper is silent or ambiguous):
+ *   - Top-k is taken per query-block row of S (k = floor(Tb*rho) counts a row).
+ *   - k is the number of DROPPED blocks; keep = Tb - k.
+ *   - Among equal S values, the higher key-block label is dropped first, so the
+ *     lower label is kept.
+ *   - The shift is a plain cyclic roll (torch.roll semantics): the rolled
+ *     position of token (r, c) is ((r + s_r) mod H, (c + s_c) mod W) and blocks
+ *     are the unshifted 8x8 tiles of the rolled grid.
+ *   - Softmax scale is 1/sqrt(d) unless given; lse is a natural log of the sum of
+ *     exp(scaled score).
+ *   - Inputs are taken as post-RoPE (Algorithm 1 applies RoPE before pooling).
+ *   - Only image tokens: the text-token padding of M is not part of this path.
+ *
+ * Pins (tests/test_oracle_*.py): closed forms, brute force over block pairs,
+ * brute-force subset search for the gate, np.roll for the partition, and the
+ * rho = 0 reduction to dense softmax attention.
+ */
+#include <math.h>
+#include <stdint.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+#include <stdlib.h>
+#include <string.h>
+
+#define ORC_OK 0
+#define ORC_BAD 1
+
+/* k = floor(Tb * rho) dropped blocks; keep = Tb - k (Sec. 2.2 Top-k gating,
+ * Algorithm 1 "k <- floor(Tb * rho)"). */
+int ssba_oracle_drop_count(int Tb, double rho)
+{
+    return (int)floor((double)Tb * rho);
+}
+
+int ssba_oracle_keep_count(int Tb, double rho)
+{
+    return Tb - ssba_oracle_drop_count(Tb, rho);
+}
+
+/* Partition into non-overlapping blk x blk blocks after shifting the grid
+ * origin (Sec. 2.2 "Block Compression", Algorithm 1 partition step, and the
+ * window-shift rule implemented with torch.roll).
+ * torch.roll(x, shifts=s) moves the element at r to (r + s) mod H, so token
+ * (r, c) sits at rolled position (u_r, u_c); the unshifted partition of the
+ * rolled grid gives its block (u_r / blk, u_c / blk), labelled row-major. */
+int ssba_oracle_partition(int H, int W, int blk, int shift_r, int shift_c,
+                          int32_t *block_of)
+{
+    if (H <= 0 || W <= 0 || blk <= 0 || H % blk || W % blk || !block_of)
+        return ORC_BAD;
+    int sr = ((shift_r % H) + H) % H;
+    int sc = ((shift_c % W) + W) % W;
+    int bw = W / blk;
+    for (int r = 0; r < H; ++r) {
+        for (int c = 0; c < W; ++c) {
+            int ur = (r + sr) % H;
+            int uc = (c + sc) % W;
+            block_of[r * W + c] = (ur / blk) * bw + (uc / blk);
+        }
+    }
+    return ORC_OK;
+}
+
+/* Block compression: the mean of the tokens of each block (Eq. for
+ * q_b = MeanPool(Q_img), k_b = MeanPool(K_img)). */
+int ssba_oracle_pool(const double *X, int N, int d, const int32_t *block_of,
+                     int Tb, double *Xb)
+{
+    if (!X || !block_of || !Xb || N <= 0 || d <= 0 || Tb <= 0) return ORC_BAD;
+    int *count = (int *)calloc((size_t)Tb, sizeof(int));
+    if (!count) return ORC_BAD;
+    memset(Xb, 0, sizeof(double) * (size_t)Tb * d);
+    for (int n = 0; n < N; ++n) {
+        int b = block_of[n];
+        if (b < 0 || b >= Tb) { free(count); return ORC_BAD; }
+        count[b] += 1;
+        for (int c = 0; c < d; ++c) Xb[(size_t)b * d + c] += X[(size_t)n * d + c];
+    }
+    for (int b = 0; b < Tb; ++b) {
+        if (count[b] == 0) { free(count); return ORC_BAD; }
+        for (int c = 0; c < d; ++c) Xb[(size_t)b * d + c] /= (double)count[b];
+    }
+    free(count);
+    return ORC_OK;
+}
+
+/* Affinity matrix S = q_b k_b^T (Sec. 2.2 "Affinity Matrix"; no scaling). */
+int ssba_oracle_affinity(const double *qb, const double *kb, int Tb, int d, double *S)
+{
+    if (!qb || !kb || !S || Tb <= 0 || d <= 0) return ORC_BAD;
+    for (int i = 0; i < Tb; ++i) {
+        for (int j = 0; j < Tb; ++j) {
+            double acc = 0.0;
+            for (int c = 0; c < d; ++c) acc += qb[(size_t)i * d + c] * kb[(size_t)j * d + c];
+            S[(size_t)i * Tb + j] = acc;
+        }
+    }
+    return ORC_OK;
+}
+
+/* Top-k gating (Sec. 2.2, Algorithm 1 "G <- Top-k Smallest(S, k)"): in each row,
+ * the k_drop smallest entries of S are set to 0 in the gate G; the rest stay 1.
+ * "Smallest" is the total order (S ascending, then label descending), so that of
+ * two equal entries the higher label is dropped. The kept labels (G = 1) are
+ * written in ascending order. */
+int ssba_oracle_gate(const double *S, int Tb, int k_drop, int32_t *idx)
+{
+    if (!S || !idx || Tb <= 0 || k_drop < 0 || k_drop >= Tb) return ORC_BAD;
+    unsigned char *G = (unsigned char *)malloc((size_t)Tb);
+    if (!G) return ORC_BAD;
+    int keep = Tb - k_drop;
+    for (int i = 0; i < Tb; ++i) {
+        const double *row = S + (size_t)i * Tb;
+        for (int j = 0; j < Tb; ++j) G[j] = 1;
+        for (int t = 0; t < k_drop; ++t) {
+            int arg = -1;
+            for (int j = 0; j < Tb; ++j) {
+                if (!G[j]) continue;
+                if (arg < 0 || row[j] < row[arg] || (row[j] == row[arg] && j > arg))
+                    arg = j;
+            }
+            G[arg] = 0;
+        }
+        int w = 0;
+        for (int j = 0; j < Tb; ++j)
+            if (G[j]) idx[(size_t)i * keep + (w++)] = j;
+        if (w != keep) { free(G); return ORC_BAD; }
+    }
+    free(G);
+    return ORC_OK;
+}
+
+/* Sparse attention restricted to the expanded mask (Sec. 2.2 "Efficient Sparse
+ * Execution", Algorithm 1 ExpandMask + SparseAttention, image tokens only).
+ * M(n, m) = 1 iff block_of[m] is among the kept labels of block_of[n]. For each
+ * query n: a_m = scale * <Q_n, K_m> over the allowed keys, mx = max a_m,
+ * lse_n = mx + ln sum exp(a_m - mx), O_n = sum exp(a_m - lse_n) V_m.
+ * Keys are visited kept block by kept block in ascending label order and, inside
+ * a block, in ascending token order. Outputs are in the original token order. */
+int ssba_oracle_attention(const double *Q, const double *K, const double *V,
+                          int N, int d, const int32_t *block_of, int Tb,
+                          const int32_t *idx, int keep, double scale,
+                          double *O, double *lse)
+{
+    if (!Q || !K || !V || !block_of || !idx || !O || !lse) return ORC_BAD;
+    if (N <= 0 || d <= 0 || Tb <= 0 || keep <= 0 || keep > Tb) return ORC_BAD;
+    /* tokens of each block, ascending */
+    int *count = (int *)calloc((size_t)Tb, sizeof(int));
+    int *start = (int *)calloc((size_t)Tb + 1, sizeof(int));
+    int *tok = (int *)malloc(sizeof(int) * (size_t)N);
+    int *fill = (int *)calloc((size_t)Tb, sizeof(int));
+    double *a = (double *)malloc(sizeof(double) * (size_t)N);
+    int *am = (int *)malloc(sizeof(int) * (size_t)N);
+    int rc = ORC_OK;
+    if (!count || !start || !tok || !fill || !a || !am) { rc = ORC_BAD; goto done; }
+    for (int n = 0; n < N; ++n) {
+        if (block_of[n] < 0 || block_of[n] >= Tb) { rc = ORC_BAD; goto done; }
+        count[block_of[n]]++;
+    }
+    for (int b = 0; b < Tb; ++b) start[b + 1] = start[b] + count[b];
+    for (int n = 0; n < N; ++n) {
+        int b = block_of[n];
+        tok[start[b] + fill[b]++] = n;
+    }
+    for (int n = 0; n < N; ++n) {
+        const int32_t *kept = idx + (size_t)block_of[n] * keep;
+        int na = 0;
+        for (int t = 0; t < keep; ++t) {
+            int j = kept[t];
+            if (j < 0 || j >= Tb) { rc = ORC_BAD; goto done; }
+            for (int u = start[j]; u < start[j + 1]; ++u) {
+                int m = tok[u];
+                double dot = 0.0;
+                for (int c = 0; c < d; ++c) dot += Q[(size_t)n * d + c] * K[(size_t)m * d + c];
+                a[na] = scale * dot;
+                am[na] = m;
+                na++;
+            }
+        }
+        double mx = -INFINITY;
+        for (int u = 0; u < na; ++u) if (a[u] > mx) mx = a[u];
+        double sum = 0.0;
+        for (int u = 0; u < na; ++u) sum += exp(a[u] - mx);
+        double l = mx + log(sum);
+        lse[n] = l;
+        for (int c = 0; c < d; ++c) O[(size_t)n * d + c] = 0.0;
+        for (int u = 0; u < na; ++u) {
+            double p = exp(a[u] - l);
+            const double *vm = V + (size_t)am[u] * d;
+            for (int c = 0; c < d; ++c) O[(size_t)n * d + c] += p * vm[c];
+        }
+    }
+done:
+    free(count); free(start); free(tok); free(fill); free(a); free(am);
+    return rc;
+}
+
+/* Dense softmax attention over all N keys (Table 2 "baseline 0%" sparsity). */
+int ssba_oracle_dense_attention(const double *Q, const double *K, const double *V,
+                                int N, int d, double scale, double *O, double *lse)
+{
+    if (!Q || !K || !V || !O || !lse || N <= 0 || d <= 0) return ORC_BAD;
+    double *a = (double *)malloc(sizeof(double) * (size_t)N);
+    if (!a) return ORC_BAD;
+    for (int n = 0; n < N; ++n) {
+        double mx = -INFINITY;
+        for (int m = 0; m < N; ++m) {
+            double dot = 0.0;
+            for (int c = 0; c < d; ++c) dot += Q[(size_t)n * d + c] * K[(size_t)m * d + c];
+            a[m] = scale * dot;
+            if (a[m] > mx) mx = a[m];
+        }
+        double sum = 0.0;
+        for (int m = 0; m < N; ++m) sum += exp(a[m] - mx);
+        double l = mx + log(sum);
+        lse[n] = l;
+        for (int c = 0; c < d; ++c) O[(size_t)n * d + c] = 0.0;
+        for (int m = 0; m < N; ++m) {
+            double p = exp(a[m] - l);
+            for (int c = 0; c < d; ++c) O[(size_t)n * d + c] += p * V[(size_t)m * d + c];
+        }
+    }
+    free(a);
+    return ORC_OK;
+}
+
+/* ---- whole-tensor drivers over [B*heads] slices --------------------------------
+ * Algorithm 1 steps 2-7 for every (batch, head) slice of contiguous
+ * [BH][N][d] tensors. Slices are independent, so the OpenMP loop over slices
+ * does not change any result. */
+
+int ssba_oracle_build_mask_all(const double *Q, const double *K, int BH, int H, int W,
+                               int d, int blk, int shift_r, int shift_c, double rho,
+                               int32_t *idx, int32_t *cnt, double *S_out)
+{
+    if (!Q || !K || !idx || !cnt || BH <= 0 || d <= 0 || blk <= 0) return ORC_BAD;
+    if (H % blk || W % blk || rho < 0.0 || rho >= 1.0) return ORC_BAD;
+    int N = H * W, Tb = N / (blk * blk);
+    int k_drop = ssba_oracle_drop_count(Tb, rho), keep = Tb - k_drop;
+    if (keep < 1) return ORC_BAD;
+    int32_t *block_of = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    if (!block_of) return ORC_BAD;
+    if (ssba_oracle_partition(H, W, blk, shift_r, shift_c, block_of) != ORC_OK) {
+        free(block_of);
+        return ORC_BAD;
+    }
+    int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(|:bad)
+    for (int s = 0; s < BH; ++s) {
+        double *qb = (double *)malloc(sizeof(double) * (size_t)Tb * d);
+        double *kb = (double *)malloc(sizeof(double) * (size_t)Tb * d);
+        double *S = (double *)malloc(sizeof(double) * (size_t)Tb * Tb);
+        if (!qb || !kb || !S) { bad |= 1; free(qb); free(kb); free(S); continue; }
+        bad |= ssba_oracle_pool(Q + (size_t)s * N * d, N, d, block_of, Tb, qb);
+        bad |= ssba_oracle_pool(K + (size_t)s * N * d, N, d, block_of, Tb, kb);
+        bad |= ssba_oracle_affinity(qb, kb, Tb, d, S);
+        bad |= ssba_oracle_gate(S, Tb, k_drop, idx + (size_t)s * Tb * keep);
+        for (int i = 0; i < Tb; ++i) cnt[(size_t)s * Tb + i] = keep;
+        if (S_out) memcpy(S_out + (size_t)s * Tb * Tb, S, sizeof(double) * (size_t)Tb * Tb);
+        free(qb); free(kb); free(S);
+    }
+    free(block_of);
+    return bad ? ORC_BAD : ORC_OK;
+}
+
+int ssba_oracle_forward_all(const double *Q, const double *K, const double *V, int BH,
+                            int H, int W, int d, int blk, int shift_r, int shift_c,
+                            const int32_t *idx, int keep, double scale,
+                            double *O, double *lse)
+{
+    if (!Q || !K || !V || !idx || !O || !lse || BH <= 0 || blk <= 0) return ORC_BAD;
+    if (H % blk || W % blk) return ORC_BAD;
+    int N = H * W, Tb = N / (blk * blk);
+    int32_t *block_of = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    if (!block_of) return ORC_BAD;
+    if (ssba_oracle_partition(H, W, blk, shift_r, shift_c, block_of) != ORC_OK) {
+        free(block_of);
+        return ORC_BAD;
+    }
+    int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(|:bad)
+    for (int s = 0; s < BH; ++s) {
+        size_t off = (size_t)s * N * d;
+        bad |= ssba_oracle_attention(Q + off, K + off, V + off, N, d, block_of, Tb,
+                                     idx + (size_t)s * Tb * keep, keep, scale,
+                                     O + off, lse + (size_t)s * N);
+    }
+    free(block_of);
+    return bad ? ORC_BAD : ORC_OK;
+}
+
+int ssba_oracle_dense_all(const double *Q, const double *K, const double *V, int BH,
+                          int N, int d, double scale, double *O, double *lse)
+{
+    if (BH <= 0) return ORC_BAD;
+    int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(|:bad)
+    for (int s = 0; s < BH; ++s) {
+        size_t off = (size_t)s * N * d;
+        bad |= ssba_oracle_dense_attention(Q + off, K + off, V + off, N, d, scale,
+                                           O + off, lse + (size_t)s * N);
+    }
+    return bad ? ORC_BAD : ORC_OK;
+}
+
+/* Thread control for the timing leg only; results do not depend on it. */
+int ssba_oracle_max_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+void ssba_oracle_set_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}

@@ -1,0 +1,297 @@
+"""Pins of the fp64 oracle against what the paper and mathematics fix.
+
+Each test checks the oracle against an independent statement: np.roll for the
+shifted partition (Sec. 2.2 window shift), pair enumeration for pooled affinity
+(Eq. for q_b/k_b and S = q_b k_b^T), subset search for Top-k gating, a textbook
+numpy softmax for the attention (rho = 0 and masked), closed forms for the
+sparsity rule (Algorithm 1, k = floor(Tb*rho)). A plausible mistake in the oracle
+(a wrong shift sign, a transposed S, a kept/dropped swap, a missing scale, a
+wrong normaliser) fails at least one of them.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "paper_geometry.json")
+
+
+# ----------------------------------------------------------------------------- helpers
+def roll_partition(H, W, blk, shift):
+    """Literal torch.roll semantics: roll the token-index grid, cut 8x8 tiles."""
+    grid = np.arange(H * W).reshape(H, W)
+    rolled = np.roll(grid, shift=(shift[0], shift[1]), axis=(0, 1))
+    lab = np.empty(H * W, dtype=np.int64)
+    bw = W // blk
+    for br in range(H // blk):
+        for bc in range(bw):
+            tile = rolled[br * blk:(br + 1) * blk, bc * blk:(bc + 1) * blk]
+            lab[tile.ravel()] = br * bw + bc
+    return lab
+
+
+def numpy_masked_softmax_attention(Q, K, V, allowed, scale):
+    """Textbook softmax(scale * Q K^T) V with -inf outside ``allowed`` (fp64)."""
+    a = scale * (Q @ K.T)
+    a = np.where(allowed, a, -np.inf)
+    mx = a.max(axis=1, keepdims=True)
+    e = np.exp(a - mx)
+    s = e.sum(axis=1, keepdims=True)
+    P = e / s
+    return P @ V, (mx + np.log(s))[:, 0], P
+
+
+def expand_mask(labels, idx):
+    """M(n, m) = 1 iff label(m) is kept for label(n) (Algorithm 1 ExpandMask)."""
+    N = labels.shape[0]
+    Tb = idx.shape[0]
+    G = np.zeros((Tb, Tb), dtype=bool)
+    for i in range(Tb):
+        G[i, idx[i]] = True
+    return G[labels[:, None], labels[None, :]]
+
+
+# ----------------------------------------------------------------------------- a1 partition
+@pytest.mark.parametrize("H,W", [(16, 16), (32, 32), (16, 40), (64, 64)])
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (-4, -4), (3, -5), (8, 0), (-1, 12), (4, 0)])
+def test_partition_matches_literal_roll(H, W, shift):
+    got = oracle.partition(H, W, 8, shift)
+    want = roll_partition(H, W, 8, shift)
+    assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (-4, -4), (2, 6)])
+def test_partition_invariants(shift):
+    H, W = 32, 48
+    lab = oracle.partition(H, W, 8, shift)
+    Tb = H * W // 64
+    counts = np.bincount(lab, minlength=Tb)
+    assert counts.shape[0] == Tb and np.all(counts == 64)  # every token once, 64 per block
+    for b in range(Tb):  # each block is an 8x8 cyclically contiguous window
+        toks = np.nonzero(lab == b)[0]
+        rows = sorted(set((toks // W).tolist()))
+        cols = sorted(set((toks % W).tolist()))
+        assert len(rows) == 8 and len(cols) == 8
+        r0 = [r for r in rows if (r - 1) % H not in rows]
+        c0 = [c for c in cols if (c - 1) % W not in cols]
+        assert len(r0) == 1 and len(c0) == 1
+        assert set(rows) == {(r0[0] + t) % H for t in range(8)}
+        assert set(cols) == {(c0[0] + t) % W for t in range(8)}
+
+
+def test_plus_minus_four_give_the_same_windows():
+    """Delta=(4,4) and (-4,-4) on an 8-periodic grid give the same set of windows."""
+    H, W = 64, 64
+    a = oracle.partition(H, W, 8, (4, 4))
+    b = oracle.partition(H, W, 8, (-4, -4))
+    sets_a = {frozenset(np.nonzero(a == i)[0].tolist()) for i in range(64)}
+    sets_b = {frozenset(np.nonzero(b == i)[0].tolist()) for i in range(64)}
+    assert sets_a == sets_b
+    # and they differ from the unshifted windows
+    c = oracle.partition(H, W, 8, (0, 0))
+    sets_c = {frozenset(np.nonzero(c == i)[0].tolist()) for i in range(64)}
+    assert sets_a != sets_c
+
+
+# ----------------------------------------------------------------------------- a2/a3 pooling + affinity
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (-3, 5)])
+def test_affinity_equals_pair_enumeration(shift):
+    """S_ij = (1/64^2) sum_{n in i} sum_{m in j} <q_n, k_m>, by explicit pair loops."""
+    rng = np.random.default_rng(1)
+    H = W = 16
+    d = 8
+    N = H * W
+    Q = rng.standard_normal((N, d))
+    K = rng.standard_normal((N, d))
+    lab = roll_partition(H, W, 8, shift)
+    Tb = 4
+    want = np.zeros((Tb, Tb))
+    for n in range(N):
+        for m in range(N):
+            want[lab[n], lab[m]] += float(np.dot(Q[n], K[m]))
+    want /= 64.0 * 64.0
+    olab = oracle.partition(H, W, 8, shift)
+    S = oracle.affinity(oracle.pool(Q, olab, Tb), oracle.pool(K, olab, Tb))
+    np.testing.assert_allclose(S, want, rtol=1e-12, atol=1e-12)
+
+
+def test_pool_constant_blocks_closed_form():
+    H = W = 16
+    lab = oracle.partition(H, W, 8, (4, 4))
+    rng = np.random.default_rng(2)
+    means = rng.standard_normal((4, 5))
+    X = means[lab]
+    np.testing.assert_allclose(oracle.pool(X, lab, 4), means, rtol=1e-14, atol=1e-15)
+
+
+def test_affinity_is_not_transposed():
+    qb = np.array([[1.0, 0.0], [0.0, 2.0]])
+    kb = np.array([[3.0, 5.0], [7.0, 11.0]])
+    S = oracle.affinity(qb, kb)
+    assert S.tolist() == [[3.0, 7.0], [10.0, 22.0]]  # S[i][j] = <qb_i, kb_j>
+
+
+# ----------------------------------------------------------------------------- a4 gate
+@pytest.mark.parametrize("Tb", [4, 5, 6, 8])
+def test_gate_keeps_max_sum_subset(Tb):
+    """With distinct values, the kept set is the unique size-keep subset of max sum."""
+    rng = np.random.default_rng(Tb)
+    S = rng.standard_normal((Tb, Tb))
+    for k_drop in range(Tb):
+        keep = Tb - k_drop
+        got = oracle.gate(S, k_drop)
+        for i in range(Tb):
+            best = max(itertools.combinations(range(Tb), keep), key=lambda c: S[i, list(c)].sum())
+            assert got[i].tolist() == list(best)
+
+
+def test_gate_direction_and_ties():
+    Tb = 8
+    up = np.tile(np.arange(Tb, dtype=float), (Tb, 1))
+    assert oracle.gate(up, 5).tolist() == [[5, 6, 7]] * Tb  # largest kept
+    assert oracle.gate(-up, 5).tolist() == [[0, 1, 2]] * Tb  # smallest dropped
+    flat = np.zeros((Tb, Tb))
+    assert oracle.gate(flat, 6).tolist() == [[0, 1]] * Tb  # ties keep the lower label
+    # a tie at the boundary only: values 3,1,1,0 -> keep 2 -> {0, 1}
+    S = np.array([[3.0, 1.0, 1.0, 0.0]] * 4)
+    assert oracle.gate(S, 2).tolist() == [[0, 1]] * 4
+    # -0.0 and +0.0 are equal values: the lower label is kept
+    S = np.array([[-0.0, 0.0, -1.0, -2.0]] * 4)
+    assert oracle.gate(S, 3).tolist() == [[0]] * 4
+
+
+def test_gate_invariants_random():
+    rng = np.random.default_rng(5)
+    Tb = 64
+    S = rng.standard_normal((Tb, Tb))
+    for k_drop in (0, 1, 32, 53, 63):
+        idx = oracle.gate(S, k_drop)
+        assert idx.shape == (Tb, Tb - k_drop)
+        for i in range(Tb):
+            row = idx[i]
+            assert np.all(np.diff(row) > 0) and row.min() >= 0 and row.max() < Tb
+            dropped = np.setdiff1d(np.arange(Tb), row)
+            if len(dropped):
+                assert S[i, row].min() >= S[i, dropped].max()
+
+
+# ----------------------------------------------------------------------------- sparsity rule
+def test_sparsity_rule_closed_forms():
+    g = json.load(open(GOLDEN))
+    assert g["vae_example"]["tokens"] == (g["vae_example"]["image_px"] // 8 // 2) ** 2
+    Tb512 = g["vae_example"]["tokens"] // g["block"]["tokens_per_block"]
+    assert Tb512 == 16
+    # Algorithm 1: k = floor(Tb * rho) dropped
+    cases = [(16, 0.75, 12), (16, 0.8416, 13), (64, 0.8416, 53), (64, 0.85, 54),
+             (256, 0.84, 215), (256, 0.9, 230), (4, 0.75, 3), (64, 0.0, 0)]
+    for Tb, rho, k in cases:
+        assert oracle.drop_count(Tb, rho) == k == math.floor(Tb * rho)
+        assert oracle.keep_count(Tb, rho) == Tb - k
+    # realised sparsity equals rho when Tb*rho is an integer (75% of 16 blocks)
+    assert oracle.drop_count(16, g["sparsity"]["vanilla"]) / 16 == g["sparsity"]["vanilla"]
+
+
+# ----------------------------------------------------------------------------- whole mask, crafted inputs
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4)])
+@pytest.mark.parametrize("sign", [1.0, -1.0])
+def test_build_mask_crafted_block_means(shift, sign):
+    """K tokens of block j equal (j+1) e1 and Q tokens equal sign*e1, so S_ij = sign*(j+1)."""
+    H = W = 32
+    d = 64
+    lab = roll_partition(H, W, 8, shift)
+    Tb = 16
+    K = np.zeros((1, 1, H * W, d))
+    K[0, 0, :, 0] = lab + 1.0
+    Q = np.zeros((1, 1, H * W, d))
+    Q[0, 0, :, 0] = sign
+    rho = 0.75
+    keep = Tb - math.floor(Tb * rho)
+    idx, cnt, S = oracle.build_mask(Q, K, H, W, 8, shift, rho, return_scores=True)
+    want_S = sign * np.tile(np.arange(1, Tb + 1, dtype=float), (Tb, 1))
+    np.testing.assert_array_equal(S[0, 0], want_S)
+    want = list(range(Tb - keep, Tb)) if sign > 0 else list(range(keep))
+    assert idx[0, 0].tolist() == [want] * Tb
+    assert np.all(cnt == keep)
+
+
+# ----------------------------------------------------------------------------- a6 attention
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (-4, -4), (3, 1)])
+def test_rho_zero_equals_dense_softmax(shift):
+    rng = np.random.default_rng(7)
+    H = W = 16
+    N, d = H * W, 64
+    Q, K, V = (rng.standard_normal((1, 2, N, d)) for _ in range(3))
+    idx, cnt = oracle.build_mask(Q, K, H, W, 8, shift, 0.0)
+    assert idx.shape[-1] == 4 and np.all(cnt == 4)
+    O, lse = oracle.forward(Q, K, V, idx, H, W, 8, shift)
+    for h in range(2):
+        want_O, want_lse, _ = numpy_masked_softmax_attention(
+            Q[0, h], K[0, h], V[0, h], np.ones((N, N), bool), 1 / 8.0)
+        np.testing.assert_allclose(O[0, h], want_O, rtol=1e-10, atol=1e-12)
+        np.testing.assert_allclose(lse[0, h], want_lse, rtol=1e-12, atol=1e-12)
+    Od, lsed = oracle.dense_forward(Q, K, V)
+    np.testing.assert_allclose(Od, O, rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(lsed, lse, rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (2, -6)])
+def test_masked_attention_equals_numpy_masked_softmax(shift):
+    rng = np.random.default_rng(11)
+    H, W = 16, 24
+    N, d = H * W, 64
+    Q, K, V = (rng.standard_normal((1, 1, N, d)) for _ in range(3))
+    rho = 0.5
+    idx, _ = oracle.build_mask(Q, K, H, W, 8, shift, rho)
+    O, lse = oracle.forward(Q, K, V, idx, H, W, 8, shift, scale=0.3)
+    allowed = expand_mask(roll_partition(H, W, 8, shift), idx[0, 0])
+    want_O, want_lse, P = numpy_masked_softmax_attention(Q[0, 0], K[0, 0], V[0, 0], allowed, 0.3)
+    np.testing.assert_allclose(O[0, 0], want_O, rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(lse[0, 0], want_lse, rtol=1e-12, atol=1e-12)
+    # realised density: each query sees exactly keep*64 keys
+    assert np.all(allowed.sum(axis=1) == idx.shape[-1] * 64)
+    np.testing.assert_allclose(P.sum(axis=1), 1.0, rtol=0, atol=1e-12)
+
+
+def test_attention_rows_normalised_and_lse_definition():
+    rng = np.random.default_rng(3)
+    H = W = 16
+    N, d = H * W, 64
+    Q, K = (rng.standard_normal((1, 1, N, d)) for _ in range(2))
+    ones = np.ones((1, 1, N, d))
+    idx, _ = oracle.build_mask(Q, K, H, W, 8, (4, 4), 0.75)
+    O, lse = oracle.forward(Q, K, ones, idx, H, W, 8, (4, 4))
+    np.testing.assert_allclose(O, 1.0, rtol=0, atol=1e-13)  # sum_m P_nm = 1
+    lab = roll_partition(H, W, 8, (4, 4))
+    allowed = expand_mask(lab, idx[0, 0])
+    a = (Q[0, 0] @ K[0, 0].T) / 8.0
+    for n in range(0, N, 17):
+        want = math.log(sum(math.exp(x) for x in a[n][allowed[n]]))
+        assert abs(lse[0, 0, n] - want) < 1e-12
+
+
+def test_keep_one_own_block_is_local_attention():
+    rng = np.random.default_rng(4)
+    H = W = 16
+    N, d = H * W, 64
+    Q, K, V = (rng.standard_normal((N, d)) for _ in range(3))
+    lab = oracle.partition(H, W, 8, (4, 4))
+    idx = np.arange(4, dtype=np.int32)[:, None]  # each block attends only to itself
+    O, lse = oracle.attention(Q, K, V, lab, idx)
+    for b in range(4):
+        toks = np.nonzero(roll_partition(H, W, 8, (4, 4)) == b)[0]
+        want_O, want_lse, _ = numpy_masked_softmax_attention(
+            Q[toks], K[toks], V[toks], np.ones((64, 64), bool), 1 / 8.0)
+        np.testing.assert_allclose(O[toks], want_O, rtol=1e-10, atol=1e-12)
+        np.testing.assert_allclose(lse[toks], want_lse, rtol=1e-12, atol=1e-12)
+
+
+def test_oracle_rejects_bad_arguments():
+    with pytest.raises(ValueError):
+        oracle.partition(12, 16, 8, (0, 0))  # 12 is not a multiple of 8
+    with pytest.raises(ValueError):
+        oracle.gate(np.zeros((4, 4)), 4)  # keep would be 0
