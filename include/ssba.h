@@ -1,0 +1,143 @@
+/*
+ * ssba.h -- C ABI of the GB300 (sm_103a) Shift Sparse Block Attention library.
+ *
+ * Shift Sparse Block Attention (SSBA) is defined in Sec. 2.2 of the ElasticDiT
+ * paper: the image-token grid is cut into non-overlapping 8x8 token blocks (the
+ * grid origin shifted by half a block on alternating layers, "Window Shift
+ * Strategy"), each block's queries and keys are mean-pooled (Eq. for q_b, k_b),
+ * the block affinity S = q_b k_b^T is formed, the k = floor(Tb * rho) smallest
+ * entries of every row of S are masked ("Top-k Gating", Algorithm 1), and
+ * softmax attention runs only over the key blocks that remain ("Efficient
+ * Sparse Execution", Algorithm 1 SparseAttention).
+ *
+ * Conventions shared by every call
+ *   Layout     Q, K, V, O are contiguous [B][heads][N][head_dim] with token
+ *              n = r * W_tok + c on the row-major H_tok x W_tok grid.
+ *   Ownership  The caller allocates every buffer (device memory unless a
+ *              parameter says otherwise); the library allocates nothing and keeps
+ *              no pointer after a call returns.
+ *   Streams    `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *              stream). Every call only enqueues work and returns.
+ *   Errors     Arguments are validated on the host; a bad descriptor, a null or
+ *              misaligned pointer, or an unsupported shape returns a non-zero
+ *              ssba_status and launches nothing. A failed launch returns
+ *              SSBA_ERR_CUDA. A device-side failure (a bounded wait that ran out)
+ *              is recorded in a device status word read by ssba_get_status().
+ *              ssba_last_error() gives the thread's last message. Nothing aborts,
+ *              throws across the ABI, or traps on the device.
+ */
+#ifndef SSBA_H_
+#define SSBA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SSBA_API __attribute__((visibility("default")))
+#else
+#define SSBA_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    SSBA_OK = 0,
+    SSBA_ERR_INVALID = 1,     /* bad descriptor, null/misaligned pointer, bad sizes        */
+    SSBA_ERR_UNSUPPORTED = 2, /* valid for the method but outside the kernels' fast path   */
+    SSBA_ERR_CUDA = 3,        /* a CUDA runtime/driver call or launch failed               */
+    SSBA_ERR_TIMEOUT = 4,     /* (device status) a bounded wait inside a kernel ran out    */
+    SSBA_ERR_WORKSPACE = 5    /* workspace missing or smaller than ssba_mask_workspace_bytes */
+} ssba_status;
+
+typedef enum { SSBA_BF16 = 0, SSBA_FP32 = 1 } ssba_dtype;
+
+/* One SSBA layer's geometry and sparsity rule.
+ *   B, heads, head_dim   tensor sizes; head_dim = C of Sec. 2.2 (per head).
+ *   H_tok, W_tok         image-token grid; both multiples of `block`.
+ *   block                block side (8 in the paper: 8x8 = 64 tokens per block).
+ *   shift_r, shift_c     window shift Delta of the layer (Sec. 2.2 Window Shift),
+ *                        torch.roll semantics: token (r, c) moves to
+ *                        ((r + shift_r) mod H_tok, (c + shift_c) mod W_tok) before
+ *                        the unshifted partition. Any integer (reduced mod H, W).
+ *   rho                  sparse ratio, 0 <= rho < 1; k_drop = floor(Tb * rho)
+ *                        blocks are dropped per query block, keep = Tb - k_drop.
+ *   dtype                ssba_dtype of Q, K, V and O.
+ *   softmax_scale        scale of q.k inside the softmax; 0 selects 1/sqrt(head_dim). */
+typedef struct {
+    int32_t B, heads, H_tok, W_tok, head_dim;
+    int32_t block;
+    int32_t shift_r, shift_c;
+    double rho;
+    int32_t dtype;
+    float softmax_scale;
+} ssba_desc;
+
+/* Number of key blocks kept per query block: Tb - floor(Tb * rho), Tb =
+ * H_tok * W_tok / block^2 (Algorithm 1, "k <- floor(Tb * rho)" with k dropped).
+ * Returns -1 for an invalid descriptor. */
+SSBA_API int ssba_keep_count(const ssba_desc* desc);
+
+/* Bytes of device workspace ssba_build_mask needs (the pooled block sums of Q
+ * and K in fp32, 2 * B * heads * Tb * head_dim * 4 bytes, 256-byte aligned).
+ * Returns 0 for an invalid descriptor. */
+SSBA_API size_t ssba_mask_workspace_bytes(const ssba_desc* desc);
+
+/* Builds the block mask of one layer (Sec. 2.2 Block Compression, Affinity
+ * Matrix, Top-k Gating; Algorithm 1 partition .. Top-k Smallest).
+ *   Q, K        device, [B][heads][N][head_dim] of desc->dtype (post-RoPE).
+ *   kv_idx      device out, int32 [B][heads][Tb][keep]: for each query block, the
+ *               labels of its kept key blocks in ascending order. Block label
+ *               i = (u_r / block) * (W_tok / block) + (u_c / block) where
+ *               (u_r, u_c) is the rolled position of the block's tokens.
+ *   kv_cnt      device out, int32 [B][heads][Tb]: number of valid entries of
+ *               each kv_idx row (always keep).
+ *   scores_opt  device out or NULL, fp32 [B][heads][Tb][Tb]: the affinity S
+ *               (block means, no scaling) the selection was made on.
+ *   workspace   device scratch of at least ssba_mask_workspace_bytes(desc),
+ *               16-byte aligned; contents are overwritten.
+ * Ties in S keep the lower label. Any shift and head_dim in [1, 256] multiple of
+ * 8 (bf16) or 4 (fp32) are supported. */
+SSBA_API int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K, int32_t* kv_idx,
+                    int32_t* kv_cnt, float* scores_opt, void* workspace, size_t ws_bytes,
+                    void* stream);
+
+/* Block-sparse attention forward (Sec. 2.2 Efficient Sparse Execution;
+ * Algorithm 1 ExpandMask + SparseAttention, image tokens only): for every query
+ * token n of block i = label(n), softmax over the keys of the blocks listed in
+ * kv_idx[b][h][i][0 .. kv_cnt-1]:
+ *   lse_n = ln sum_m exp(scale * q_n.k_m),  O_n = sum_m exp(scale * q_n.k_m - lse_n) v_m.
+ *   Q, K, V     device, [B][heads][N][head_dim] of desc->dtype.
+ *   kv_idx      device, int32 [B][heads][Tb][keep] labels in [0, Tb) (as written by
+ *               ssba_build_mask for the same desc; any order, no repeats).
+ *   kv_cnt      device, int32 [B][heads][Tb], each in [1, keep].
+ *   O           device out, [B][heads][N][head_dim] of desc->dtype, original token order.
+ *   lse         device out, fp32 [B][heads][N], natural log.
+ * bf16 runs on the tcgen05 tensor-core kernel and needs head_dim = 64, block = 8
+ * and shifts that are multiples of 4; fp32 runs on the CUDA-core kernel with any
+ * shift and head_dim = 64. Anything else returns SSBA_ERR_UNSUPPORTED. */
+SSBA_API int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void* V,
+                 const int32_t* kv_idx, const int32_t* kv_cnt, void* O, float* lse,
+                 void* stream);
+
+/* Dense softmax attention over all N keys with the same layout and outputs as
+ * ssba_forward (the 0% sparsity "baseline" of Table 2), from the same build:
+ * bf16 only, head_dim = 64, H_tok and W_tok multiples of 8 (block is ignored).
+ * Shift and rho are ignored. */
+SSBA_API int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, const void* V,
+                       void* O, float* lse, void* stream);
+
+/* Reads and clears the device status word of the current device (SSBA_OK or
+ * SSBA_ERR_TIMEOUT). Synchronous: call after the caller's stream sync. Returns
+ * SSBA_OK, or SSBA_ERR_CUDA if the read failed. */
+SSBA_API int ssba_get_status(int32_t* device_status_out);
+
+/* Message of the calling thread's last failed call ("" if none). */
+SSBA_API const char* ssba_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SSBA_H_ */

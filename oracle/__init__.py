@@ -56,6 +56,8 @@ def _load():
         lib.ssba_oracle_gate.argtypes = [_F64P, c_int, c_int, _I32P]
         lib.ssba_oracle_attention.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, _I32P, c_int,
                                               _I32P, c_int, c_double, _F64P, _F64P]
+        lib.ssba_oracle_attention_rows.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, _I32P, c_int,
+                                                   _I32P, c_int, c_double, _I32P, c_int, _F64P, _F64P]
         lib.ssba_oracle_dense_attention.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, c_double,
                                                     _F64P, _F64P]
         lib.ssba_oracle_build_mask_all.argtypes = [_F64P, _F64P, c_int, c_int, c_int, c_int, c_int,
@@ -145,6 +147,22 @@ def attention(Q, K, V, block_of, idx, scale=None):
     lse = np.empty(N, dtype=np.float64)
     _check(_load().ssba_oracle_attention(Q, K, V, N, d, np.ascontiguousarray(block_of, np.int32),
                                          Tb, idx, keep, scale, O, lse), "attention")
+    return O, lse
+
+
+def attention_rows(Q, K, V, block_of, idx, rows, scale=None):
+    """Single-slice sparse attention for the listed query tokens only."""
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    N, d = Q.shape
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    Tb, keep = idx.shape
+    rows = np.ascontiguousarray(rows, dtype=np.int32)
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    O = np.empty((rows.shape[0], d), dtype=np.float64)
+    lse = np.empty(rows.shape[0], dtype=np.float64)
+    _check(_load().ssba_oracle_attention_rows(Q, K, V, N, d, np.ascontiguousarray(block_of, np.int32),
+                                              Tb, idx, keep, scale, rows, rows.shape[0], O, lse),
+           "attention_rows")
     return O, lse
 
 

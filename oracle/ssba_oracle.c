@@ -148,13 +148,68 @@ int ssba_oracle_gate(const double *S, int Tb, int k_drop, int32_t *idx)
     return ORC_OK;
 }
 
+/* Tokens of every block in ascending token order: tok[start[b] .. start[b+1]). */
+static int block_lists(int N, const int32_t *block_of, int Tb, int *start, int *tok)
+{
+    int *fill = (int *)calloc((size_t)Tb + 1, sizeof(int));
+    if (!fill) return ORC_BAD;
+    for (int b = 0; b <= Tb; ++b) start[b] = 0;
+    for (int n = 0; n < N; ++n) {
+        if (block_of[n] < 0 || block_of[n] >= Tb) { free(fill); return ORC_BAD; }
+        start[block_of[n] + 1]++;
+    }
+    for (int b = 0; b < Tb; ++b) start[b + 1] += start[b];
+    for (int n = 0; n < N; ++n) {
+        int b = block_of[n];
+        tok[start[b] + fill[b]++] = n;
+    }
+    free(fill);
+    return ORC_OK;
+}
+
+/* One query row of the sparse attention (see ssba_oracle_attention). a and am are
+ * scratch arrays of N entries. */
+static int attend_row(const double *Q, const double *K, const double *V, int d, int n,
+                      const int32_t *block_of, int Tb, const int32_t *idx, int keep,
+                      double scale, const int *start, const int *tok, double *a, int *am,
+                      double *O_row, double *lse_n)
+{
+    const int32_t *kept = idx + (size_t)block_of[n] * keep;
+    int na = 0;
+    for (int t = 0; t < keep; ++t) {
+        int j = kept[t];
+        if (j < 0 || j >= Tb) return ORC_BAD;
+        for (int u = start[j]; u < start[j + 1]; ++u) {
+            int m = tok[u];
+            double dot = 0.0;
+            for (int c = 0; c < d; ++c) dot += Q[(size_t)n * d + c] * K[(size_t)m * d + c];
+            a[na] = scale * dot;
+            am[na] = m;
+            na++;
+        }
+    }
+    double mx = -INFINITY;
+    for (int u = 0; u < na; ++u) if (a[u] > mx) mx = a[u];
+    double sum = 0.0;
+    for (int u = 0; u < na; ++u) sum += exp(a[u] - mx);
+    double l = mx + log(sum);
+    *lse_n = l;
+    for (int c = 0; c < d; ++c) O_row[c] = 0.0;
+    for (int u = 0; u < na; ++u) {
+        double p = exp(a[u] - l);
+        const double *vm = V + (size_t)am[u] * d;
+        for (int c = 0; c < d; ++c) O_row[c] += p * vm[c];
+    }
+    return ORC_OK;
+}
+
 /* Sparse attention restricted to the expanded mask (Sec. 2.2 "Efficient Sparse
  * Execution", Algorithm 1 ExpandMask + SparseAttention, image tokens only).
  * M(n, m) = 1 iff block_of[m] is among the kept labels of block_of[n]. For each
  * query n: a_m = scale * <Q_n, K_m> over the allowed keys, mx = max a_m,
  * lse_n = mx + ln sum exp(a_m - mx), O_n = sum exp(a_m - lse_n) V_m.
- * Keys are visited kept block by kept block in ascending label order and, inside
- * a block, in ascending token order. Outputs are in the original token order. */
+ * Keys are visited kept block by kept block in list order and, inside a block, in
+ * ascending token order. Outputs are in the original token order. */
 int ssba_oracle_attention(const double *Q, const double *K, const double *V,
                           int N, int d, const int32_t *block_of, int Tb,
                           const int32_t *idx, int keep, double scale,
@@ -162,54 +217,38 @@ int ssba_oracle_attention(const double *Q, const double *K, const double *V,
 {
     if (!Q || !K || !V || !block_of || !idx || !O || !lse) return ORC_BAD;
     if (N <= 0 || d <= 0 || Tb <= 0 || keep <= 0 || keep > Tb) return ORC_BAD;
-    /* tokens of each block, ascending */
-    int *count = (int *)calloc((size_t)Tb, sizeof(int));
-    int *start = (int *)calloc((size_t)Tb + 1, sizeof(int));
+    int *start = (int *)malloc(sizeof(int) * ((size_t)Tb + 1));
     int *tok = (int *)malloc(sizeof(int) * (size_t)N);
-    int *fill = (int *)calloc((size_t)Tb, sizeof(int));
     double *a = (double *)malloc(sizeof(double) * (size_t)N);
     int *am = (int *)malloc(sizeof(int) * (size_t)N);
-    int rc = ORC_OK;
-    if (!count || !start || !tok || !fill || !a || !am) { rc = ORC_BAD; goto done; }
-    for (int n = 0; n < N; ++n) {
-        if (block_of[n] < 0 || block_of[n] >= Tb) { rc = ORC_BAD; goto done; }
-        count[block_of[n]]++;
+    int rc = (start && tok && a && am) ? block_lists(N, block_of, Tb, start, tok) : ORC_BAD;
+    for (int n = 0; n < N && rc == ORC_OK; ++n)
+        rc = attend_row(Q, K, V, d, n, block_of, Tb, idx, keep, scale, start, tok, a, am,
+                        O + (size_t)n * d, lse + n);
+    free(start); free(tok); free(a); free(am);
+    return rc;
+}
+
+/* The same attention for the listed query tokens only: O_rows[r], lse_rows[r] are
+ * the outputs of token rows[r]. Used to check full-size runs on sampled rows. */
+int ssba_oracle_attention_rows(const double *Q, const double *K, const double *V,
+                               int N, int d, const int32_t *block_of, int Tb,
+                               const int32_t *idx, int keep, double scale,
+                               const int32_t *rows, int nrows, double *O_rows, double *lse_rows)
+{
+    if (!Q || !K || !V || !block_of || !idx || !rows || !O_rows || !lse_rows) return ORC_BAD;
+    if (N <= 0 || d <= 0 || Tb <= 0 || keep <= 0 || keep > Tb || nrows < 0) return ORC_BAD;
+    int *start = (int *)malloc(sizeof(int) * ((size_t)Tb + 1));
+    int *tok = (int *)malloc(sizeof(int) * (size_t)N);
+    double *a = (double *)malloc(sizeof(double) * (size_t)N);
+    int *am = (int *)malloc(sizeof(int) * (size_t)N);
+    int rc = (start && tok && a && am) ? block_lists(N, block_of, Tb, start, tok) : ORC_BAD;
+    for (int r = 0; r < nrows && rc == ORC_OK; ++r) {
+        if (rows[r] < 0 || rows[r] >= N) { rc = ORC_BAD; break; }
+        rc = attend_row(Q, K, V, d, rows[r], block_of, Tb, idx, keep, scale, start, tok, a, am,
+                        O_rows + (size_t)r * d, lse_rows + r);
     }
-    for (int b = 0; b < Tb; ++b) start[b + 1] = start[b] + count[b];
-    for (int n = 0; n < N; ++n) {
-        int b = block_of[n];
-        tok[start[b] + fill[b]++] = n;
-    }
-    for (int n = 0; n < N; ++n) {
-        const int32_t *kept = idx + (size_t)block_of[n] * keep;
-        int na = 0;
-        for (int t = 0; t < keep; ++t) {
-            int j = kept[t];
-            if (j < 0 || j >= Tb) { rc = ORC_BAD; goto done; }
-            for (int u = start[j]; u < start[j + 1]; ++u) {
-                int m = tok[u];
-                double dot = 0.0;
-                for (int c = 0; c < d; ++c) dot += Q[(size_t)n * d + c] * K[(size_t)m * d + c];
-                a[na] = scale * dot;
-                am[na] = m;
-                na++;
-            }
-        }
-        double mx = -INFINITY;
-        for (int u = 0; u < na; ++u) if (a[u] > mx) mx = a[u];
-        double sum = 0.0;
-        for (int u = 0; u < na; ++u) sum += exp(a[u] - mx);
-        double l = mx + log(sum);
-        lse[n] = l;
-        for (int c = 0; c < d; ++c) O[(size_t)n * d + c] = 0.0;
-        for (int u = 0; u < na; ++u) {
-            double p = exp(a[u] - l);
-            const double *vm = V + (size_t)am[u] * d;
-            for (int c = 0; c < d; ++c) O[(size_t)n * d + c] += p * vm[c];
-        }
-    }
-done:
-    free(count); free(start); free(tok); free(fill); free(a); free(am);
+    free(start); free(tok); free(a); free(am);
     return rc;
 }
 

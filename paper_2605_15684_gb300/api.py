@@ -1,0 +1,239 @@
+"""ctypes binding of libssba.so (include/ssba.h), same names as the C entry points.
+
+Argument marshalling only: tensors are checked for device, dtype, shape and
+contiguity, their ``data_ptr()`` and the current CUDA stream are handed to the C
+call, and a non-zero status is raised as ``SsbaError``. Every step of the path
+runs in the library's kernels; there is no Python or CPU fallback, and the
+library must exist (``paper_2605_15684_gb300.build.build()`` makes it).
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+import threading
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libssba.so")
+_lock = threading.Lock()
+_lib = None
+
+SSBA_OK, SSBA_ERR_INVALID, SSBA_ERR_UNSUPPORTED, SSBA_ERR_CUDA, SSBA_ERR_TIMEOUT, SSBA_ERR_WORKSPACE = range(6)
+SSBA_BF16, SSBA_FP32 = 0, 1
+_STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED", 3: "SSBA_ERR_CUDA",
+                 4: "SSBA_ERR_TIMEOUT", 5: "SSBA_ERR_WORKSPACE"}
+
+EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_forward",
+            "ssba_forward_dense", "ssba_get_status", "ssba_last_error")
+
+
+class SsbaError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{_STATUS_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+class _Desc(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("heads", ctypes.c_int32), ("H_tok", ctypes.c_int32),
+                ("W_tok", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("block", ctypes.c_int32),
+                ("shift_r", ctypes.c_int32), ("shift_c", ctypes.c_int32), ("rho", ctypes.c_double),
+                ("dtype", ctypes.c_int32), ("softmax_scale", ctypes.c_float)]
+
+
+@dataclass
+class SsbaDesc:
+    """Python mirror of ``ssba_desc``."""
+    B: int
+    heads: int
+    H_tok: int
+    W_tok: int
+    head_dim: int = 64
+    block: int = 8
+    shift_r: int = 0
+    shift_c: int = 0
+    rho: float = 0.0
+    dtype: torch.dtype = torch.bfloat16
+    softmax_scale: float = 0.0
+
+    @property
+    def N(self) -> int:
+        return self.H_tok * self.W_tok
+
+    @property
+    def Tb(self) -> int:
+        return self.N // (self.block * self.block)
+
+    def c(self) -> _Desc:
+        if self.dtype == torch.bfloat16:
+            dt = SSBA_BF16
+        elif self.dtype == torch.float32:
+            dt = SSBA_FP32
+        else:
+            raise SsbaError(SSBA_ERR_INVALID, f"unsupported dtype {self.dtype}")
+        return _Desc(self.B, self.heads, self.H_tok, self.W_tok, self.head_dim, self.block,
+                     self.shift_r, self.shift_c, float(self.rho), dt, float(self.softmax_scale))
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def load_library():
+    """Load libssba.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(_LIB_PATH):
+            raise SsbaError(SSBA_ERR_CUDA, f"{_LIB_PATH} is missing: run paper_2605_15684_gb300.build.build()")
+        lib = ctypes.CDLL(_LIB_PATH)
+        P = ctypes.c_void_p
+        DP = ctypes.POINTER(_Desc)
+        lib.ssba_keep_count.argtypes = [DP]
+        lib.ssba_keep_count.restype = ctypes.c_int
+        lib.ssba_mask_workspace_bytes.argtypes = [DP]
+        lib.ssba_mask_workspace_bytes.restype = ctypes.c_size_t
+        lib.ssba_build_mask.argtypes = [DP, P, P, P, P, P, P, ctypes.c_size_t, P]
+        lib.ssba_build_mask.restype = ctypes.c_int
+        lib.ssba_forward.argtypes = [DP, P, P, P, P, P, P, P, P]
+        lib.ssba_forward.restype = ctypes.c_int
+        lib.ssba_forward_dense.argtypes = [DP, P, P, P, P, P, P]
+        lib.ssba_forward_dense.restype = ctypes.c_int
+        lib.ssba_get_status.argtypes = [ctypes.POINTER(ctypes.c_int32)]
+        lib.ssba_get_status.restype = ctypes.c_int
+        lib.ssba_last_error.argtypes = []
+        lib.ssba_last_error.restype = ctypes.c_char_p
+        _lib = lib
+        return lib
+
+
+def _raise_on(rc: int) -> None:
+    if rc != SSBA_OK:
+        raise SsbaError(rc, _lib.ssba_last_error().decode(errors="replace"))
+
+
+def _stream_ptr(stream) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+def _check(t: torch.Tensor, name: str, shape, dtype) -> None:
+    if not isinstance(t, torch.Tensor):
+        raise SsbaError(SSBA_ERR_INVALID, f"{name} must be a torch.Tensor")
+    if t.device.type != "cuda":
+        raise SsbaError(SSBA_ERR_INVALID, f"{name} must be a CUDA tensor (got {t.device})")
+    if tuple(t.shape) != tuple(shape):
+        raise SsbaError(SSBA_ERR_INVALID, f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    if t.dtype != dtype:
+        raise SsbaError(SSBA_ERR_INVALID, f"{name} has dtype {t.dtype}, expected {dtype}")
+    if not t.is_contiguous():
+        raise SsbaError(SSBA_ERR_INVALID, f"{name} must be contiguous")
+
+
+def keep_count(desc: SsbaDesc) -> int:
+    lib = load_library()
+    d = desc.c()
+    k = lib.ssba_keep_count(ctypes.byref(d))
+    if k < 0:
+        _raise_on(SSBA_ERR_INVALID)
+    return k
+
+
+def mask_workspace_bytes(desc: SsbaDesc) -> int:
+    lib = load_library()
+    d = desc.c()
+    return int(lib.ssba_mask_workspace_bytes(ctypes.byref(d)))
+
+
+def build_mask(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=None, kv_cnt=None,
+               scores: bool | torch.Tensor = False, workspace=None, stream=None):
+    """ssba_build_mask: returns (kv_idx [B,h,Tb,keep] int32, kv_cnt [B,h,Tb] int32[, S])."""
+    lib = load_library()
+    d = desc.c()
+    keep = lib.ssba_keep_count(ctypes.byref(d))
+    if keep < 0:
+        _raise_on(SSBA_ERR_INVALID)
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    _check(Q, "Q", shp, desc.dtype)
+    _check(K, "K", shp, desc.dtype)
+    dev = Q.device
+    if kv_idx is None:
+        kv_idx = torch.empty((desc.B, desc.heads, desc.Tb, keep), dtype=torch.int32, device=dev)
+    if kv_cnt is None:
+        kv_cnt = torch.empty((desc.B, desc.heads, desc.Tb), dtype=torch.int32, device=dev)
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    S = None
+    if isinstance(scores, torch.Tensor):
+        S = scores
+        _check(S, "scores", (desc.B, desc.heads, desc.Tb, desc.Tb), torch.float32)
+    elif scores:
+        S = torch.empty((desc.B, desc.heads, desc.Tb, desc.Tb), dtype=torch.float32, device=dev)
+    ws_need = int(lib.ssba_mask_workspace_bytes(ctypes.byref(d)))
+    if workspace is None:
+        workspace = torch.empty(ws_need, dtype=torch.uint8, device=dev)
+    rc = lib.ssba_build_mask(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), kv_idx.data_ptr(),
+                             kv_cnt.data_ptr(), S.data_ptr() if S is not None else None,
+                             workspace.data_ptr(), workspace.numel() * workspace.element_size(),
+                             _stream_ptr(stream))
+    _raise_on(rc)
+    return (kv_idx, kv_cnt, S) if S is not None else (kv_idx, kv_cnt)
+
+
+def forward(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O=None, lse=None, stream=None):
+    """ssba_forward: returns (O [B,h,N,d] in desc.dtype, lse [B,h,N] fp32)."""
+    lib = load_library()
+    d = desc.c()
+    keep = lib.ssba_keep_count(ctypes.byref(d))
+    if keep < 0:
+        _raise_on(SSBA_ERR_INVALID)
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
+        _check(t, n, shp, desc.dtype)
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    if O is None:
+        O = torch.empty(shp, dtype=desc.dtype, device=Q.device)
+    if lse is None:
+        lse = torch.empty(shp[:3], dtype=torch.float32, device=Q.device)
+    _check(O, "O", shp, desc.dtype)
+    _check(lse, "lse", shp[:3], torch.float32)
+    rc = lib.ssba_forward(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), kv_idx.data_ptr(),
+                          kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), _stream_ptr(stream))
+    _raise_on(rc)
+    return O, lse
+
+
+def forward_dense(desc: SsbaDesc, Q, K, V, O=None, lse=None, stream=None):
+    """ssba_forward_dense: dense softmax attention from the same build."""
+    lib = load_library()
+    d = desc.c()
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
+        _check(t, n, shp, desc.dtype)
+    if O is None:
+        O = torch.empty(shp, dtype=desc.dtype, device=Q.device)
+    if lse is None:
+        lse = torch.empty(shp[:3], dtype=torch.float32, device=Q.device)
+    _check(O, "O", shp, desc.dtype)
+    _check(lse, "lse", shp[:3], torch.float32)
+    rc = lib.ssba_forward_dense(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), O.data_ptr(),
+                                lse.data_ptr(), _stream_ptr(stream))
+    _raise_on(rc)
+    return O, lse
+
+
+def get_status() -> int:
+    """ssba_get_status: read-and-clear the device status word (call after a sync)."""
+    lib = load_library()
+    v = ctypes.c_int32(0)
+    _raise_on(lib.ssba_get_status(ctypes.byref(v)))
+    return int(v.value)
+
+
+def realized_sparsity(desc: SsbaDesc) -> float:
+    """k_drop / Tb with k_drop = floor(Tb * rho) (host arithmetic, no device call)."""
+    return math.floor(desc.Tb * desc.rho) / desc.Tb

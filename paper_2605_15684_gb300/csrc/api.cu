@@ -1,0 +1,231 @@
+// api.cu -- the extern "C" boundary declared in include/ssba.h: argument
+// validation on the host, workspace carving, and kernel launches on the caller's
+// stream. Nothing here allocates device memory.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "common.cuh"
+
+namespace ssba {
+
+__device__ int g_status = 0;
+
+int* device_status_word()
+{
+    constexpr int kMaxDev = 64;
+    static int* addr[kMaxDev] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return nullptr;
+    if (!addr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
+        addr[dev] = static_cast<int*>(p);
+    }
+    return addr[dev];
+}
+
+namespace {
+thread_local char t_err[512] = "";
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Shared validation of a descriptor; fills the grid geometry and the keep count.
+int check_desc(const ssba_desc* d, const char* who, Grid* g, int* keep)
+{
+    if (!d) {
+        set_error("%s: null descriptor", who);
+        return SSBA_ERR_INVALID;
+    }
+    if (d->B <= 0 || d->heads <= 0 || d->H_tok <= 0 || d->W_tok <= 0 || d->head_dim <= 0 || d->block <= 0) {
+        set_error("%s: sizes must be positive (B=%d heads=%d H=%d W=%d d=%d block=%d)", who, d->B, d->heads,
+                  d->H_tok, d->W_tok, d->head_dim, d->block);
+        return SSBA_ERR_INVALID;
+    }
+    if (d->H_tok % d->block || d->W_tok % d->block) {
+        set_error("%s: H_tok=%d and W_tok=%d must be multiples of block=%d", who, d->H_tok, d->W_tok, d->block);
+        return SSBA_ERR_INVALID;
+    }
+    if (!(d->rho >= 0.0 && d->rho < 1.0)) {
+        set_error("%s: rho=%g must satisfy 0 <= rho < 1", who, d->rho);
+        return SSBA_ERR_INVALID;
+    }
+    if (d->dtype != SSBA_BF16 && d->dtype != SSBA_FP32) {
+        set_error("%s: unknown dtype %d", who, d->dtype);
+        return SSBA_ERR_INVALID;
+    }
+    if (!(d->softmax_scale >= 0.f) || std::isinf(d->softmax_scale)) {
+        set_error("%s: softmax_scale must be finite and >= 0 (0 = 1/sqrt(head_dim))", who);
+        return SSBA_ERR_INVALID;
+    }
+    const long long N = (long long)d->H_tok * d->W_tok;
+    const long long total = N * d->B * d->heads * d->head_dim;
+    if (total > (1LL << 40) || N > (1LL << 26)) {
+        set_error("%s: tensor too large", who);
+        return SSBA_ERR_INVALID;
+    }
+    g->H = d->H_tok;
+    g->W = d->W_tok;
+    g->blk = d->block;
+    g->sr = ((d->shift_r % d->H_tok) + d->H_tok) % d->H_tok;
+    g->sc = ((d->shift_c % d->W_tok) + d->W_tok) % d->W_tok;
+    g->bw = d->W_tok / d->block;
+    const int Tb = g->Tb();
+    const int k_drop = (int)std::floor((double)Tb * d->rho);
+    *keep = Tb - k_drop;
+    if (*keep < 1) {
+        set_error("%s: keep = Tb - floor(Tb*rho) = %d must be >= 1", who, *keep);
+        return SSBA_ERR_INVALID;
+    }
+    return SSBA_OK;
+}
+
+float resolve_scale(const ssba_desc* d)
+{
+    return d->softmax_scale > 0.f ? d->softmax_scale : 1.0f / std::sqrt((float)d->head_dim);
+}
+
+size_t elem_size(const ssba_desc* d) { return d->dtype == SSBA_BF16 ? 2 : 4; }
+
+}  // namespace
+
+void set_error(const char* fmt, ...)
+{
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(t_err, sizeof(t_err), fmt, ap);
+    va_end(ap);
+}
+
+}  // namespace ssba
+
+using namespace ssba;
+
+extern "C" {
+
+int ssba_keep_count(const ssba_desc* desc)
+{
+    Grid g;
+    int keep;
+    if (check_desc(desc, "ssba_keep_count", &g, &keep) != SSBA_OK) return -1;
+    return keep;
+}
+
+size_t ssba_mask_workspace_bytes(const ssba_desc* desc)
+{
+    Grid g;
+    int keep;
+    if (check_desc(desc, "ssba_mask_workspace_bytes", &g, &keep) != SSBA_OK) return 0;
+    size_t one = (size_t)desc->B * desc->heads * g.Tb() * desc->head_dim * sizeof(float);
+    one = (one + 255) & ~(size_t)255;
+    return 2 * one;
+}
+
+int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K, int32_t* kv_idx, int32_t* kv_cnt,
+                    float* scores_opt, void* workspace, size_t ws_bytes, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_build_mask", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !kv_idx || !kv_cnt) {
+        set_error("ssba_build_mask: Q, K, kv_idx and kv_cnt must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    const size_t es = elem_size(desc);
+    if ((desc->head_dim * es) % 16 || desc->head_dim > 256) {
+        set_error("ssba_build_mask: head_dim*elem must be a multiple of 16 bytes and head_dim <= 256");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) ||
+        (scores_opt && !aligned(scores_opt, 4))) {
+        set_error("ssba_build_mask: Q and K must be 16-byte aligned, outputs 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    const size_t need = ssba_mask_workspace_bytes(desc);
+    if (!workspace || ws_bytes < need || !aligned(workspace, 16)) {
+        set_error("ssba_build_mask: workspace of %zu bytes (16-byte aligned) required, got %zu", need, ws_bytes);
+        return SSBA_ERR_WORKSPACE;
+    }
+    float* qb = static_cast<float*>(workspace);
+    float* kb = reinterpret_cast<float*>(static_cast<char*>(workspace) + need / 2);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    rc = launch_pool(*desc, g, Q, K, qb, kb, st);
+    if (rc != SSBA_OK) return rc;
+    return launch_select(*desc, g, keep, qb, kb, kv_idx, kv_cnt, scores_opt, st);
+}
+
+int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void* V, const int32_t* kv_idx,
+                 const int32_t* kv_cnt, void* O, float* lse, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_forward", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !V || !kv_idx || !kv_cnt || !O || !lse) {
+        set_error("ssba_forward: every pointer must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(lse, 4) ||
+        !aligned(kv_idx, 4) || !aligned(kv_cnt, 4)) {
+        set_error("ssba_forward: Q, K, V, O must be 16-byte aligned; lse, kv_idx, kv_cnt 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    const float scale = resolve_scale(desc);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (desc->dtype == SSBA_FP32)
+        return launch_attn_simt_f32(*desc, g, keep, scale, static_cast<const float*>(Q),
+                                    static_cast<const float*>(K), static_cast<const float*>(V), kv_idx, kv_cnt,
+                                    static_cast<float*>(O), lse, st);
+    return launch_attn_tc_bf16(*desc, g, keep, scale, Q, K, V, kv_idx, kv_cnt, O, lse, st);
+}
+
+int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, const void* V, void* O, float* lse,
+                       void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_forward_dense", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !V || !O || !lse) {
+        set_error("ssba_forward_dense: every pointer must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(lse, 4)) {
+        set_error("ssba_forward_dense: Q, K, V, O must be 16-byte aligned; lse 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    if (desc->dtype != SSBA_BF16) {
+        set_error("ssba_forward_dense: bf16 only");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    return launch_dense_tc_bf16(*desc, resolve_scale(desc), Q, K, V, O, lse,
+                                static_cast<cudaStream_t>(stream));
+}
+
+int ssba_get_status(int32_t* device_status_out)
+{
+    if (!device_status_out) {
+        set_error("ssba_get_status: null output");
+        return SSBA_ERR_INVALID;
+    }
+    int v = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(&v, g_status, sizeof(int));
+    if (e != cudaSuccess) {
+        set_error("ssba_get_status: %s", cudaGetErrorString(e));
+        return SSBA_ERR_CUDA;
+    }
+    const int zero = 0;
+    e = cudaMemcpyToSymbol(g_status, &zero, sizeof(int));
+    if (e != cudaSuccess) {
+        set_error("ssba_get_status: %s", cudaGetErrorString(e));
+        return SSBA_ERR_CUDA;
+    }
+    *device_status_out = v;
+    return SSBA_OK;
+}
+
+const char* ssba_last_error(void) { return t_err; }
+
+}  // extern "C"

@@ -1,0 +1,55 @@
+// common.cuh -- shared definitions of the CUDA library (not shared with the oracle).
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+
+#include "ssba.h"
+
+namespace ssba {
+
+// Device address of the status word (SSBA_OK or SSBA_ERR_TIMEOUT) of the current
+// device, read by ssba_get_status(); kernels that wait receive it as a parameter.
+int* device_status_word();
+
+// Token grid with the window shift of one layer (Sec. 2.2, Window Shift Strategy).
+// A block label is row-major over the blk x blk tiles of the rolled grid; the
+// token at in-block position (a, b) of label (br, bc) sits at rolled position
+// (br*blk + a, bc*blk + b), i.e. at original position (rolled - shift) mod size.
+struct Grid {
+    int H, W, blk;
+    int sr, sc;  // shifts reduced to [0, H) and [0, W)
+    int bw;      // W / blk (labels per block-row)
+
+    __host__ __device__ int Tb() const { return (H / blk) * bw; }
+
+    __device__ __forceinline__ int token(int label, int pos) const
+    {
+        int br = label / bw, bc = label - br * bw;
+        int a = pos / blk, b = pos - a * blk;
+        int r = br * blk + a - sr;
+        if (r < 0) r += H;
+        int c = bc * blk + b - sc;
+        if (c < 0) c += W;
+        return r * W + c;
+    }
+};
+
+// Host-side launchers (defined in the .cu files, called by api.cu).
+int launch_pool(const ssba_desc& d, const Grid& g, const void* Q, const void* K, float* qb, float* kb,
+                cudaStream_t st);
+int launch_select(const ssba_desc& d, const Grid& g, int keep, const float* qb, const float* kb,
+                  int32_t* idx, int32_t* cnt, float* scores, cudaStream_t st);
+int launch_attn_simt_f32(const ssba_desc& d, const Grid& g, int keep, float scale, const float* Q,
+                         const float* K, const float* V, const int32_t* idx, const int32_t* cnt, float* O,
+                         float* lse, cudaStream_t st);
+int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q,
+                        const void* K, const void* V, const int32_t* idx, const int32_t* cnt, void* O,
+                        float* lse, cudaStream_t st);
+int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V,
+                         void* O, float* lse, cudaStream_t st);
+
+// Thread-local error text for ssba_last_error().
+void set_error(const char* fmt, ...);
+
+}  // namespace ssba

@@ -1,0 +1,120 @@
+"""Host-side checks of the C-ABI library: it builds, loads without a GPU, exports
+every symbol include/ssba.h declares, and its host validation returns the
+documented status codes before any device work (no compute call is made here)."""
+import ctypes
+import math
+import os
+import re
+import subprocess
+
+import pytest
+
+import oracle
+from paper_2605_15684_gb300 import api, build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "ssba.h")
+FAKE = 0x100000  # a 16-byte aligned, never dereferenced address
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return api.load_library()
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"SSBA_API\s+[\w\s\*]+?\b(ssba_\w+)\s*\(", text)))
+
+
+def desc(**kw):
+    base = dict(B=1, heads=2, H_tok=16, W_tok=16, head_dim=64, block=8, shift_r=4, shift_c=4, rho=0.75,
+                dtype=api.SSBA_BF16, softmax_scale=0.0)
+    base.update(kw)
+    return api._Desc(**base)
+
+
+def test_header_declares_the_documented_entry_points():
+    assert declared_symbols() == sorted(api.EXPORTED)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_symbols():
+        assert hasattr(lib, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", api.library_path()], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (ssba_\w+)", out))
+    assert set(declared_symbols()) <= exported
+    # nothing else of ours leaks out of the library
+    assert exported == set(declared_symbols())
+
+
+@pytest.mark.parametrize("H,W,rho", [(16, 16, 0.75), (32, 32, 0.8416), (64, 64, 0.8416), (64, 64, 0.85),
+                                     (128, 128, 0.84), (128, 128, 0.9), (16, 40, 0.5), (64, 64, 0.0)])
+def test_keep_count_matches_the_sparsity_rule(lib, H, W, rho):
+    Tb = H * W // 64
+    d = desc(H_tok=H, W_tok=W, rho=rho)
+    assert lib.ssba_keep_count(ctypes.byref(d)) == Tb - math.floor(Tb * rho) == oracle.keep_count(Tb, rho)
+
+
+def test_workspace_bytes(lib):
+    d = desc(B=1, heads=24, H_tok=64, W_tok=64)
+    one = 24 * 64 * 64 * 4
+    assert lib.ssba_mask_workspace_bytes(ctypes.byref(d)) == 2 * ((one + 255) // 256 * 256)
+    assert lib.ssba_mask_workspace_bytes(ctypes.byref(desc(H_tok=12))) == 0
+
+
+@pytest.mark.parametrize("bad", [dict(H_tok=12), dict(W_tok=0), dict(rho=1.0), dict(rho=-0.1),
+                                 dict(dtype=7), dict(B=0), dict(softmax_scale=-1.0),
+                                 dict(head_dim=0)])
+def test_invalid_descriptors_are_rejected(lib, bad):
+    d = desc(**bad)
+    assert lib.ssba_keep_count(ctypes.byref(d)) == -1
+    rc = lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None)
+    assert rc == api.SSBA_ERR_INVALID
+    assert lib.ssba_last_error()
+
+
+def test_null_and_misaligned_pointers(lib):
+    d = desc()
+    ws = lib.ssba_mask_workspace_bytes(ctypes.byref(d))
+    assert lib.ssba_build_mask(ctypes.byref(d), None, FAKE, FAKE, FAKE, None, FAKE, ws, None) == \
+        api.SSBA_ERR_INVALID
+    assert lib.ssba_build_mask(ctypes.byref(d), FAKE + 2, FAKE, FAKE, FAKE, None, FAKE, ws, None) == \
+        api.SSBA_ERR_INVALID
+    assert lib.ssba_build_mask(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, None, FAKE, ws - 1, None) == \
+        api.SSBA_ERR_WORKSPACE
+    assert lib.ssba_build_mask(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, None, None, ws, None) == \
+        api.SSBA_ERR_WORKSPACE
+    assert lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, None) == \
+        api.SSBA_ERR_INVALID
+    assert lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE + 8, FAKE, FAKE, FAKE, FAKE, None) == \
+        api.SSBA_ERR_INVALID
+    assert b"aligned" in lib.ssba_last_error()
+
+
+@pytest.mark.parametrize("bad", [dict(shift_r=2), dict(shift_c=-6), dict(head_dim=128), dict(block=16, H_tok=32,
+                                                                                            W_tok=32)])
+def test_tensor_core_path_rejects_unsupported_shapes(lib, bad):
+    """The bf16 path needs head_dim 64, 8x8 blocks and 4-aligned shifts; it says so before launching."""
+    d = desc(**bad)
+    rc = lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None)
+    assert rc == api.SSBA_ERR_UNSUPPORTED
+    assert b"multiples of 4" in lib.ssba_last_error()
+
+
+def test_build_mask_rejects_unsupported_head_dim(lib):
+    d = desc(head_dim=12)  # 24 bytes per bf16 row: not a multiple of 16
+    ws = lib.ssba_mask_workspace_bytes(ctypes.byref(d))
+    assert lib.ssba_build_mask(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, None, FAKE, ws, None) == \
+        api.SSBA_ERR_UNSUPPORTED
+
+
+def test_python_binding_validates_before_calling(lib):
+    import torch
+    dsc = api.SsbaDesc(B=1, heads=2, H_tok=16, W_tok=16, rho=0.75)
+    q = torch.zeros(1, 2, 256, 64, dtype=torch.bfloat16)
+    with pytest.raises(api.SsbaError, match="CUDA tensor"):
+        api.build_mask(dsc, q, q)
+    assert api.realized_sparsity(api.SsbaDesc(1, 24, 64, 64, rho=0.8416)) == 53 / 64

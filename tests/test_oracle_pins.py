@@ -295,3 +295,18 @@ def test_oracle_rejects_bad_arguments():
         oracle.partition(12, 16, 8, (0, 0))  # 12 is not a multiple of 8
     with pytest.raises(ValueError):
         oracle.gate(np.zeros((4, 4)), 4)  # keep would be 0
+
+
+def test_attention_rows_matches_numpy_on_sampled_rows():
+    rng = np.random.default_rng(12)
+    H, W = 16, 32
+    N, d = H * W, 64
+    Q, K, V = (rng.standard_normal((N, d)) for _ in range(3))
+    lab = oracle.partition(H, W, 8, (4, 4))
+    idx = oracle.gate(rng.standard_normal((8, 8)), 5)
+    rows = np.array([0, 5, 77, 300, N - 1], dtype=np.int32)
+    O, lse = oracle.attention_rows(Q, K, V, lab, idx, rows)
+    allowed = expand_mask(roll_partition(H, W, 8, (4, 4)), idx)
+    want_O, want_lse, _ = numpy_masked_softmax_attention(Q, K, V, allowed, 1 / 8.0)
+    np.testing.assert_allclose(O, want_O[rows], rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(lse, want_lse[rows], rtol=1e-12, atol=1e-12)

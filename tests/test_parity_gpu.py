@@ -1,0 +1,183 @@
+"""GPU parity: the CUDA path through the C-ABI against the fp64 oracle, element by
+element, on the seeded synthetic workloads (tolerances in tests/parity.py)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2605_15684_gb300 import api, build, synthetic
+from tests.parity import check_mask, check_out
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    api.load_library()
+    yield
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
+
+
+def _inputs(B, h, H, W, dtype, seed=0, std=1.0):
+    q, k, v = synthetic.qkv(B, h, H * W, 64, dtype, seed, std)
+    return q, k, v, q.cuda(), k.cuda(), v.cuda()
+
+
+def _mask_case(B, h, H, W, dtype, shift, rho, seed=0, std=1.0):
+    q, k, v, qd, kd, vd = _inputs(B, h, H, W, dtype, seed, std)
+    desc = api.SsbaDesc(B, h, H, W, shift_r=shift[0], shift_c=shift[1], rho=rho, dtype=dtype)
+    idx, cnt, S = api.build_mask(desc, qd, kd, scores=True)
+    torch.cuda.synchronize()
+    idx_o, cnt_o, S_o = oracle.build_mask(q, k, H, W, 8, shift, rho, return_scores=True)
+    keep = oracle.keep_count(H * W // 64, rho)
+    near = check_mask(idx.cpu().numpy(), cnt.cpu().numpy(), S.cpu().numpy(), S_o, idx_o, keep)
+    return desc, (q, k, v, qd, kd, vd), idx_o, near
+
+
+# ----------------------------------------------------------------------------- mask (K1)
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (-4, -4), (3, -5)])
+def test_mask_tiny(dtype, shift):
+    """Tiny case: 16x16 grid, 2 heads, 4 blocks, ~75% sparsity."""
+    _mask_case(1, 2, 16, 16, dtype, shift, 0.75)
+
+
+@pytest.mark.parametrize("H,W,B,rho,shift", [
+    (32, 32, 1, 0.8416, (0, 0)),      # 512 px, unshifted layer
+    (32, 32, 1, 0.8416, (4, 4)),      # 512 px, shifted layer
+    (64, 64, 1, 0.8416, (4, 4)),      # 1024 px headline
+    (64, 64, 4, 0.5, (0, 0)),         # elastic sweep, batch 4
+    (24, 40, 2, 0.6, (4, -4)),        # non-square, odd block count (15)
+    (128, 128, 1, 0.84, (4, 4)),      # 2048 px stress (Tb = 256, two key chunks)
+])
+def test_mask_full_configs(H, W, B, rho, shift):
+    std = 0.125 if H == 32 else 1.0
+    _, _, _, near = _mask_case(B, 24, H, W, torch.bfloat16, shift, rho, std=std)
+    assert near < 0.1 * B * 24 * (H * W // 64)
+
+
+def test_mask_ties_keep_lower_label():
+    """Constant Q/K make every S entry equal: each row keeps labels 0..keep-1."""
+    H = W = 32
+    q = torch.ones(1, 2, H * W, 64, dtype=torch.bfloat16, device="cuda")
+    desc = api.SsbaDesc(1, 2, H, W, shift_r=4, shift_c=4, rho=0.75)
+    idx, cnt = api.build_mask(desc, q, q)
+    keep = 16 - 12
+    assert idx.shape == (1, 2, 16, keep)
+    assert bool((idx.cpu() == torch.arange(keep, dtype=torch.int32)).all())
+    assert bool((cnt.cpu() == keep).all())
+
+
+def test_mask_keep_one_and_all():
+    for rho, keep in ((0.95, 1), (0.0, 16)):
+        desc, _, idx_o, _ = _mask_case(1, 3, 32, 32, torch.bfloat16, (4, 4), rho)
+        assert idx_o.shape[-1] == keep
+
+
+# ----------------------------------------------------------------------------- forward (K2/K3)
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (3, -5)])
+@pytest.mark.parametrize("rho", [0.75, 0.0])
+def test_forward_fp32_tiny(shift, rho):
+    """fp32 tiny case (CUDA-core kernel): <= 1e-4 against the oracle; rho = 0 is dense."""
+    H = W = 16
+    q, k, v, qd, kd, vd = _inputs(1, 2, H, W, torch.float32)
+    desc = api.SsbaDesc(1, 2, H, W, shift_r=shift[0], shift_c=shift[1], rho=rho, dtype=torch.float32)
+    idx_o, cnt_o = oracle.build_mask(q, k, H, W, 8, shift, rho)
+    O, lse = api.forward(desc, qd, kd, vd, torch.from_numpy(idx_o).cuda(), torch.from_numpy(cnt_o).cuda())
+    torch.cuda.synchronize()
+    O_o, lse_o = oracle.forward(q, k, v, idx_o, H, W, 8, shift)
+    check_out(O.cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "fp32")
+    if rho == 0.0:
+        O_d, lse_d = oracle.dense_forward(q, k, v)
+        check_out(O.cpu().numpy(), lse.cpu().numpy(), O_d, lse_d, "fp32")
+
+
+def _bf16_forward_case(B, h, H, W, shift, rho, std=1.0, seed=0):
+    q, k, v, qd, kd, vd = _inputs(B, h, H, W, torch.bfloat16, seed, std)
+    desc = api.SsbaDesc(B, h, H, W, shift_r=shift[0], shift_c=shift[1], rho=rho)
+    idx_o, cnt_o = oracle.build_mask(q, k, H, W, 8, shift, rho)
+    O, lse = api.forward(desc, qd, kd, vd, torch.from_numpy(idx_o).cuda(), torch.from_numpy(cnt_o).cuda())
+    torch.cuda.synchronize()
+    O_o, lse_o = oracle.forward(q, k, v, idx_o, H, W, 8, shift)
+    return check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (-4, -4), (4, -8)])
+def test_forward_bf16_tiny_grid(shift):
+    _bf16_forward_case(1, 2, 16, 16, shift, 0.75)
+
+
+@pytest.mark.parametrize("H,W,B,h,rho,shift,std", [
+    (32, 32, 1, 24, 0.8416, (4, 4), 0.125),   # 512 px config (scaled inputs)
+    (32, 32, 1, 24, 0.8416, (0, 0), 1.0),     # 512 px grid, unit variance
+    (64, 64, 1, 24, 0.8416, (4, 4), 1.0),     # 1024 px headline (1536 items, ragged over the grid)
+    (64, 64, 1, 8, 0.0, (0, 0), 1.0),         # keep = Tb: dense through the sparse kernel
+    (32, 32, 2, 6, 0.95, (4, 4), 1.0),        # keep = 1
+    (24, 40, 2, 5, 0.6, (4, -4), 1.0),        # non-square grid, odd Tb
+])
+def test_forward_bf16_configs(H, W, B, h, rho, shift, std):
+    _bf16_forward_case(B, h, H, W, shift, rho, std)
+
+
+def test_forward_bf16_large_logits_rescale_path():
+    """Inputs scaled so that scores span tens of units: the running max must grow
+    mid-row, exercising the in-TMEM O rescale."""
+    H = W = 32
+    q, k, v, qd, kd, vd = _inputs(1, 4, H, W, torch.float32, seed=3)
+    ramp = torch.linspace(0.2, 4.0, H * W).view(1, 1, H * W, 1)
+    q = (q * 3.0).to(torch.bfloat16)
+    k = (k * ramp).to(torch.bfloat16)
+    v = v.to(torch.bfloat16)
+    desc = api.SsbaDesc(1, 4, H, W, rho=0.5)
+    idx_o, cnt_o = oracle.build_mask(q, k, H, W, 8, (0, 0), 0.5)
+    O, lse = api.forward(desc, q.cuda(), k.cuda(), v.cuda(), torch.from_numpy(idx_o).cuda(),
+                         torch.from_numpy(cnt_o).cuda())
+    torch.cuda.synchronize()
+    O_o, lse_o = oracle.forward(q, k, v, idx_o, H, W, 8, (0, 0))
+    check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
+def test_forward_bf16_2048px_sampled_rows():
+    """Full 2048 px size (N=16384, 24 heads, keep 41): GPU mask on every head against the
+    oracle, GPU forward checked on sampled query rows of two heads."""
+    H = W = 128
+    desc, (q, k, v, qd, kd, vd), idx_o, _ = _mask_case(1, 24, H, W, torch.bfloat16, (4, 4), 0.84)
+    O, lse = api.forward(desc, qd, kd, vd, torch.from_numpy(idx_o).cuda(),
+                         torch.full((1, 24, 256), idx_o.shape[-1], dtype=torch.int32, device="cuda"))
+    torch.cuda.synchronize()
+    lab = oracle.partition(H, W, 8, (4, 4))
+    rng = np.random.default_rng(0)
+    rows = np.sort(rng.choice(H * W, 96, replace=False)).astype(np.int32)
+    for head in (0, 23):
+        O_o, lse_o = oracle.attention_rows(q[0, head], k[0, head], v[0, head], lab, idx_o[0, head], rows)
+        check_out(O[0, head].float().cpu().numpy()[rows], lse[0, head].cpu().numpy()[rows], O_o, lse_o, "bf16")
+
+
+def test_forward_dense_bf16():
+    H = W = 32
+    q, k, v, qd, kd, vd = _inputs(1, 4, H, W, torch.bfloat16)
+    desc = api.SsbaDesc(1, 4, H, W)
+    O, lse = api.forward_dense(desc, qd, kd, vd)
+    torch.cuda.synchronize()
+    O_o, lse_o = oracle.dense_forward(q, k, v)
+    check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
+def test_end_to_end_layer_with_gpu_mask():
+    """build_mask then forward on the GPU (the path bench.py times), against the oracle
+    forward run on the GPU's own lists."""
+    H = W = 64
+    q, k, v, qd, kd, vd = _inputs(1, 24, H, W, torch.bfloat16, seed=1)
+    desc = api.SsbaDesc(1, 24, H, W, shift_r=4, shift_c=4, rho=0.8416)
+    idx, cnt = api.build_mask(desc, qd, kd)
+    O, lse = api.forward(desc, qd, kd, vd, idx, cnt)
+    torch.cuda.synchronize()
+    O_o, lse_o = oracle.forward(q, k, v, idx.cpu().numpy(), H, W, 8, (4, 4))
+    check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
+def test_status_word_reads_ok():
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
