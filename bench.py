@@ -1,0 +1,443 @@
+#!/usr/bin/env python3
+"""Benchmark of the SSBA forward (mask build + block-sparse attention) on GB300.
+
+A step is one pass of the whole hot path over one batch: the 24 SSBA layers of the
+1024 px DiT (64 x 64 image tokens, B=1, 24 heads x 64, rho = 0.8416 -> keep 11 of 64
+blocks per query block), layer l with window shift (0,0) if l is even else (4,4); each
+layer builds its mask from its own Q/K and then runs the block-sparse forward. Each
+layer has its own seeded synthetic Q/K/V (906 MB in all), so every layer's inputs are
+cold in L2 when it runs.
+
+Prints one JSON line. value = effective TFLOP/s counting only the kept blocks
+(4 * B * heads * Tb * keep * 64 * 64 * head_dim per layer) over the whole step.
+``--impl reference`` times the CPU oracle on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "SSBA fwd latency (ms) and effective TFLOP/s @4096 tok, 84% sparse, bf16"
+ATTN_SOURCES = ("paper_2605_15684_gb300/csrc/attn_tc.cu", "paper_2605_15684_gb300/csrc/ptx.cuh")
+ATTN_PROFILE = os.path.join(ROOT, "profiles", "ssba_attn_tc_kernel_1024px.md")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--layers", type=int, default=24)
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------------------- workload
+def workload():
+    from paper_2605_15684_gb300 import synthetic
+    return synthetic.PX1024
+
+
+def layer_shift(l: int):
+    return (0, 0) if l % 2 == 0 else (4, 4)
+
+
+def kept_flops(B, h, Tb, keep, d, blk=8):
+    """QK^T plus PV over the kept blocks only (2 * 2 * rows * keys * d)."""
+    return 4.0 * B * h * Tb * keep * (blk * blk) * (blk * blk) * d
+
+
+def config_dict(w, keep, layers):
+    Tb = w.N // 64
+    return {
+        "workload": f"{w.name} x{layers} layers, shifts (0,0)/(4,4) alternating, mask rebuilt per layer",
+        "B": w.B, "heads": w.heads, "grid": [w.H_tok, w.W_tok], "N": w.N, "head_dim": w.head_dim,
+        "block": 8, "rho": w.rho, "Tb": Tb, "keep": keep,
+        "realized_sparsity": round((Tb - keep) / Tb, 6), "layers": layers,
+        "l2": "inputs larger than L2: each layer has its own Q/K/V, "
+              f"{layers * 3 * w.B * w.heads * w.N * w.head_dim * 2 / 1e6:.0f} MB per step",
+    }
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampled every 50 ms in a background process; samples are stamped with
+    the host clock on arrival so the timed window can be selected afterwards."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str | None):
+        self.samples = []
+        self.proc = None
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50"]
+        if gpu_id:
+            cmd += ["-i", gpu_id]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.strip().split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                self.samples.append((time.time(), float(parts[0]), float(parts[1]), parts[2], parts[3:]))
+            except ValueError:
+                continue
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        win = [s for s in self.samples if t0 <= s[0] <= t1] or self.samples
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = set()
+        for s in win:
+            for nm, flag in zip(names, s[4][1:]):
+                if flag.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(s[1] for s in win), "sm_max_mhz": max(s[2] for s in win),
+                "reasons": sorted(reasons), "samples": len(win),
+                "power_w_max": max((float(s[3]) for s in win if s[3].replace(".", "", 1).isdigit()),
+                                   default=None)}
+
+
+# ----------------------------------------------------------------------------- roofline helpers
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return j.get("hbm_gbs", 6800.0), j.get("bf16_tflops", 1900.0), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+def profiled_traffic():
+    """DRAM bytes per launch of the attention kernel from the committed ncu summary, if
+    the kernel source is unchanged since the capture (else None)."""
+    if not os.path.exists(ATTN_PROFILE):
+        return None
+    text = open(ATTN_PROFILE).read()
+    m_b = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
+    m_h = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
+    if not m_b or not m_h:
+        return None
+    h = hashlib.sha256()
+    for rel in ATTN_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return int(m_b.group(1)) if h.hexdigest() == m_h.group(1) else None
+
+
+# ----------------------------------------------------------------------------- reference arm
+def oracle_sample(w, heads_sample: int, seed: int = 0):
+    """Times the fp64 CPU oracle (mask + forward) on `heads_sample` heads of one layer."""
+    import oracle
+    from paper_2605_15684_gb300 import synthetic
+    q, k, v = synthetic.qkv(1, heads_sample, w.N, w.head_dim, w.dtype, seed, w.std)
+    Qd, Kd, Vd = (oracle._f64(x) for x in (q, k, v))
+    shift = layer_shift(0)
+    t0 = time.perf_counter()
+    idx, _ = oracle.build_mask(Qd, Kd, w.H_tok, w.W_tok, 8, shift, w.rho)
+    oracle.forward(Qd, Kd, Vd, idx, w.H_tok, w.W_tok, 8, shift)
+    dt = time.perf_counter() - t0
+    Tb = w.N // 64
+    keep = idx.shape[-1]
+    return kept_flops(1, heads_sample, Tb, keep, w.head_dim) / dt / 1e12, dt
+
+
+def run_reference(args, rank):
+    if rank != 0:
+        return
+    import oracle
+    w = workload()
+    threads = oracle.max_threads()
+    heads_sample = max(1, min(w.heads, threads))
+    Tb = w.N // 64
+    keep = oracle.keep_count(Tb, w.rho)
+    for _ in range(args.warmup):
+        oracle_sample(w, heads_sample)
+    rates, times = [], []
+    for s in range(args.steps):
+        r, dt = oracle_sample(w, heads_sample, seed=s)
+        rates.append(r)
+        times.append(dt)
+    total_flops = kept_flops(1, heads_sample, Tb, keep, w.head_dim) * args.steps
+    value = total_flops / sum(times) / 1e12
+    sample = (f"{heads_sample} of {w.heads} heads of layer 0 per step (mask + forward), "
+              f"OpenMP over heads")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_dict(w, keep, args.layers),
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": min(threads, heads_sample),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- our arm
+def run_ours(args, rank, world):
+    import torch
+    from paper_2605_15684_gb300 import api, build, synthetic
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    torch.cuda.set_device(dev)
+    if rank == 0 or world == 1:
+        build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    api.load_library()
+    w = workload()
+    L = args.layers
+    Tb = w.N // 64
+    descs = [api.SsbaDesc(w.B, w.heads, w.H_tok, w.W_tok, w.head_dim, 8, *layer_shift(l), w.rho, w.dtype)
+             for l in range(L)]
+    keep = api.keep_count(descs[0])
+    shp = (w.B, w.heads, w.N, w.head_dim)
+
+    # per-layer inputs: seed = layer + 1000 * rank (independent problems per rank)
+    host_qkv = [synthetic.qkv(w.B, w.heads, w.N, w.head_dim, w.dtype, seed=l + 1000 * rank, std=w.std)
+                for l in range(L)]
+    Qs = [h[0].to(dev) for h in host_qkv]
+    Ks = [h[1].to(dev) for h in host_qkv]
+    Vs = [h[2].to(dev) for h in host_qkv]
+    idx = [torch.empty((w.B, w.heads, Tb, keep), dtype=torch.int32, device=dev) for _ in range(L)]
+    cnt = [torch.empty((w.B, w.heads, Tb), dtype=torch.int32, device=dev) for _ in range(L)]
+    Os = [torch.empty(shp, dtype=w.dtype, device=dev) for _ in range(L)]
+    lses = [torch.empty(shp[:3], dtype=torch.float32, device=dev) for _ in range(L)]
+    ws = torch.empty(api.mask_workspace_bytes(descs[0]), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    layers = [api.BoundLayer(descs[l], Qs[l], Ks[l], Vs[l], idx[l], cnt[l], Os[l], lses[l], ws, stream)
+              for l in range(L)]
+
+    def step(ev=None):
+        for l, ly in enumerate(layers):
+            if ev is not None:
+                ev[0][l].record(stream)
+            ly.mask()
+            if ev is not None:
+                ev[1][l].record(stream)
+            ly.attend()
+            if ev is not None:
+                ev[2][l].record(stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    st = torch.zeros(1, dtype=torch.int32)
+    st[0] = api.get_status()
+    if int(st[0]) != api.SSBA_OK:
+        raise RuntimeError(f"device status {int(st[0])} after warm-up")
+
+    # ---- timed region: K steps, per-kernel events on the launching stream
+    K = args.steps
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(L)] for _ in range(3)] for _ in range(K)]
+    gpu_id = None
+    try:
+        gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
+        gpu_id = gpu_id if gpu_id.startswith("GPU-") else "GPU-" + gpu_id
+    except Exception:
+        gpu_id = None
+    clocks = ClockSampler(gpu_id)
+    time.sleep(0.3)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    wall0 = time.time()
+    t_start.record(stream)
+    for s in range(K):
+        step(evs[s])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    wall1 = time.time()
+    if world > 1:
+        torch.distributed.barrier()
+    time.sleep(0.1)
+    clocks.stop()
+    ms_total = t_start.elapsed_time(t_end)
+    if world > 1:
+        tt = torch.tensor([ms_total], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms_total = float(tt.item())
+    ms_step = ms_total / K
+    mask_ms = statistics.mean(evs[s][0][l].elapsed_time(evs[s][1][l]) for s in range(K) for l in range(L))
+    attn_ms = statistics.mean(evs[s][1][l].elapsed_time(evs[s][2][l]) for s in range(K) for l in range(L))
+    st[0] = api.get_status()
+    if int(st[0]) != api.SSBA_OK:
+        raise RuntimeError(f"device status {int(st[0])} after the timed region")
+
+    F_layer = kept_flops(w.B, w.heads, Tb, keep, w.head_dim)
+    value = world * L * F_layer / (ms_step * 1e-3) / 1e12
+
+    # ---- roofline of the dominant kernel (the attention kernel)
+    hbm_gbs, bf16_tflops, peak_src = measured_peaks()
+    attn_tflops = F_layer / (attn_ms * 1e-3) / 1e12
+    attn_bytes = 4 * w.B * w.heads * w.N * w.head_dim * 2 + w.B * w.heads * w.N * 4
+    traffic = profiled_traffic()
+    roofline = {"kernel": "ssba_attn_tc_kernel", "bound": "tensor", "achieved": attn_tflops,
+                "peak": bf16_tflops, "unit": "TFLOP/s", "frac": attn_tflops / bf16_tflops,
+                "traffic": traffic, "algorithmic_bytes": attn_bytes,
+                "algorithmic_flops": F_layer, "avg_launch_ms": attn_ms,
+                "peak_source": f"{peak_src} dense bf16 (burst)",
+                "hbm_frac": attn_bytes / (attn_ms * 1e-3) / 1e9 / hbm_gbs}
+    mask_bytes = 2 * w.B * w.heads * w.N * w.head_dim * 2 + w.B * w.heads * Tb * (keep + 1) * 4
+    mask_roof = {"kernels": "ssba_pool_kernel + ssba_select_kernel", "bound": "hbm",
+                 "achieved": mask_bytes / (mask_ms * 1e-3) / 1e9, "peak": hbm_gbs, "unit": "GB/s",
+                 "frac": mask_bytes / (mask_ms * 1e-3) / 1e9 / hbm_gbs, "algorithmic_bytes": mask_bytes,
+                 "avg_call_ms": mask_ms}
+
+    # ---- dense attention from the same build, same shape (outside the timed region)
+    dense_ms = None
+    try:
+        Od = torch.empty(shp, dtype=w.dtype, device=dev)
+        ld = torch.empty(shp[:3], dtype=torch.float32, device=dev)
+        for _ in range(3):
+            api.forward_dense(descs[0], Qs[0], Ks[0], Vs[0], Od, ld)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 20
+        e0.record(stream)
+        for r in range(reps):
+            api.forward_dense(descs[r % 2], Qs[r % L], Ks[r % L], Vs[r % L], Od, ld)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        dense_ms = e0.elapsed_time(e1) / reps
+    except Exception as exc:  # reported, not fatal
+        dense_ms = f"failed: {exc}"
+
+    # ---- end to end through the public API with host buffers (pinned), copies timed
+    e2e = None
+    if args.e2e_steps > 0:
+        pin = [[t.pin_memory() for t in h] for h in host_qkv]
+        O_h = [torch.empty(shp, dtype=w.dtype).pin_memory() for _ in range(L)]
+        l_h = [torch.empty(shp[:3], dtype=torch.float32).pin_memory() for _ in range(L)]
+        h2d_s = torch.cuda.Stream(device=dev)
+        d2h_s = torch.cuda.Stream(device=dev)
+        h2d_done = [torch.cuda.Event() for _ in range(L)]
+        comp_done = [torch.cuda.Event() for _ in range(L)]
+        d2h_done = [torch.cuda.Event() for _ in range(L)]
+
+        def e2e_step():
+            for l in range(L):
+                h2d_s.wait_event(comp_done[l])  # previous step's layer l no longer reads its inputs
+                with torch.cuda.stream(h2d_s):
+                    Qs[l].copy_(pin[l][0], non_blocking=True)
+                    Ks[l].copy_(pin[l][1], non_blocking=True)
+                    Vs[l].copy_(pin[l][2], non_blocking=True)
+                h2d_done[l].record(h2d_s)
+            for l, ly in enumerate(layers):
+                stream.wait_event(h2d_done[l])
+                stream.wait_event(d2h_done[l])  # previous step's read-back of O[l] finished
+                ly.mask()
+                ly.attend()
+                comp_done[l].record(stream)
+                d2h_s.wait_event(comp_done[l])
+                with torch.cuda.stream(d2h_s):
+                    O_h[l].copy_(Os[l], non_blocking=True)
+                    l_h[l].copy_(lses[l], non_blocking=True)
+                d2h_done[l].record(d2h_s)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        torch.cuda.synchronize()
+        e2e_s = (time.perf_counter() - t0) / args.e2e_steps
+        if world > 1:
+            tt = torch.tensor([e2e_s], device=dev)
+            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+            e2e_s = float(tt.item())
+        h2d = L * 3 * w.B * w.heads * w.N * w.head_dim * 2
+        d2h = L * (w.B * w.heads * w.N * w.head_dim * 2 + w.B * w.heads * w.N * 4)
+        e2e = {"value": world * L * F_layer / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "steps": args.e2e_steps,
+               "how": "pinned host Q/K/V -> device on a copy stream, mask + forward, O and lse -> "
+                      "pinned host on a second copy stream; host wall clock around the steps"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        threads = oracle.max_threads()
+        heads_sample = max(1, min(w.heads, threads))
+        rate, dt = oracle_sample(w, heads_sample)
+        cpu = {"value": rate, "unit": "TFLOP/s", "cores": min(threads, heads_sample), "kind": "oracle",
+               "sample": f"{heads_sample} of {w.heads} heads of one layer (mask + forward), {dt:.2f} s, "
+                         f"fp64 C with OpenMP over heads"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": K,
+            "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": dict(config_dict(w, keep, L), parallelism="replicas" if world > 1 else "single GPU"),
+            "latency_ms_per_layer": ms_step / L,
+            "attention_ms_per_layer": attn_ms, "mask_ms_per_layer": mask_ms,
+            "roofline": roofline, "roofline_mask": mask_roof,
+            "dense_attention_ms_per_layer": dense_ms,
+            "speedup_vs_dense": (dense_ms / attn_ms) if isinstance(dense_ms, float) else None,
+            "ideal_speedup_vs_dense": Tb / keep,
+            "e2e": e2e, "cpu_baseline": cpu,
+            "gpu_launches": K * L * 3,
+            "clocks": clocks.summary(wall0, wall1),
+        }
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank)
+        return
+    if world > 1:
+        import torch
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        torch.distributed.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world)
+    finally:
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

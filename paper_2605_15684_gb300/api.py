@@ -237,3 +237,41 @@ def get_status() -> int:
 def realized_sparsity(desc: SsbaDesc) -> float:
     """k_drop / Tb with k_drop = floor(Tb * rho) (host arithmetic, no device call)."""
     return math.floor(desc.Tb * desc.rho) / desc.Tb
+
+
+class BoundLayer:
+    """One SSBA layer with its buffers validated once; ``mask()`` and ``attend()`` then
+    make the bare C calls (ssba_build_mask, ssba_forward) with no per-call checks, so
+    that host overhead stays far below the kernels' run time in tight loops."""
+
+    def __init__(self, desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O, lse, workspace, stream=None):
+        lib = load_library()
+        self._lib = lib
+        self._d = desc.c()
+        keep = keep_count(desc)
+        shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+        for t, n in ((Q, "Q"), (K, "K"), (V, "V"), (O, "O")):
+            _check(t, n, shp, desc.dtype)
+        _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+        _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+        _check(lse, "lse", shp[:3], torch.float32)
+        need = mask_workspace_bytes(desc)
+        if workspace.numel() * workspace.element_size() < need:
+            raise SsbaError(SSBA_ERR_WORKSPACE, f"workspace needs {need} bytes")
+        self.tensors = (Q, K, V, kv_idx, kv_cnt, O, lse, workspace)  # keep alive
+        st = _stream_ptr(stream)
+        self._mask_args = (ctypes.byref(self._d), Q.data_ptr(), K.data_ptr(), kv_idx.data_ptr(),
+                           kv_cnt.data_ptr(), None, workspace.data_ptr(),
+                           workspace.numel() * workspace.element_size(), st)
+        self._fwd_args = (ctypes.byref(self._d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), kv_idx.data_ptr(),
+                          kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), st)
+
+    def mask(self) -> None:
+        rc = self._lib.ssba_build_mask(*self._mask_args)
+        if rc:
+            _raise_on(rc)
+
+    def attend(self) -> None:
+        rc = self._lib.ssba_forward(*self._fwd_args)
+        if rc:
+            _raise_on(rc)

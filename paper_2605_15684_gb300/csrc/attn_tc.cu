@@ -3,27 +3,34 @@
 // and its MMAs; Algorithm 1 SparseAttention over image tokens).
 //
 // Work item = one query block (64 tokens, an 8x8 window of the shifted grid) of one
-// (batch, head); it visits only the key blocks listed for it. Per CTA (192 threads):
-//   warp 0      TMA producer: for each listed key block, K and V land in a 5-stage
-//               shared-memory ring as four 4x4-token boxes each (box = 64 d x 4 x 4 of a
-//               [B*heads, H, W, d] tensor map, 128-byte swizzle). A half-block shift is a
-//               multiple of 4 tokens, so every shifted 8x8 window is exactly four aligned
-//               4x4 quadrants of the unshifted grid: no gather pass, no out-of-range fill.
+// (batch, head); it visits only the key blocks listed for it. Persistent CTAs, two per
+// SM, 352 threads each, warp-specialised:
+//   warp 0      TMA producer (Q, K). Q of each item and K, V of each listed key block arrive as
+//               8 KB tiles cut from [B*heads, H, W, d] tensor maps (128-byte swizzle): one
+//               8x8-token box when the shifted window does not cross the grid edge, else two
+//               or four boxes. A half-block shift is a multiple of 4 tokens, so a crossing
+//               window splits 4 + 4: no gather pass and no out-of-range fill. Q is
+//               double-buffered; K and V have separate 5-stage rings (a K slot frees when
+//               its QK is done, a V slot when its PV is done).
+//   warp 10     TMA producer of the V ring (warp 0 keeps Q and K), so that two threads
+//               share the per-box issue latency.
 //   warp 1      TMEM owner and MMA issuer (one elected lane):
-//                 S_t = Q K_t^T   tcgen05.mma kind::f16, M=64 N=64, A = Q from TMEM,
-//                                 B = K tile (K-major, SW128) from shared memory
+//                 S_t = Q K_t^T   tcgen05.mma kind::f16, M=64 N=64, A = Q tile and
+//                                 B = K tile from shared memory (K-major, SW128)
 //                 O  += P_t V_t   tcgen05.mma kind::f16, M=64 N=64, A = P from TMEM
 //                                 (written over S_t), B = V tile (MN-major, SW128)
-//               S is double-buffered so QK of block t+2 overlaps the softmax of t+1.
-//   warps 2-5   softmax + epilogue, one TMEM lane quadrant each; the M=64 data path puts
-//               query row r at lane 32*(r/16) + r%16, so two threads share a row (16x32bx2
-//               TMEM loads), each holding 32 of its 64 scores. Online softmax in fp32 with
-//               exp2 in the log2-scaled domain; the running max is only raised when it
-//               grows by more than 2^8 (the O rescale then reads and writes O in TMEM),
-//               which keeps P <= 256 in bf16 and l, O exact up to rounding.
-//               They also stage the next item's Q into TMEM, and write O (bf16) and lse.
-// All mbarrier waits are bounded (globaltimer budget + CTA abort flag); a timeout is
-// reported in the device status word and the CTA drains its async work and exits.
+//               S is triple-buffered: QK of block t+3 is issued right after PV of block t.
+//   warps 2-5   softmax, one TMEM lane quadrant each. The M=64 data path puts tile row r
+//               at lane 32*(r/16) + r%16, so two threads share a row (16x32bx2 TMEM
+//               loads), each holding 32 of its 64 scores. Online softmax in fp32 with exp2
+//               in the log2-scaled domain; the running max is only raised when it grows by
+//               more than 2^8 (then O is rescaled in TMEM), which keeps P <= 256 in bf16.
+//               At the end of an item the row statistics (max, sum) go to shared memory.
+//   warps 6-9   epilogue: O / l in bf16 and lse, overlapping the next item's softmax;
+//               warp 6 also prefetches the tiles of the item two ahead into L2.
+// Tile rows follow the TMA box order of the window (tile_row_pos). All mbarrier waits are bounded (globaltimer budget + CTA abort
+// flag); a timeout is reported in the device status word and the CTA drains its
+// in-flight copies and MMAs before it exits.
 #include <cuda.h>
 #include <cstdio>
 
@@ -39,41 +46,62 @@ using namespace ptx;
 constexpr int kD = 64;
 constexpr int kRows = 64;  // query rows per item = tokens per block
 constexpr int kStages = 5;
-constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColS = 0;    // S/P double buffer: [0,64) and [64,128)
-constexpr uint32_t kColO = 128;  // O accumulator: [128,192)
-constexpr uint32_t kColQ = 192;  // Q double buffer: [192,224) and [224,256)
+constexpr int kSBuf = 3;
+constexpr int kSlotWarps = 11;                // warps of one pipeline (see the role map above)
+constexpr int kSlots = 2;                     // independent pipelines per CTA
+constexpr int kThreads = kSlots * kSlotWarps * 32;
+constexpr uint32_t kSlotCols = 256;           // TMEM columns of one pipeline
+constexpr uint32_t kTmemCols = kSlots * kSlotCols;
+constexpr uint32_t kColS = 0;    // S/P buffers: [0,64), [64,128), [128,192)
+constexpr uint32_t kColO = 192;  // O accumulator: [192,256)
 constexpr uint32_t kTileBytes = kRows * kD * 2;  // 8 KB
-constexpr uint32_t kBoxBytes = 16 * kD * 2;      // 2 KB per 4x4 box
+// Tensor-map box shapes (d x cols x rows) used to cut a shifted 8x8 window out of the grid.
+enum BoxShape { kBox8x8 = 0, kBox8c4r = 1, kBox4c8r = 2, kBox4x4 = 3 };
 constexpr uint64_t kBudgetNs = 2000000000ull;    // 2 s per wait
 constexpr float kRescaleLog2 = 8.0f;
+constexpr int kLabelCap = 256;  // labels staged per producer warp; longer lists are read per block
 
 // QK: M=64 N=64, A (Q) and B (K) K-major. PV: M=64 N=64, A (P) K-major, B (V) MN-major.
 constexpr uint32_t kIdescQK = idesc_bf16_f32(64, 64, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(64, 64, false, true);
 
-struct __align__(1024) SmemLayout {
+struct __align__(1024) SlotSmem {
     uint8_t k[kStages][kTileBytes];
     uint8_t v[kStages][kTileBytes];
-    uint64_t kv_full[kStages];
-    uint64_t kv_empty[kStages];
-    uint64_t s_full[2];
-    uint64_t p_full[2];
+    uint8_t q[2][kTileBytes];
+    float2 stats[2][kRows];  // (max in log2 units, row sum) per item parity
+    uint64_t k_full[kStages];
+    uint64_t k_empty[kStages];
+    uint64_t v_full[kStages];
+    uint64_t v_empty[kStages];
     uint64_t q_full[2];
-    uint64_t pv_done;
+    uint64_t q_empty[2];
+    uint64_t s_full[kSBuf];
+    uint64_t p_full[kSBuf];
+    uint64_t pv_done[kSBuf];
+    uint64_t stats_full[2];
+    uint64_t stats_free[2];
     uint64_t o_full;
     uint64_t o_free;
     uint64_t drain;
+    int32_t labels[2][kLabelCap];  // key-block labels of the current item, per producer warp
+};
+
+struct __align__(1024) SmemLayout {
+    SlotSmem slot[kSlots];
     uint32_t tmem_base;
     int abort_flag;
 };
 
+// Four maps per tensor, one per box shape, over the [B*heads][H][W][d] bf16 view.
+struct TileMaps {
+    CUtensorMap q[4], k[4], v[4];
+};
+
 struct TcParams {
-    const __nv_bfloat16* Q;
     __nv_bfloat16* O;
     float* lse;
-    const int32_t* idx;
+    const int32_t* idx;  // null: dense mode, every block of the head
     const int32_t* cnt;
     Grid g;
     int keep;
@@ -124,131 +152,226 @@ __device__ __forceinline__ int item_nblk(const TcParams& p, int item)
     return p.idx ? min(max(__ldg(p.cnt + item), 0), p.keep) : p.keep;
 }
 
-__global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_constant__ CUtensorMap tmK,
-                                                                    const __grid_constant__ CUtensorMap tmV,
+__device__ __forceinline__ int item_label(const TcParams& p, int item, int t, int Tb)
+{
+    return p.idx ? clamp_label(__ldg(p.idx + (size_t)item * p.keep + t), Tb) : t;
+}
+
+// Origin (row, col) of the shifted 8x8 window `label` in the unshifted grid. With block
+// 8 and a shift that is a multiple of 4, a window either fits (origin <= size - 8) or is
+// split 4 + 4 by the grid edge (origin = size - 4).
+__device__ __forceinline__ void window_origin(const Grid& g, int label, int& r0, int& c0)
+{
+    const int br = label / g.bw, bc = label - br * g.bw;
+    r0 = br * 8 - g.sr;
+    if (r0 < 0) r0 += g.H;
+    c0 = bc * 8 - g.sc;
+    if (c0 < 0) c0 += g.W;
+}
+
+// Loads the 64 tokens of window `label` into an 8 KB tile with as few boxes as the grid
+// edge allows: one 8x8 box; two 8-col x 4-row boxes (split rows); two 4-col x 8-row
+// boxes (split columns); or four 4x4 boxes. The tile row order is set by the shape
+// class and decoded by tile_row_pos(); K and V of one label always share it.
+template <bool kPrefetch>
+__device__ __forceinline__ void window_boxes(const CUtensorMap* m4, uint32_t dst, uint32_t bar, const Grid& g,
+                                             int label, int bh)
+{
+    int r0, c0;
+    window_origin(g, label, r0, c0);
+    const bool wr = r0 + 8 > g.H, wc = c0 + 8 > g.W;
+    auto box = [&](int shape, uint32_t off, int c, int r) {
+        if (kPrefetch) tma_prefetch_l2_4d(&m4[shape], 0, c, r, bh);
+        else tma_load_4d(dst + off, &m4[shape], bar, 0, c, r, bh);
+    };
+    if (!wr && !wc) {
+        box(kBox8x8, 0, c0, r0);
+    } else if (wr && !wc) {
+        box(kBox8c4r, 0, c0, r0);
+        box(kBox8c4r, 4096, c0, 0);
+    } else if (!wr && wc) {
+        box(kBox4c8r, 0, c0, r0);
+        box(kBox4c8r, 4096, 0, r0);
+    } else {
+        box(kBox4x4, 0, c0, r0);
+        box(kBox4x4, 2048, 0, r0);
+        box(kBox4x4, 4096, c0, 0);
+        box(kBox4x4, 6144, 0, 0);
+    }
+}
+
+// Tile row r of window `label` -> in-window position (row-major over the 8x8 window).
+__device__ __forceinline__ int tile_row_pos(const Grid& g, int label, int r)
+{
+    int r0, c0;
+    window_origin(g, label, r0, c0);
+    const bool wr = r0 + 8 > g.H, wc = c0 + 8 > g.W;
+    if (!wc) return r;  // 8-wide rows, row-major (one box or two row halves)
+    if (!wr) {          // two 8x4 column halves
+        const int h = r >> 5, a = (r >> 2) & 7, b = r & 3;
+        return a * 8 + 4 * h + b;
+    }
+    const int q = r >> 4, a = (r >> 2) & 3, b = r & 3;  // four 4x4 quadrants
+    return (4 * (q >> 1) + a) * 8 + 4 * (q & 1) + b;
+}
+
+__global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ TileMaps maps,
                                                                     const TcParams p)
 {
     extern __shared__ uint8_t smem_raw[];
-    SmemLayout& sm = *reinterpret_cast<SmemLayout*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+    SmemLayout& cs = *reinterpret_cast<SmemLayout*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                     ~static_cast<uintptr_t>(1023));
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    volatile int* abortf = &sm.abort_flag;
+    const int gwarp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int slot = gwarp / kSlotWarps;   // which pipeline of this CTA
+    const int warp = gwarp % kSlotWarps;   // role within the pipeline
+    SlotSmem& sm = cs.slot[slot];
+    volatile int* abortf = &cs.abort_flag;
+    // pipeline `slot` of CTA b is virtual CTA 2b + slot of a grid of 2 * gridDim.x
+    const int vcta = blockIdx.x * kSlots + slot;
+    const int vgrid = gridDim.x * kSlots;
     const Grid g = p.g;
     const int Tb = g.Tb();
     const int N = g.H * g.W;
 
-    if (threadIdx.x == 0) {
-        sm.abort_flag = 0;
+    if (threadIdx.x % (kSlotWarps * 32) == 0) {
+        if (slot == 0) cs.abort_flag = 0;
         for (int s = 0; s < kStages; ++s) {
-            mbar_init(smem_u32(&sm.kv_full[s]), 1);
-            mbar_init(smem_u32(&sm.kv_empty[s]), 1);
+            mbar_init(smem_u32(&sm.k_full[s]), 1);
+            mbar_init(smem_u32(&sm.k_empty[s]), 1);
+            mbar_init(smem_u32(&sm.v_full[s]), 1);
+            mbar_init(smem_u32(&sm.v_empty[s]), 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < kSBuf; ++b) {
             mbar_init(smem_u32(&sm.s_full[b]), 1);
             mbar_init(smem_u32(&sm.p_full[b]), 4);
-            mbar_init(smem_u32(&sm.q_full[b]), 4);
+            mbar_init(smem_u32(&sm.pv_done[b]), 1);
         }
-        mbar_init(smem_u32(&sm.pv_done), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&sm.q_full[b]), 1);
+            mbar_init(smem_u32(&sm.q_empty[b]), 1);
+            mbar_init(smem_u32(&sm.stats_full[b]), 4);
+            mbar_init(smem_u32(&sm.stats_free[b]), 4);
+        }
         mbar_init(smem_u32(&sm.o_full), 1);
         mbar_init(smem_u32(&sm.o_free), 4);
         mbar_init(smem_u32(&sm.drain), 1);
         fence_mbar_init();
     }
-    if (warp == 0 && lane == 0) {
-        tma_prefetch_desc(&tmK);
-        tma_prefetch_desc(&tmV);
-    }
-    if (warp == 1) {
-        tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+    if (gwarp == 0 && lane < 12) tma_prefetch_desc(lane < 4 ? &maps.q[lane] : (lane < 8 ? &maps.k[lane - 4] : &maps.v[lane - 8]));
+    if (gwarp == 1) {
+        tmem_alloc(smem_u32(&cs.tmem_base), kTmemCols);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tbase = sm.tmem_base;
+    const uint32_t tbase = cs.tmem_base + slot * kSlotCols;
     bool dead = false;
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ TMA producer
-        const bool leader = elect_one_sync();
-        uint32_t gkv = 0;
-        for (int item = blockIdx.x; item < p.num_items && !dead; item += gridDim.x) {
-            const int bh = item / Tb;
+    if (warp == 0 || warp == 10) {
+        // ------------------------------------------------------------ TMA producers
+        // Warp 0 loads each item's Q tile and the K tiles of its key blocks into the K ring,
+        // warp 10 the V tiles into the V ring; one elected lane each, blocking (suspending)
+        // waits. A K slot frees when its QK is done and a V slot when its PV is done, so the
+        // rings do not wait on each other, and the two issuing threads overlap their TMA
+        // issue latency (about 140 cycles per box per thread).
+        const bool is_k = warp == 0;
+        int32_t* lab = sm.labels[is_k ? 0 : 1];
+        uint32_t g = 0, nq = 0;
+        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nq) {
+            const int bh = item / Tb, label = item - bh * Tb;
             const int nblk = item_nblk(p, item);
             const int32_t* list = p.idx ? p.idx + (size_t)item * p.keep : nullptr;
-            for (int t = 0; t < nblk; ++t, ++gkv) {
-                const uint32_t slot = gkv % kStages, ph = (gkv / kStages) & 1;
-                if (!mbar_wait(smem_u32(&sm.kv_empty[slot]), ph ^ 1, abortf, kBudgetNs)) {
-                    dead = true;
-                    break;
-                }
-                if (leader) {
-                    const int j = list ? clamp_label(__ldg(list + t), Tb) : t;
-                    const int br = j / g.bw, bc = j - br * g.bw;
-                    const uint32_t bar = smem_u32(&sm.kv_full[slot]);
-                    mbar_arrive_expect_tx(bar, 2 * kTileBytes);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        int r0 = br * 8 + (q >> 1) * 4 - g.sr;
-                        if (r0 < 0) r0 += g.H;
-                        int c0 = bc * 8 + (q & 1) * 4 - g.sc;
-                        if (c0 < 0) c0 += g.W;
-                        tma_load_4d(smem_u32(&sm.k[slot][q * kBoxBytes]), &tmK, bar, 0, c0, r0, bh);
-                        tma_load_4d(smem_u32(&sm.v[slot][q * kBoxBytes]), &tmV, bar, 0, c0, r0, bh);
+            // all lanes fetch the item's labels in one round; lane 0 then issues the copies
+            if (list)
+                for (int t = lane; t < nblk && t < kLabelCap; t += 32) lab[t] = clamp_label(__ldg(list + t), Tb);
+            __syncwarp();
+            if (lane == 0) {
+                if (is_k) {
+                    const uint32_t qb = nq & 1;
+                    if (!mbar_wait(smem_u32(&sm.q_empty[qb]), ((nq >> 1) & 1) ^ 1, abortf, kBudgetNs)) dead = true;
+                    if (!dead) {
+                        mbar_arrive_expect_tx(smem_u32(&sm.q_full[qb]), kTileBytes);
+                        window_boxes<false>(maps.q, smem_u32(&sm.q[qb][0]), smem_u32(&sm.q_full[qb]), p.g, label, bh);
                     }
                 }
-                __syncwarp();
+                for (int t = 0; t < nblk && !dead; ++t, ++g) {
+                    const int j = !list ? t : (t < kLabelCap ? lab[t] : clamp_label(__ldg(list + t), Tb));
+                    const uint32_t slot = g % kStages;
+                    uint64_t* empty = is_k ? &sm.k_empty[slot] : &sm.v_empty[slot];
+                    uint64_t* full = is_k ? &sm.k_full[slot] : &sm.v_full[slot];
+                    if (!mbar_wait(smem_u32(empty), ((g / kStages) & 1) ^ 1, abortf, kBudgetNs)) {
+                        dead = true;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(smem_u32(full), kTileBytes);
+                    window_boxes<false>(is_k ? maps.k : maps.v, smem_u32(is_k ? &sm.k[slot][0] : &sm.v[slot][0]),
+                                        smem_u32(full), p.g, j, bh);
+                }
             }
+            dead = __shfl_sync(0xffffffffu, dead, 0);
+            g = __shfl_sync(0xffffffffu, g, 0);
         }
-        if (dead && leader) {
-            // drain: wait for the loads this warp issued that nobody consumed
-            uint32_t first = gkv > (uint32_t)kStages ? gkv - kStages : 0;
-            for (uint32_t x = first; x < gkv; ++x)
-                wait_raw(smem_u32(&sm.kv_full[x % kStages]), (x / kStages) & 1);
+        if (dead && lane == 0) {
+            // drain: wait for the copies this thread issued that may still be in flight
+            for (uint32_t x = g > (uint32_t)kStages ? g - kStages : 0; x < g; ++x)
+                wait_raw(smem_u32(is_k ? &sm.k_full[x % kStages] : &sm.v_full[x % kStages]), (x / kStages) & 1);
+            if (is_k)
+                for (uint32_t n = nq > 1 ? nq - 1 : 0; n <= nq; ++n)
+                    wait_raw(smem_u32(&sm.q_full[n & 1]), (n >> 1) & 1);
         }
+        __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         const bool leader = elect_one_sync();
         uint32_t gblk = 0, nloc = 0;
         const uint32_t kbase = smem_u32(&sm.k[0][0]);
         const uint32_t vbase = smem_u32(&sm.v[0][0]);
-        for (int item = blockIdx.x; item < p.num_items && !dead; item += gridDim.x, ++nloc) {
+        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
             const int nblk = item_nblk(p, item);
-            const uint32_t qcol = tbase + kColQ + (nloc & 1) * 32;
-            if (!mbar_wait(smem_u32(&sm.q_full[nloc & 1]), (nloc >> 1) & 1, abortf, kBudgetNs)) {
+            const uint32_t qb = nloc & 1;
+            const uint32_t qaddr = smem_u32(&sm.q[qb][0]);
+            if (!mbar_wait(smem_u32(&sm.q_full[qb]), (nloc >> 1) & 1, abortf, kBudgetNs)) {
                 dead = true;
                 break;
             }
             tc_fence_after();
-            auto issue_qk = [&](uint32_t gb) -> bool {
-                const uint32_t slot = gb % kStages;
-                if (!mbar_wait(smem_u32(&sm.kv_full[slot]), (gb / kStages) & 1, abortf, kBudgetNs))
-                    return false;
+            auto issue_qk = [&](int t) -> bool {
+                const uint32_t gb = gblk + t, slot = gb % kStages, sb = gb % kSBuf;
+                if (!mbar_wait(smem_u32(&sm.k_full[slot]), (gb / kStages) & 1, abortf, kBudgetNs)) return false;
                 tc_fence_after();
                 if (leader) {
+                    const uint64_t adesc = sdesc_sw128(qaddr, 16, 1024);
                     const uint64_t bdesc = sdesc_sw128(kbase + slot * kTileBytes, 16, 1024);
-                    const uint32_t d = tbase + kColS + (gb & 1) * 64;
+                    const uint32_t d = tbase + kColS + sb * 64;
 #pragma unroll
                     for (int k = 0; k < 4; ++k)
-                        mma_ts(d, qcol + k * 8, bdesc + (uint64_t)(k * 2), kIdescQK, k > 0 ? 1u : 0u);
-                    mma_commit(smem_u32(&sm.s_full[gb & 1]));
+                        mma_ss(d, adesc + (uint64_t)(k * 2), bdesc + (uint64_t)(k * 2), kIdescQK, k > 0 ? 1u : 0u);
+                    mma_commit(smem_u32(&sm.s_full[sb]));
+                    mma_commit(smem_u32(&sm.k_empty[slot]));
+                    if (t == nblk - 1) mma_commit(smem_u32(&sm.q_empty[qb]));  // last read of this Q tile
                 }
                 __syncwarp();
                 return true;
             };
-            for (int t = 0; t < nblk && t < 2; ++t)
-                if (!issue_qk(gblk + t)) {
+            if (nblk == 0 && leader) mma_commit(smem_u32(&sm.q_empty[qb]));
+            for (int t = 0; t < nblk && t < kSBuf; ++t)
+                if (!issue_qk(t)) {
                     dead = true;
                     break;
                 }
             for (int t = 0; t < nblk && !dead; ++t) {
-                const uint32_t gb = gblk + t, sb = gb & 1, slot = gb % kStages;
-                if (!mbar_wait(smem_u32(&sm.p_full[sb]), (gb >> 1) & 1, abortf, kBudgetNs)) {
+                const uint32_t gb = gblk + t, sb = gb % kSBuf, slot = gb % kStages;
+                if (!mbar_wait(smem_u32(&sm.p_full[sb]), (gb / kSBuf) & 1, abortf, kBudgetNs)) {
                     dead = true;
                     break;
                 }
                 if (t == 0 && nloc > 0 &&
                     !mbar_wait(smem_u32(&sm.o_free), (nloc - 1) & 1, abortf, kBudgetNs)) {
+                    dead = true;
+                    break;
+                }
+                if (!mbar_wait(smem_u32(&sm.v_full[slot]), (gb / kStages) & 1, abortf, kBudgetNs)) {
                     dead = true;
                     break;
                 }
@@ -260,11 +383,11 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_
                     for (int k = 0; k < 4; ++k)
                         mma_ts(tbase + kColO, pcol + k * 8, vdesc + (uint64_t)(k * 128), kIdescPV,
                                (t > 0 || k > 0) ? 1u : 0u);
-                    mma_commit(smem_u32(&sm.kv_empty[slot]));
-                    mma_commit(smem_u32(&sm.pv_done));
+                    mma_commit(smem_u32(&sm.v_empty[slot]));
+                    mma_commit(smem_u32(&sm.pv_done[sb]));
                 }
                 __syncwarp();
-                if (t + 2 < nblk && !issue_qk(gb + 2)) {
+                if (t + kSBuf < nblk && !issue_qk(t + kSBuf)) {
                     dead = true;
                     break;
                 }
@@ -284,45 +407,20 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_
             mma_commit(smem_u32(&sm.drain));
             wait_raw(smem_u32(&sm.drain), 0);
         }
-    } else {
-        // ------------------------------------------------------------ softmax + epilogue
-        const int quad = warp & 3;           // TMEM lane quadrant of this warp
-        const int half = lane >> 4;          // which 32 of the row's 64 columns
+    } else if (warp < 6) {
+        // ------------------------------------------------------------ softmax
+        const int quad = gwarp & 3;  // TMEM lane quadrant of this warp
+        const int half = lane >> 4;
         const int row = quad * 16 + (lane & 15);
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
         const float c = p.scale_log2;
         uint32_t gblk = 0, nloc = 0;
-
-        auto stage_q = [&](int item, uint32_t buf) {
-            const int bh = item / Tb, label = item - (item / Tb) * Tb;
-            const int tok = g.token(label, row);
-            const uint4* src = reinterpret_cast<const uint4*>(p.Q + ((size_t)bh * N + tok) * kD + half * 32);
-            uint32_t r[16];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                uint4 v = __ldg(src + i);
-                r[4 * i] = v.x;
-                r[4 * i + 1] = v.y;
-                r[4 * i + 2] = v.z;
-                r[4 * i + 3] = v.w;
-            }
-            tmem_st_16x32bx2_x16_off16(tbase + lane_off + kColQ + buf * 32, r);
-            tmem_wait_st();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&sm.q_full[buf]));
-        };
-
-        if ((int)blockIdx.x < p.num_items) stage_q(blockIdx.x, 0);
-        for (int item = blockIdx.x; item < p.num_items && !dead; item += gridDim.x, ++nloc) {
-            const int bh = item / Tb, label = item - bh * Tb;
+        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
             const int nblk = item_nblk(p, item);
-            if (item + (int)gridDim.x < p.num_items) stage_q(item + gridDim.x, (nloc + 1) & 1);
-
             float m_used = 0.f, l = 0.f;
             for (int t = 0; t < nblk; ++t) {
-                const uint32_t gb = gblk + t, sb = gb & 1;
-                if (!mbar_wait(smem_u32(&sm.s_full[sb]), (gb >> 1) & 1, abortf, kBudgetNs)) {
+                const uint32_t gb = gblk + t, sb = gb % kSBuf;
+                if (!mbar_wait(smem_u32(&sm.s_full[sb]), (gb / kSBuf) & 1, abortf, kBudgetNs)) {
                     dead = true;
                     break;
                 }
@@ -332,9 +430,17 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_
                 tmem_ld_16x32bx2_x16_off32(scol, *reinterpret_cast<uint32_t(*)[16]>(&sr[0]));
                 tmem_ld_16x32bx2_x16_off32(scol + 16, *reinterpret_cast<uint32_t(*)[16]>(&sr[16]));
                 tmem_wait_ld();
-                float mx = __uint_as_float(sr[0]);
+                float mx;
+                {
+                    float t8[8];
 #pragma unroll
-                for (int i = 1; i < 32; ++i) mx = fmaxf(mx, __uint_as_float(sr[i]));
+                    for (int i = 0; i < 8; ++i)
+                        t8[i] = fmaxf(fmaxf(__uint_as_float(sr[i]), __uint_as_float(sr[i + 8])),
+                                      fmaxf(__uint_as_float(sr[i + 16]), __uint_as_float(sr[i + 24])));
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) t8[i] = fmaxf(t8[i], t8[i + 4]);
+                    mx = fmaxf(fmaxf(t8[0], t8[1]), fmaxf(t8[2], t8[3]));
+                }
                 mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
                 const float mx2 = mx * c;
                 if (t == 0) {
@@ -343,7 +449,8 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_
                     const bool need = mx2 > m_used + kRescaleLog2;
                     if (__any_sync(0xffffffffu, need)) {
                         // O must hold every earlier PV before it is rescaled
-                        if (!mbar_wait(smem_u32(&sm.pv_done), (gb - 1) & 1, abortf, kBudgetNs)) {
+                        const uint32_t pb = (gb - 1) % kSBuf;
+                        if (!mbar_wait(smem_u32(&sm.pv_done[pb]), ((gb - 1) / kSBuf) & 1, abortf, kBudgetNs)) {
                             dead = true;
                             break;
                         }
@@ -367,15 +474,15 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_
                     }
                 }
                 uint32_t pk[16];
-                float ls = 0.f;
+                float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int i = 0; i < 16; ++i) {
                     const float p0 = fast_exp2(fmaf(__uint_as_float(sr[2 * i]), c, -m_used));
                     const float p1 = fast_exp2(fmaf(__uint_as_float(sr[2 * i + 1]), c, -m_used));
-                    ls += p0 + p1;
+                    ls[i & 3] += p0 + p1;
                     pk[i] = pack_bf16(p0, p1);
                 }
-                l += ls;
+                l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
                 tmem_st_16x32bx2_x16_off16(tbase + lane_off + kColS + sb * 64, pk);
                 tmem_wait_st();
                 tc_fence_before();
@@ -383,9 +490,28 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_
                 if (lane == 0) mbar_arrive(smem_u32(&sm.p_full[sb]));
             }
             if (dead) break;
-
-            // ---- epilogue: O / l in bf16, lse = ln(sum exp(scale * s))
+            // hand the row statistics to the epilogue warps
             const float ltot = l + __shfl_xor_sync(0xffffffffu, l, 16);
+            const uint32_t eb = nloc & 1;
+            if (!mbar_wait(smem_u32(&sm.stats_free[eb]), ((nloc >> 1) & 1) ^ 1, abortf, kBudgetNs)) {
+                dead = true;
+                break;
+            }
+            if (half == 0) sm.stats[eb][row] = make_float2(m_used, ltot);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&sm.stats_full[eb]));
+            gblk += nblk;
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int quad = gwarp & 3;
+        const int half = lane >> 4;
+        const int row = quad * 16 + (lane & 15);
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        uint32_t nloc = 0;
+        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
+            const int bh = item / Tb, label = item - bh * Tb;
+            const uint32_t eb = nloc & 1;
             if (!mbar_wait(smem_u32(&sm.o_full), nloc & 1, abortf, kBudgetNs)) {
                 dead = true;
                 break;
@@ -398,23 +524,44 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&sm.o_free));
+            if (!mbar_wait(smem_u32(&sm.stats_full[eb]), (nloc >> 1) & 1, abortf, kBudgetNs)) {
+                dead = true;
+                break;
+            }
+            const float2 st = sm.stats[eb][row];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&sm.stats_free[eb]));
 
-            const bool ok = ltot > 0.f;
-            const float inv = ok ? 1.f / ltot : 0.f;
-            const int tok = g.token(label, row);
+            const bool ok = st.y > 0.f;
+            const float inv = ok ? 1.f / st.y : 0.f;
+            const int tok = g.token(label, tile_row_pos(g, label, row));
             uint4* dst = reinterpret_cast<uint4*>(p.O + ((size_t)bh * N + tok) * kD + half * 32);
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
+                float f[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) f[e] = ok ? __uint_as_float(o[8 * i + e]) * inv : 0.f;
                 uint4 v;
-                v.x = pack_bf16(ok ? __uint_as_float(o[8 * i + 0]) * inv : 0.f, ok ? __uint_as_float(o[8 * i + 1]) * inv : 0.f);
-                v.y = pack_bf16(ok ? __uint_as_float(o[8 * i + 2]) * inv : 0.f, ok ? __uint_as_float(o[8 * i + 3]) * inv : 0.f);
-                v.z = pack_bf16(ok ? __uint_as_float(o[8 * i + 4]) * inv : 0.f, ok ? __uint_as_float(o[8 * i + 5]) * inv : 0.f);
-                v.w = pack_bf16(ok ? __uint_as_float(o[8 * i + 6]) * inv : 0.f, ok ? __uint_as_float(o[8 * i + 7]) * inv : 0.f);
+                v.x = pack_bf16(f[0], f[1]);
+                v.y = pack_bf16(f[2], f[3]);
+                v.z = pack_bf16(f[4], f[5]);
+                v.w = pack_bf16(f[6], f[7]);
                 dst[i] = v;
             }
             if (half == 0)
-                p.lse[(size_t)bh * N + tok] = ok ? (m_used * 0.69314718055994531f + logf(ltot)) : -INFINITY;
-            gblk += nblk;
+                p.lse[(size_t)bh * N + tok] = ok ? (st.x * 0.69314718055994531f + logf(st.y)) : -INFINITY;
+            // warm L2 with the tiles of the item two ahead (one lane per key block)
+            const int nxt = item + 2 * vgrid;
+            if (warp == 6 && nxt < p.num_items) {
+                const int nbh = nxt / Tb, nlabel = nxt - nbh * Tb;
+                if (lane == 0) window_boxes<true>(maps.q, 0, 0, g, nlabel, nbh);
+                const int nn = item_nblk(p, nxt);
+                for (int t = lane; t < nn; t += 32) {
+                    const int j = item_label(p, nxt, t, Tb);
+                    window_boxes<true>(maps.k, 0, 0, g, j, nbh);
+                    window_boxes<true>(maps.v, 0, 0, g, j, nbh);
+                }
+            }
         }
     }
 
@@ -422,7 +569,7 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_attn_tc_kernel(const __grid_
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tbase, kTmemCols);
+    if (gwarp == 1) tmem_dealloc(cs.tmem_base, kTmemCols);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -443,19 +590,24 @@ EncodeTiledFn get_encode_fn()
     return fn;
 }
 
-// [B*heads][H][W][d] bf16 viewed as a 4-D tensor map with a 64 x 4 x 4 x 1 box.
-bool encode_qtile_map(CUtensorMap* m, const void* base, int BH, int H, int W)
+// [B*heads][H][W][d] bf16 viewed as 4-D tensor maps, one per box shape (BoxShape order:
+// 8x8, 8 cols x 4 rows, 4 cols x 8 rows, 4x4), 128-byte swizzle.
+bool encode_window_maps(CUtensorMap* m4, const void* base, int BH, int H, int W)
 {
     EncodeTiledFn fn = get_encode_fn();
     if (!fn) return false;
-    cuuint64_t dims[4] = {(cuuint64_t)kD, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)BH};
-    cuuint64_t strides[3] = {(cuuint64_t)kD * 2, (cuuint64_t)W * kD * 2, (cuuint64_t)H * W * kD * 2};
-    cuuint32_t box[4] = {kD, 4, 4, 1};
-    cuuint32_t es[4] = {1, 1, 1, 1};
-    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
+    const cuuint32_t cols[4] = {8, 8, 4, 4}, rows[4] = {8, 4, 8, 4};
+    for (int s = 0; s < 4; ++s) {
+        cuuint64_t dims[4] = {(cuuint64_t)kD, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)BH};
+        cuuint64_t strides[3] = {(cuuint64_t)kD * 2, (cuuint64_t)W * kD * 2, (cuuint64_t)H * W * kD * 2};
+        cuuint32_t box[4] = {kD, cols[s], rows[s], 1};
+        cuuint32_t es[4] = {1, 1, 1, 1};
+        CUresult r = fn(&m4[s], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return false;
+    }
+    return true;
 }
 
 int num_sms()
@@ -481,13 +633,13 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
         return SSBA_ERR_UNSUPPORTED;
     }
     const int BH = d.B * d.heads;
-    CUtensorMap tmK, tmV;
-    if (!encode_qtile_map(&tmK, K, BH, g.H, g.W) || !encode_qtile_map(&tmV, V, BH, g.H, g.W)) {
+    TileMaps maps;
+    if (!encode_window_maps(maps.q, Q, BH, g.H, g.W) || !encode_window_maps(maps.k, K, BH, g.H, g.W) ||
+        !encode_window_maps(maps.v, V, BH, g.H, g.W)) {
         set_error("ssba_forward (bf16): cuTensorMapEncodeTiled failed");
         return SSBA_ERR_CUDA;
     }
     TcParams p;
-    p.Q = static_cast<const __nv_bfloat16*>(Q);
     p.O = static_cast<__nv_bfloat16*>(O);
     p.lse = lse;
     p.idx = idx;
@@ -505,10 +657,15 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
     static bool attr_set = false;
     if (!attr_set) {
         cudaFuncSetAttribute(ssba_attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(ssba_attn_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
         attr_set = true;
     }
-    const int grid = p.num_items < 2 * num_sms() ? p.num_items : 2 * num_sms();
-    ssba_attn_tc_kernel<<<grid, kThreads, smem, st>>>(tmK, tmV, p);
+    // A kernel that uses tensor memory gets one CTA per SM, so each CTA runs kSlots
+    // pipelines; the persistent grid has one CTA per SM (fewer for small problems).
+    const int want = (p.num_items + kSlots - 1) / kSlots;
+    const int grid = want < num_sms() ? want : num_sms();
+    ssba_attn_tc_kernel<<<grid, kThreads, smem, st>>>(maps, p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
         set_error("ssba_attn_tc_kernel launch: %s", cudaGetErrorString(e));

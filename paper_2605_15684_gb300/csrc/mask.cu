@@ -1,16 +1,16 @@
 // mask.cu -- block compression, affinity and Top-k gating (Sec. 2.2; Algorithm 1,
 // partition .. Top-k Smallest) as two HBM-friendly kernels:
 //
-//   ssba_pool_kernel    one CTA per (batch*head, block): gathers the block's 64
-//                       shifted tokens of Q and K with 16-byte loads, and writes the
-//                       fp32 block means q_b, k_b (Eq. for q_b/k_b) to the workspace.
-//                       Dominant cost: reading Q and K once (algorithmic bytes
-//                       2 * B * heads * N * head_dim * elem).
+//   ssba_pool_kernel    one CTA per (batch*head, block): gathers the block's 64 shifted
+//                       tokens of Q and K with 16-byte loads, and writes the fp32 block
+//                       means q_b, k_b (Eq. for q_b/k_b) to the workspace. Dominant cost:
+//                       reading Q and K once (algorithmic bytes 2 * B * heads * N *
+//                       head_dim * elem); HBM-bound.
 //   ssba_select_kernel  one warp per query block: S row = q_b[i] . k_b[j] for all j in
-//                       fp32, then an exact radix select of the `keep` largest entries
-//                       under the total order (S descending, label ascending), i.e. the
-//                       k_drop smallest are dropped and ties keep the lower label; the
-//                       kept labels are written in ascending order.
+//                       fp32, then an exact selection of the `keep` largest entries under
+//                       the total order (S descending, label ascending), i.e. the k_drop
+//                       smallest are dropped and ties keep the lower label; the kept labels
+//                       are written in ascending order.
 #include <cstdio>
 
 #include "common.cuh"
@@ -19,7 +19,6 @@ namespace ssba {
 
 namespace {
 
-constexpr int kPoolThreads = 128;
 
 template <typename T>
 struct Vec;
@@ -49,13 +48,65 @@ struct Vec<float> {
     }
 };
 
-// smem: tokens of the block staged in fp32, [2 tensors][blk*blk][d]; column sums are
-// then taken in in-block position order (a deterministic order).
+// One CTA per (batch*head, block) for head_dim = 64, 256 threads: warp w reads tensor
+// (w / 4 ? K : Q), rows [16 * (w % 4), +16) of the block. Lane l covers 16-byte chunk
+// (l % 8) of rows l/8 + 4i, i < 4: four independent 16-byte loads per lane, so the whole
+// block is requested in one round. Partial sums are combined in a fixed order (lanes by
+// shuffles, warps through shared memory), then the block means are written.
 template <typename T>
-__global__ void __launch_bounds__(kPoolThreads) ssba_pool_kernel(const T* __restrict__ Q,
-                                                                 const T* __restrict__ K, Grid g, int d,
-                                                                 float* __restrict__ qb,
-                                                                 float* __restrict__ kb)
+__global__ void __launch_bounds__(256) ssba_pool_kernel(const T* __restrict__ Q, const T* __restrict__ K, Grid g,
+                                                        float* __restrict__ qb, float* __restrict__ kb)
+{
+    constexpr int kD = 64;
+    constexpr int VE = Vec<T>::kElems;
+    constexpr int CPR = kD / VE;            // 16-byte chunks per token row (8 bf16 / 16 fp32)
+    constexpr int RPI = 32 / CPR;           // rows per warp instruction
+    constexpr int ROWS = 16;                // rows per warp
+    constexpr int LOADS = ROWS / RPI;       // loads per lane
+    __shared__ float part[2][4][kD];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int which = warp >> 2, quarter = warp & 3;
+    const int label = blockIdx.x, bh = blockIdx.y;
+    const int N = g.H * g.W;
+    const T* X = (which ? K : Q) + (size_t)bh * N * kD;
+    const int col = lane % CPR, r0 = lane / CPR;
+    uint4 v[LOADS];
+#pragma unroll
+    for (int i = 0; i < LOADS; ++i) {
+        const int pos = quarter * ROWS + r0 + i * RPI;
+        v[i] = __ldg(reinterpret_cast<const uint4*>(X + (size_t)g.token(label, pos) * kD + col * VE));
+    }
+    float acc[VE];
+#pragma unroll
+    for (int e = 0; e < VE; ++e) acc[e] = 0.f;
+#pragma unroll
+    for (int i = 0; i < LOADS; ++i) {
+        float f[VE];
+        Vec<T>::to_f32(v[i], f);
+#pragma unroll
+        for (int e = 0; e < VE; ++e) acc[e] += f[e];
+    }
+#pragma unroll
+    for (int o = CPR; o < 32; o <<= 1)
+#pragma unroll
+        for (int e = 0; e < VE; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+    if (r0 == 0)
+#pragma unroll
+        for (int e = 0; e < VE; ++e) part[which][quarter][col * VE + e] = acc[e];
+    __syncthreads();
+    if (threadIdx.x < 2 * kD) {
+        const int w = threadIdx.x >> 6, c = threadIdx.x & (kD - 1);
+        const float sum = (part[w][0][c] + part[w][1][c]) + (part[w][2][c] + part[w][3][c]);
+        (w ? kb : qb)[((size_t)bh * g.Tb() + label) * kD + c] = sum * (1.0f / 64.0f);
+    }
+}
+
+// Generic-width fallback (any head_dim multiple of 16 bytes): the block's tokens are
+// staged in fp32 in shared memory and column sums taken in in-block position order.
+template <typename T>
+__global__ void __launch_bounds__(128) ssba_pool_generic_kernel(const T* __restrict__ Q, const T* __restrict__ K,
+                                                                Grid g, int d, float* __restrict__ qb,
+                                                                float* __restrict__ kb)
 {
     extern __shared__ float stage[];  // [2][P][d]
     const int label = blockIdx.x;
@@ -63,40 +114,38 @@ __global__ void __launch_bounds__(kPoolThreads) ssba_pool_kernel(const T* __rest
     const int P = g.blk * g.blk;
     const int N = g.H * g.W;
     constexpr int VE = Vec<T>::kElems;
-    const int cpr = d / VE;  // 16-byte chunks per token row
+    const int cpr = d / VE;
     const int chunks = P * cpr;
     const T* Qh = Q + (size_t)bh * N * d;
     const T* Kh = K + (size_t)bh * N * d;
-
-    for (int ci = threadIdx.x; ci < 2 * chunks; ci += kPoolThreads) {
+    for (int ci = threadIdx.x; ci < 2 * chunks; ci += 128) {
         int which = ci >= chunks;
         int cc = which ? ci - chunks : ci;
-        int pos = cc / cpr, col = cc - pos * cpr;
+        int pos = cc / cpr, c = cc - pos * cpr;
         int tok = g.token(label, pos);
-        const T* src = (which ? Kh : Qh) + (size_t)tok * d + col * VE;
-        uint4 v = __ldg(reinterpret_cast<const uint4*>(src));
+        uint4 v = __ldg(reinterpret_cast<const uint4*>((which ? Kh : Qh) + (size_t)tok * d + c * VE));
         float f[VE];
         Vec<T>::to_f32(v, f);
-        float* dst = stage + ((size_t)which * P + pos) * d + col * VE;
+        float* dst = stage + ((size_t)which * P + pos) * d + c * VE;
 #pragma unroll
         for (int e = 0; e < VE; ++e) dst[e] = f[e];
     }
     __syncthreads();
     const float inv = 1.0f / (float)P;
-    for (int t = threadIdx.x; t < 2 * d; t += kPoolThreads) {
+    for (int t = threadIdx.x; t < 2 * d; t += 128) {
         int which = t >= d;
         int c = which ? t - d : t;
         const float* src = stage + (size_t)which * P * d + c;
         float acc = 0.f;
         for (int pos = 0; pos < P; ++pos) acc += src[(size_t)pos * d];
-        float* out = which ? kb : qb;
-        out[((size_t)bh * g.Tb() + label) * d + c] = acc * inv;
+        (which ? kb : qb)[((size_t)bh * g.Tb() + label) * d + c] = acc * inv;
     }
 }
 
 constexpr int kSelWarps = 8;
 constexpr int kSelKeyChunk = 256;
 constexpr int kMaxTb = 2048;
+constexpr int kRankMaxTb = 256;  // rows up to this length use rank counting, longer ones radix select
 
 __device__ __forceinline__ uint32_t order_key(float s)
 {
@@ -105,7 +154,42 @@ __device__ __forceinline__ uint32_t order_key(float s)
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// smem: kbT [d][kSelKeyChunk] | q rows [kSelWarps][d] | S rows [kSelWarps][Tb]
+// Kept labels of one row by rank counting; lane l owns labels l + 32m, m < kPer.
+template <int kPer>
+__device__ __forceinline__ void rank_select(const uint32_t* S, int Tb, int keep, int lane, int32_t* dst)
+{
+    uint32_t mine[kPer];
+    int rank[kPer];
+#pragma unroll
+    for (int m = 0; m < kPer; ++m) {
+        const int j = lane + 32 * m;
+        mine[m] = j < Tb ? S[j] : 0u;
+        rank[m] = 0;
+    }
+#pragma unroll 8
+    for (int k = 0; k < Tb; ++k) {
+        const uint32_t v = S[k];  // broadcast read
+#pragma unroll
+        for (int m = 0; m < kPer; ++m) rank[m] += (v > mine[m]) || (v == mine[m] && k < lane + 32 * m);
+    }
+    int out = 0;
+#pragma unroll
+    for (int m = 0; m < kPer; ++m) {
+        const int j = lane + 32 * m;
+        const bool kept = j < Tb && rank[m] < keep;
+        const uint32_t km = __ballot_sync(0xffffffffu, kept);
+        if (kept) dst[out + __popc(km & ((1u << lane) - 1u))] = j;
+        out += __popc(km);
+    }
+}
+
+// One warp per query block (row i of S), kSelWarps rows per CTA.
+// smem: kbT [d][kSelKeyChunk + 1] (padded transpose of a key chunk) | q rows [kSelWarps][d]
+//       | S rows as order keys [kSelWarps][Tb]
+// S[i][j] = q_b[i] . k_b[j] in fp32 (FMA over d in order); the row is then reduced to its
+// `keep` largest entries under (S descending, label ascending): rank(j) = #{k : key_k > key_j,
+// or key_k == key_j and k < j} is unique, and j is kept iff rank(j) < keep. Kept labels
+// are written in ascending order.
 __global__ void __launch_bounds__(kSelWarps * 32) ssba_select_kernel(const float* __restrict__ qb,
                                                                      const float* __restrict__ kb, int Tb,
                                                                      int d, int keep,
@@ -114,72 +198,90 @@ __global__ void __launch_bounds__(kSelWarps * 32) ssba_select_kernel(const float
                                                                      float* __restrict__ scores)
 {
     extern __shared__ float sm[];
+    constexpr int kLd = kSelKeyChunk + 1;
     float* kbT = sm;
-    float* qs = kbT + (size_t)d * kSelKeyChunk;
-    float* Srow = qs + (size_t)kSelWarps * d;
+    float* qs = kbT + (size_t)d * kLd;
+    uint32_t* Skey = reinterpret_cast<uint32_t*>(qs + (size_t)kSelWarps * d);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int bh = blockIdx.y;
     const int row = blockIdx.x * kSelWarps + warp;
     const bool active = row < Tb;
     const float* kbh = kb + (size_t)bh * Tb * d;
-    float* S = Srow + (size_t)warp * Tb;
+    uint32_t* S = Skey + (size_t)warp * Tb;
+    const size_t rowoff = (size_t)bh * Tb + row;
 
     if (active)
-        for (int c = lane; c < d; c += 32) qs[warp * d + c] = qb[((size_t)bh * Tb + row) * d + c];
+        for (int c = lane; c < d; c += 32) qs[warp * d + c] = qb[rowoff * d + c];
 
-    // S row in key chunks: kbT holds a transposed chunk so lanes read consecutive keys.
     for (int j0 = 0; j0 < Tb; j0 += kSelKeyChunk) {
         const int nk = min(kSelKeyChunk, Tb - j0);
         __syncthreads();
-        for (int e = threadIdx.x; e < nk * d; e += kSelWarps * 32) {
-            int j = e / d, c = e - j * d;
-            kbT[c * kSelKeyChunk + j] = kbh[(size_t)(j0 + j) * d + c];
+        // float4 loads (d % 4 == 0), unrolled so that each thread's loads are all in flight
+        const float4* src4 = reinterpret_cast<const float4*>(kbh + (size_t)j0 * d);
+        const int n4 = nk * d / 4;
+#pragma unroll 4
+        for (int e4 = threadIdx.x; e4 < n4; e4 += kSelWarps * 32) {
+            const float4 v = __ldg(src4 + e4);
+            const int e = e4 * 4, j = e / d, c = e - j * d;
+            kbT[(c + 0) * kLd + j] = v.x;
+            kbT[(c + 1) * kLd + j] = v.y;
+            kbT[(c + 2) * kLd + j] = v.z;
+            kbT[(c + 3) * kLd + j] = v.w;
         }
         __syncthreads();
         if (active) {
             for (int j = lane; j < nk; j += 32) {
-                float acc = 0.f;
-                for (int c = 0; c < d; ++c) acc = fmaf(qs[warp * d + c], kbT[c * kSelKeyChunk + j], acc);
-                S[j0 + j] = acc;
+                // four interleaved partial sums over d (c = 4t + u), combined in a fixed order
+                float a[4] = {0.f, 0.f, 0.f, 0.f};
+                int c = 0;
+                for (; c + 4 <= d; c += 4)
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) a[u] = fmaf(qs[warp * d + c + u], kbT[(c + u) * kLd + j], a[u]);
+                for (; c < d; ++c) a[0] = fmaf(qs[warp * d + c], kbT[c * kLd + j], a[0]);
+                const float acc = (a[0] + a[1]) + (a[2] + a[3]);
+                if (scores) scores[rowoff * Tb + j0 + j] = acc;
+                S[j0 + j] = order_key(acc);
             }
         }
     }
     __syncwarp();
     if (!active) return;
-
-    const size_t rowoff = (size_t)bh * Tb + row;
-    if (scores)
-        for (int j = lane; j < Tb; j += 32) scores[rowoff * Tb + j] = S[j];
-
-    // keep-th largest key by MSB-first radix select
-    uint32_t prefix = 0, pmask = 0;
-    int remaining = keep;
-    for (int bit = 31; bit >= 0; --bit) {
-        const uint32_t trial = prefix | (1u << bit), tmask = pmask | (1u << bit);
-        int c = 0;
-        for (int j = lane; j < Tb; j += 32) c += (order_key(S[j]) & tmask) == trial;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
-        if (c >= remaining) prefix = trial;
-        else remaining -= c;
-        pmask = tmask;
-    }
-    // kept: key > T, or key == T among the first `remaining` equal ones (lowest labels)
-    const uint32_t T = prefix;
-    int out = 0, eq_seen = 0;
     int32_t* dst = idx + rowoff * keep;
-    for (int j0 = 0; j0 < Tb; j0 += 32) {
-        const int j = j0 + lane;
-        uint32_t key = j < Tb ? order_key(S[j]) : 0u;
-        bool gt = j < Tb && key > T;
-        bool eq = j < Tb && key == T;
-        uint32_t eqm = __ballot_sync(0xffffffffu, eq);
-        int eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
-        bool kept = gt || (eq && eq_rank < remaining);
-        uint32_t km = __ballot_sync(0xffffffffu, kept);
-        if (kept) dst[out + __popc(km & ((1u << lane) - 1u))] = j;
-        out += __popc(km);
-        eq_seen += __popc(eqm);
+
+    if (Tb <= 32) rank_select<1>(S, Tb, keep, lane, dst);
+    else if (Tb <= 64) rank_select<2>(S, Tb, keep, lane, dst);
+    else if (Tb <= 128) rank_select<4>(S, Tb, keep, lane, dst);
+    else if (Tb <= kRankMaxTb) rank_select<8>(S, Tb, keep, lane, dst);
+    else {
+        // keep-th largest key by MSB-first radix select
+        uint32_t prefix = 0, pmask = 0;
+        int remaining = keep;
+        for (int bit = 31; bit >= 0; --bit) {
+            const uint32_t trial = prefix | (1u << bit), tmask = pmask | (1u << bit);
+            int c = 0;
+            for (int j = lane; j < Tb; j += 32) c += (S[j] & tmask) == trial;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+            if (c >= remaining) prefix = trial;
+            else remaining -= c;
+            pmask = tmask;
+        }
+        // kept: key > T, or key == T among the first `remaining` equal ones (lowest labels)
+        const uint32_t T = prefix;
+        int out = 0, eq_seen = 0;
+        for (int j0 = 0; j0 < Tb; j0 += 32) {
+            const int j = j0 + lane;
+            const uint32_t key = j < Tb ? S[j] : 0u;
+            const bool gt = j < Tb && key > T;
+            const bool eq = j < Tb && key == T;
+            const uint32_t eqm = __ballot_sync(0xffffffffu, eq);
+            const int eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
+            const bool kept = gt || (eq && eq_rank < remaining);
+            const uint32_t km = __ballot_sync(0xffffffffu, kept);
+            if (kept) dst[out + __popc(km & ((1u << lane) - 1u))] = j;
+            out += __popc(km);
+            eq_seen += __popc(eqm);
+        }
     }
     if (lane == 0) cnt[rowoff] = keep;
 }
@@ -189,25 +291,37 @@ __global__ void __launch_bounds__(kSelWarps * 32) ssba_select_kernel(const float
 int launch_pool(const ssba_desc& d, const Grid& g, const void* Q, const void* K, float* qb, float* kb,
                 cudaStream_t st)
 {
-    const int P = g.blk * g.blk;
-    size_t smem = (size_t)2 * P * d.head_dim * sizeof(float);
-    dim3 grid(g.Tb(), d.B * d.heads);
-    if (smem > 200 * 1024) {
-        set_error("ssba_build_mask: block*block*head_dim too large for the pooling kernel");
-        return SSBA_ERR_UNSUPPORTED;
-    }
-    if (d.dtype == SSBA_BF16) {
-        auto k = ssba_pool_kernel<__nv_bfloat16>;
-        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        k<<<grid, kPoolThreads, smem, st>>>(static_cast<const __nv_bfloat16*>(Q),
-                                            static_cast<const __nv_bfloat16*>(K), g, d.head_dim, qb, kb);
+    cudaError_t e = cudaSuccess;
+    if (d.head_dim == 64 && g.blk == 8) {
+        dim3 grid(g.Tb(), d.B * d.heads);
+        if (d.dtype == SSBA_BF16)
+            ssba_pool_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(Q),
+                                                                  static_cast<const __nv_bfloat16*>(K), g, qb, kb);
+        else
+            ssba_pool_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float*>(Q), static_cast<const float*>(K),
+                                                          g, qb, kb);
+        e = cudaGetLastError();
     } else {
-        auto k = ssba_pool_kernel<float>;
-        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        k<<<grid, kPoolThreads, smem, st>>>(static_cast<const float*>(Q), static_cast<const float*>(K), g,
-                                            d.head_dim, qb, kb);
+        const int P = g.blk * g.blk;
+        const size_t smem = (size_t)2 * P * d.head_dim * sizeof(float);
+        if (smem > 200 * 1024) {
+            set_error("ssba_build_mask: block*block*head_dim too large for the pooling kernel");
+            return SSBA_ERR_UNSUPPORTED;
+        }
+        dim3 grid(g.Tb(), d.B * d.heads);
+        if (d.dtype == SSBA_BF16) {
+            auto k = ssba_pool_generic_kernel<__nv_bfloat16>;
+            if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            k<<<grid, 128, smem, st>>>(static_cast<const __nv_bfloat16*>(Q), static_cast<const __nv_bfloat16*>(K), g,
+                                       d.head_dim, qb, kb);
+        } else {
+            auto k = ssba_pool_generic_kernel<float>;
+            if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            k<<<grid, 128, smem, st>>>(static_cast<const float*>(Q), static_cast<const float*>(K), g, d.head_dim, qb,
+                                       kb);
+        }
+        e = cudaGetLastError();
     }
-    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
         set_error("ssba_pool_kernel launch: %s", cudaGetErrorString(e));
         return SSBA_ERR_CUDA;
@@ -223,12 +337,14 @@ int launch_select(const ssba_desc& d, const Grid& g, int keep, const float* qb, 
         set_error("ssba_build_mask: Tb=%d exceeds the selection kernel's limit of %d blocks", Tb, kMaxTb);
         return SSBA_ERR_UNSUPPORTED;
     }
-    size_t smem = ((size_t)d.head_dim * kSelKeyChunk + (size_t)kSelWarps * d.head_dim +
+    size_t smem = ((size_t)d.head_dim * (kSelKeyChunk + 1) + (size_t)kSelWarps * d.head_dim +
                    (size_t)kSelWarps * Tb) * sizeof(float);
     if (smem > 220 * 1024) {
         set_error("ssba_build_mask: selection working set too large (%zu bytes)", smem);
         return SSBA_ERR_UNSUPPORTED;
     }
+    cudaFuncSetAttribute(ssba_select_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                         cudaSharedmemCarveoutMaxShared);
     if (smem > 48 * 1024)
         cudaFuncSetAttribute(ssba_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid((Tb + kSelWarps - 1) / kSelWarps, d.B * d.heads);
