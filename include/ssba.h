@@ -128,6 +128,34 @@ SSBA_API int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, c
 SSBA_API int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, const void* V,
                        void* O, float* lse, void* stream);
 
+/* Size of the scratch area built into the library for ssba_build_mask_noalloc (4 MiB). */
+#define SSBA_NOALLOC_SCRATCH_BYTES (4u << 20)
+
+/* ssba_build_mask without a workspace argument: the same kernels and results as
+ * ssba_build_mask, but the scratch (the pooled q_b and k_b) lives in a fixed
+ * SSBA_NOALLOC_SCRATCH_BYTES area inside the library. The paper has no counterpart to this
+ * call. It is for callers that cannot allocate device memory themselves, for example a
+ * plug-in running inside a host runtime that owns all device memory and offers it no
+ * workspace, or a latency-critical loop where a cudaMalloc/cudaFree pair (which can
+ * synchronise the device) is not acceptable.
+ *   Arguments, layouts and outputs are those of ssba_build_mask; the caller still passes
+ *   Q, K and the output buffers.
+ *   Size limit: a layer whose scratch (ssba_mask_workspace_bytes, 2 * B * heads * Tb *
+ *   head_dim * 4 bytes in two 256-byte-aligned halves) exceeds SSBA_NOALLOC_SCRATCH_BYTES is
+ *   rejected with SSBA_ERR_UNSUPPORTED and a message, before any device work. 1024 px and
+ *   2048 px layers with B = 1 and 24 heads of 64 fit.
+ *   Allocation: none. No cudaMalloc, cudaFree or allocating library routine is called; every
+ *   GPU that loads the library holds the scratch area until the process exits.
+ *   Set-up: the first call on each device looks up the area's device address with that
+ *   device current (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   Sharing: every call uses the same area, which keeps the last call's contents. Nothing in
+ *   it needs to start at zero (the pooling kernel writes every value the selection kernel
+ *   reads). Calls that overlap on the GPU -- on two streams, or from two host threads --
+ *   race on the area and must be serialised by the caller. */
+SSBA_API int ssba_build_mask_noalloc(const ssba_desc* desc, const void* Q, const void* K,
+                                     int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt,
+                                     void* stream);
+
 /* Reads and clears the device status word of the current device (SSBA_OK or
  * SSBA_ERR_TIMEOUT). Synchronous: call after the caller's stream sync. Returns
  * SSBA_OK, or SSBA_ERR_CUDA if the read failed. */

@@ -26,8 +26,8 @@ SSBA_BF16, SSBA_FP32 = 0, 1
 _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED", 3: "SSBA_ERR_CUDA",
                  4: "SSBA_ERR_TIMEOUT", 5: "SSBA_ERR_WORKSPACE"}
 
-EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_forward",
-            "ssba_forward_dense", "ssba_get_status", "ssba_last_error")
+EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
+            "ssba_forward", "ssba_forward_dense", "ssba_get_status", "ssba_last_error")
 
 
 class SsbaError(RuntimeError):
@@ -98,6 +98,8 @@ def load_library():
         lib.ssba_mask_workspace_bytes.restype = ctypes.c_size_t
         lib.ssba_build_mask.argtypes = [DP, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_build_mask.restype = ctypes.c_int
+        lib.ssba_build_mask_noalloc.argtypes = [DP, P, P, P, P, P, P]
+        lib.ssba_build_mask_noalloc.restype = ctypes.c_int
         lib.ssba_forward.argtypes = [DP, P, P, P, P, P, P, P, P]
         lib.ssba_forward.restype = ctypes.c_int
         lib.ssba_forward_dense.argtypes = [DP, P, P, P, P, P, P]
@@ -179,6 +181,38 @@ def build_mask(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=None, kv
                              kv_cnt.data_ptr(), S.data_ptr() if S is not None else None,
                              workspace.data_ptr(), workspace.numel() * workspace.element_size(),
                              _stream_ptr(stream))
+    _raise_on(rc)
+    return (kv_idx, kv_cnt, S) if S is not None else (kv_idx, kv_cnt)
+
+
+def build_mask_noalloc(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=None, kv_cnt=None,
+                       scores: bool | torch.Tensor = False, stream=None):
+    """ssba_build_mask_noalloc: build_mask with the library's built-in scratch area (no
+    workspace argument; see include/ssba.h for the size limit and the sharing rule)."""
+    lib = load_library()
+    d = desc.c()
+    keep = lib.ssba_keep_count(ctypes.byref(d))
+    if keep < 0:
+        _raise_on(SSBA_ERR_INVALID)
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    _check(Q, "Q", shp, desc.dtype)
+    _check(K, "K", shp, desc.dtype)
+    dev = Q.device
+    if kv_idx is None:
+        kv_idx = torch.empty((desc.B, desc.heads, desc.Tb, keep), dtype=torch.int32, device=dev)
+    if kv_cnt is None:
+        kv_cnt = torch.empty((desc.B, desc.heads, desc.Tb), dtype=torch.int32, device=dev)
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    S = None
+    if isinstance(scores, torch.Tensor):
+        S = scores
+        _check(S, "scores", (desc.B, desc.heads, desc.Tb, desc.Tb), torch.float32)
+    elif scores:
+        S = torch.empty((desc.B, desc.heads, desc.Tb, desc.Tb), dtype=torch.float32, device=dev)
+    rc = lib.ssba_build_mask_noalloc(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), kv_idx.data_ptr(),
+                                     kv_cnt.data_ptr(), S.data_ptr() if S is not None else None,
+                                     _stream_ptr(stream))
     _raise_on(rc)
     return (kv_idx, kv_cnt, S) if S is not None else (kv_idx, kv_cnt)
 
