@@ -3,8 +3,9 @@
 // and its MMAs; Algorithm 1 SparseAttention over image tokens).
 //
 // Work item = one query block (64 tokens, an 8x8 window of the shifted grid) of one
-// (batch, head); it visits only the key blocks listed for it. Persistent CTAs, two per
-// SM, 352 threads each, warp-specialised:
+// (batch, head); it visits only the key blocks listed for it. Persistent CTAs, one per SM
+// (a kernel that uses tensor memory gets one CTA per SM), each running two independent
+// pipelines of 12 warps (768 threads), warp-specialised:
 //   warp 0      TMA producer (Q, K). Q of each item and K, V of each listed key block arrive as
 //               8 KB tiles cut from [B*heads, H, W, d] tensor maps (128-byte swizzle): one
 //               8x8-token box when the shifted window does not cross the grid edge, else two
@@ -14,20 +15,23 @@
 //               its QK is done, a V slot when its PV is done).
 //   warp 10     TMA producer of the V ring (warp 0 keeps Q and K), so that two threads
 //               share the per-box issue latency.
-//   warp 1      TMEM owner and MMA issuer (one elected lane):
+//   warp 1      QK issuer (one elected lane; warp 1 of the CTA also owns the TMEM allocation):
 //                 S_t = Q K_t^T   tcgen05.mma kind::f16, M=64 N=64, A = Q tile and
 //                                 B = K tile from shared memory (K-major, SW128)
+//               S is triple-buffered: QK of block t waits until PV of block t-3 has read
+//               the P it overwrites.
+//   warp 11     PV issuer (one elected lane):
 //                 O  += P_t V_t   tcgen05.mma kind::f16, M=64 N=64, A = P from TMEM
 //                                 (written over S_t), B = V tile (MN-major, SW128)
-//               S is triple-buffered: QK of block t+3 is issued right after PV of block t.
+//               Two issuing threads keep one's barrier waits (about 100 cycles per query)
+//               off the other's issue path.
 //   warps 2-5   softmax, one TMEM lane quadrant each. The M=64 data path puts tile row r
 //               at lane 32*(r/16) + r%16, so two threads share a row (16x32bx2 TMEM
 //               loads), each holding 32 of its 64 scores. Online softmax in fp32 with exp2
 //               in the log2-scaled domain; the running max is only raised when it grows by
 //               more than 2^8 (then O is rescaled in TMEM), which keeps P <= 256 in bf16.
 //               At the end of an item the row statistics (max, sum) go to shared memory.
-//   warps 6-9   epilogue: O / l in bf16 and lse, overlapping the next item's softmax;
-//               warp 6 also prefetches the tiles of the item two ahead into L2.
+//   warps 6-9   epilogue: O / l in bf16 and lse, overlapping the next item's softmax.
 // Tile rows follow the TMA box order of the window (tile_row_pos). All mbarrier waits are bounded (globaltimer budget + CTA abort
 // flag); a timeout is reported in the device status word and the CTA drains its
 // in-flight copies and MMAs before it exits.
@@ -47,7 +51,7 @@ constexpr int kD = 64;
 constexpr int kRows = 64;  // query rows per item = tokens per block
 constexpr int kStages = 5;
 constexpr int kSBuf = 3;
-constexpr int kSlotWarps = 11;                // warps of one pipeline (see the role map above)
+constexpr int kSlotWarps = 12;                // warps of one pipeline (see the role map above)
 constexpr int kSlots = 2;                     // independent pipelines per CTA
 constexpr int kThreads = kSlots * kSlotWarps * 32;
 constexpr uint32_t kSlotCols = 256;           // TMEM columns of one pipeline
@@ -83,7 +87,7 @@ struct __align__(1024) SlotSmem {
     uint64_t stats_free[2];
     uint64_t o_full;
     uint64_t o_free;
-    uint64_t drain;
+    uint64_t drain[2];
     int32_t labels[2][kLabelCap];  // key-block labels of the current item, per producer warp
 };
 
@@ -254,7 +258,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         }
         mbar_init(smem_u32(&sm.o_full), 1);
         mbar_init(smem_u32(&sm.o_free), 4);
-        mbar_init(smem_u32(&sm.drain), 1);
+        mbar_init(smem_u32(&sm.drain[0]), 1);
+        mbar_init(smem_u32(&sm.drain[1]), 1);
         fence_mbar_init();
     }
     if (gwarp == 0 && lane < 12) tma_prefetch_desc(lane < 4 ? &maps.q[lane] : (lane < 8 ? &maps.k[lane - 4] : &maps.v[lane - 8]));
@@ -322,11 +327,12 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         }
         __syncwarp();
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+        // ------------------------------------------------------------ QK issuer
+        // S_t = Q K_t^T into S buffer t % 3. The buffer still holds P_{t-3} until PV_{t-3}
+        // has finished reading it, so QK_t waits for that PV's completion (pv_done).
         const bool leader = elect_one_sync();
         uint32_t gblk = 0, nloc = 0;
         const uint32_t kbase = smem_u32(&sm.k[0][0]);
-        const uint32_t vbase = smem_u32(&sm.v[0][0]);
         for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
             const int nblk = item_nblk(p, item);
             const uint32_t qb = nloc & 1;
@@ -335,10 +341,18 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 dead = true;
                 break;
             }
-            tc_fence_after();
-            auto issue_qk = [&](int t) -> bool {
+            if (nblk == 0 && leader) mma_commit(smem_u32(&sm.q_empty[qb]));
+            for (int t = 0; t < nblk; ++t) {
                 const uint32_t gb = gblk + t, slot = gb % kStages, sb = gb % kSBuf;
-                if (!mbar_wait(smem_u32(&sm.k_full[slot]), (gb / kStages) & 1, abortf, kBudgetNs)) return false;
+                if (gb >= (uint32_t)kSBuf &&
+                    !mbar_wait(smem_u32(&sm.pv_done[sb]), ((gb / kSBuf) - 1) & 1, abortf, kBudgetNs)) {
+                    dead = true;
+                    break;
+                }
+                if (!mbar_wait(smem_u32(&sm.k_full[slot]), (gb / kStages) & 1, abortf, kBudgetNs)) {
+                    dead = true;
+                    break;
+                }
                 tc_fence_after();
                 if (leader) {
                     const uint64_t adesc = sdesc_sw128(qaddr, 16, 1024);
@@ -352,15 +366,23 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     if (t == nblk - 1) mma_commit(smem_u32(&sm.q_empty[qb]));  // last read of this Q tile
                 }
                 __syncwarp();
-                return true;
-            };
-            if (nblk == 0 && leader) mma_commit(smem_u32(&sm.q_empty[qb]));
-            for (int t = 0; t < nblk && t < kSBuf; ++t)
-                if (!issue_qk(t)) {
-                    dead = true;
-                    break;
-                }
-            for (int t = 0; t < nblk && !dead; ++t) {
+            }
+            gblk += nblk;
+        }
+        if (dead && leader) {
+            mma_commit(smem_u32(&sm.drain[0]));
+            wait_raw(smem_u32(&sm.drain[0]), 0);
+        }
+    } else if (warp == 11) {
+        // ------------------------------------------------------------ PV issuer
+        // O += P_t V_t once the softmax has written P_t and V_t has landed; PVs of a pipeline
+        // are issued by this one thread, so they accumulate into O in order.
+        const bool leader = elect_one_sync();
+        uint32_t gblk = 0, nloc = 0;
+        const uint32_t vbase = smem_u32(&sm.v[0][0]);
+        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
+            const int nblk = item_nblk(p, item);
+            for (int t = 0; t < nblk; ++t) {
                 const uint32_t gb = gblk + t, sb = gb % kSBuf, slot = gb % kStages;
                 if (!mbar_wait(smem_u32(&sm.p_full[sb]), (gb / kSBuf) & 1, abortf, kBudgetNs)) {
                     dead = true;
@@ -387,10 +409,6 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     mma_commit(smem_u32(&sm.pv_done[sb]));
                 }
                 __syncwarp();
-                if (t + kSBuf < nblk && !issue_qk(t + kSBuf)) {
-                    dead = true;
-                    break;
-                }
             }
             if (dead) break;
             // an empty item writes no O, but o_full must still not run two phases ahead
@@ -404,8 +422,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             gblk += nblk;
         }
         if (dead && leader) {
-            mma_commit(smem_u32(&sm.drain));
-            wait_raw(smem_u32(&sm.drain), 0);
+            mma_commit(smem_u32(&sm.drain[1]));
+            wait_raw(smem_u32(&sm.drain[1]), 0);
         }
     } else if (warp < 6) {
         // ------------------------------------------------------------ softmax
@@ -473,16 +491,20 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                         }
                     }
                 }
+                // x = s * c - m and the row sums in packed fp32x2 arithmetic (two lanes per op)
                 uint32_t pk[16];
-                float ls[4] = {0.f, 0.f, 0.f, 0.f};
+                const float2 c2 = make_float2(c, c), nm2 = make_float2(-m_used, -m_used);
+                float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
                 for (int i = 0; i < 16; ++i) {
-                    const float p0 = fast_exp2(fmaf(__uint_as_float(sr[2 * i]), c, -m_used));
-                    const float p1 = fast_exp2(fmaf(__uint_as_float(sr[2 * i + 1]), c, -m_used));
-                    ls[i & 3] += p0 + p1;
-                    pk[i] = pack_bf16(p0, p1);
+                    const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[2 * i]), __uint_as_float(sr[2 * i + 1])),
+                                                c2, nm2);
+                    const float2 pp = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+                    ls2[i & 1] = __fadd2_rn(ls2[i & 1], pp);
+                    pk[i] = pack_bf16(pp.x, pp.y);
                 }
-                l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+                const float2 lsum = __fadd2_rn(ls2[0], ls2[1]);
+                l += lsum.x + lsum.y;
                 tmem_st_16x32bx2_x16_off16(tbase + lane_off + kColS + sb * 64, pk);
                 tmem_wait_st();
                 tc_fence_before();
@@ -550,18 +572,6 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             }
             if (half == 0)
                 p.lse[(size_t)bh * N + tok] = ok ? (st.x * 0.69314718055994531f + logf(st.y)) : -INFINITY;
-            // warm L2 with the tiles of the item two ahead (one lane per key block)
-            const int nxt = item + 2 * vgrid;
-            if (warp == 6 && nxt < p.num_items) {
-                const int nbh = nxt / Tb, nlabel = nxt - nbh * Tb;
-                if (lane == 0) window_boxes<true>(maps.q, 0, 0, g, nlabel, nbh);
-                const int nn = item_nblk(p, nxt);
-                for (int t = lane; t < nn; t += 32) {
-                    const int j = item_label(p, nxt, t, Tb);
-                    window_boxes<true>(maps.k, 0, 0, g, j, nbh);
-                    window_boxes<true>(maps.v, 0, 0, g, j, nbh);
-                }
-            }
         }
     }
 
