@@ -114,19 +114,38 @@ SSBA_API int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K
  *   kv_cnt      device, int32 [B][heads][Tb], each in [1, keep].
  *   O           device out, [B][heads][N][head_dim] of desc->dtype, original token order.
  *   lse         device out, fp32 [B][heads][N], natural log.
+ *   workspace   device, optional (NULL and 0 allowed): the split-merge area of the
+ *               bf16 kernel, at least ssba_forward_workspace_bytes(desc) bytes,
+ *               16-byte aligned. With it, and with lists of at least 24 blocks, the
+ *               persistent kernel gives its pipelines equal shares of key blocks and
+ *               cuts at most one query block per share boundary in two, merging the
+ *               parts' partial softmax sums; otherwise shares are whole query blocks
+ *               (up to one query block's work of imbalance).
+ *               Rules: zero-fill it once before its first use. Every call that
+ *               returns SSBA_OK and runs to completion leaves it zero-filled again,
+ *               so later calls ordered after it on the GPU reuse it as is. Calls that
+ *               may overlap on the GPU (two streams) need separate workspaces. After a
+ *               call that ends with the device status SSBA_ERR_TIMEOUT, zero it again.
+ *               fp32 ignores it.
  * bf16 runs on the tcgen05 tensor-core kernel and needs head_dim = 64, block = 8
  * and shifts that are multiples of 4; fp32 runs on the CUDA-core kernel with any
- * shift and head_dim = 64. Anything else returns SSBA_ERR_UNSUPPORTED. */
+ * shift and head_dim = 64. Anything else returns SSBA_ERR_UNSUPPORTED. A workspace
+ * smaller than required returns SSBA_ERR_WORKSPACE before any device work. */
 SSBA_API int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void* V,
                  const int32_t* kv_idx, const int32_t* kv_cnt, void* O, float* lse,
-                 void* stream);
+                 void* workspace, size_t ws_bytes, void* stream);
+
+/* Bytes of the optional ssba_forward / ssba_forward_dense workspace for desc on the
+ * current device (it scales with the device's SM count: about 10 MB on 152 SMs);
+ * 0 for an fp32 or an invalid descriptor. Host only, no device work. */
+SSBA_API size_t ssba_forward_workspace_bytes(const ssba_desc* desc);
 
 /* Dense softmax attention over all N keys with the same layout and outputs as
  * ssba_forward (the 0% sparsity "baseline" of Table 2), from the same build:
  * bf16 only, head_dim = 64, H_tok and W_tok multiples of 8 (block is ignored).
- * Shift and rho are ignored. */
+ * Shift and rho are ignored. The workspace follows the rules of ssba_forward. */
 SSBA_API int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, const void* V,
-                       void* O, float* lse, void* stream);
+                       void* O, float* lse, void* workspace, size_t ws_bytes, void* stream);
 
 /* Size of the scratch area built into the library for ssba_build_mask_noalloc (4 MiB). */
 #define SSBA_NOALLOC_SCRATCH_BYTES (4u << 20)

@@ -27,7 +27,8 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
                  4: "SSBA_ERR_TIMEOUT", 5: "SSBA_ERR_WORKSPACE"}
 
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
-            "ssba_forward", "ssba_forward_dense", "ssba_get_status", "ssba_last_error")
+            "ssba_forward", "ssba_forward_workspace_bytes", "ssba_forward_dense", "ssba_get_status",
+            "ssba_last_error")
 
 
 class SsbaError(RuntimeError):
@@ -100,9 +101,11 @@ def load_library():
         lib.ssba_build_mask.restype = ctypes.c_int
         lib.ssba_build_mask_noalloc.argtypes = [DP, P, P, P, P, P, P]
         lib.ssba_build_mask_noalloc.restype = ctypes.c_int
-        lib.ssba_forward.argtypes = [DP, P, P, P, P, P, P, P, P]
+        lib.ssba_forward.argtypes = [DP, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_forward.restype = ctypes.c_int
-        lib.ssba_forward_dense.argtypes = [DP, P, P, P, P, P, P]
+        lib.ssba_forward_workspace_bytes.argtypes = [DP]
+        lib.ssba_forward_workspace_bytes.restype = ctypes.c_size_t
+        lib.ssba_forward_dense.argtypes = [DP, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_forward_dense.restype = ctypes.c_int
         lib.ssba_get_status.argtypes = [ctypes.POINTER(ctypes.c_int32)]
         lib.ssba_get_status.restype = ctypes.c_int
@@ -148,6 +151,38 @@ def mask_workspace_bytes(desc: SsbaDesc) -> int:
     lib = load_library()
     d = desc.c()
     return int(lib.ssba_mask_workspace_bytes(ctypes.byref(d)))
+
+
+def forward_workspace_bytes(desc: SsbaDesc) -> int:
+    lib = load_library()
+    d = desc.c()
+    return int(lib.ssba_forward_workspace_bytes(ctypes.byref(d)))
+
+
+_fwd_ws: dict = {}
+
+
+def default_forward_workspace(desc: SsbaDesc, device) -> torch.Tensor:
+    """A zero-filled forward workspace kept per device and reused by every call that
+    passes none. The kernels leave it zero-filled, so calls ordered on one stream can
+    share it; calls that may overlap on the GPU must pass workspaces of their own."""
+    need = forward_workspace_bytes(desc)
+    dev = torch.device(device)
+    key = dev.index if dev.index is not None else torch.cuda.current_device()
+    with _lock:
+        ws = _fwd_ws.get(key)
+        if ws is None or ws.numel() < need:
+            ws = torch.zeros(max(need, 1), dtype=torch.uint8, device=dev)
+            _fwd_ws[key] = ws
+    return ws
+
+
+def _ws_args(ws):
+    if ws is None:
+        return None, 0
+    if not isinstance(ws, torch.Tensor) or ws.device.type != "cuda" or not ws.is_contiguous():
+        raise SsbaError(SSBA_ERR_INVALID, "workspace must be a contiguous CUDA tensor")
+    return ws.data_ptr(), ws.numel() * ws.element_size()
 
 
 def build_mask(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=None, kv_cnt=None,
@@ -217,8 +252,10 @@ def build_mask_noalloc(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=
     return (kv_idx, kv_cnt, S) if S is not None else (kv_idx, kv_cnt)
 
 
-def forward(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O=None, lse=None, stream=None):
-    """ssba_forward: returns (O [B,h,N,d] in desc.dtype, lse [B,h,N] fp32)."""
+def forward(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O=None, lse=None, workspace="default", stream=None):
+    """ssba_forward: returns (O [B,h,N,d] in desc.dtype, lse [B,h,N] fp32).
+    ``workspace``: "default" (the per-device one of default_forward_workspace), None (no
+    workspace: whole-query-block shares) or a zero-filled uint8 CUDA tensor."""
     lib = load_library()
     d = desc.c()
     keep = lib.ssba_keep_count(ctypes.byref(d))
@@ -235,14 +272,17 @@ def forward(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O=None, lse=None, stream=No
         lse = torch.empty(shp[:3], dtype=torch.float32, device=Q.device)
     _check(O, "O", shp, desc.dtype)
     _check(lse, "lse", shp[:3], torch.float32)
+    if isinstance(workspace, str):
+        workspace = default_forward_workspace(desc, Q.device) if desc.dtype == torch.bfloat16 else None
+    wp, wn = _ws_args(workspace)
     rc = lib.ssba_forward(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), kv_idx.data_ptr(),
-                          kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), _stream_ptr(stream))
+                          kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), wp, wn, _stream_ptr(stream))
     _raise_on(rc)
     return O, lse
 
 
-def forward_dense(desc: SsbaDesc, Q, K, V, O=None, lse=None, stream=None):
-    """ssba_forward_dense: dense softmax attention from the same build."""
+def forward_dense(desc: SsbaDesc, Q, K, V, O=None, lse=None, workspace="default", stream=None):
+    """ssba_forward_dense: dense softmax attention from the same build (workspace as in forward)."""
     lib = load_library()
     d = desc.c()
     shp = (desc.B, desc.heads, desc.N, desc.head_dim)
@@ -254,8 +294,11 @@ def forward_dense(desc: SsbaDesc, Q, K, V, O=None, lse=None, stream=None):
         lse = torch.empty(shp[:3], dtype=torch.float32, device=Q.device)
     _check(O, "O", shp, desc.dtype)
     _check(lse, "lse", shp[:3], torch.float32)
+    if isinstance(workspace, str):
+        workspace = default_forward_workspace(desc, Q.device) if desc.dtype == torch.bfloat16 else None
+    wp, wn = _ws_args(workspace)
     rc = lib.ssba_forward_dense(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), O.data_ptr(),
-                                lse.data_ptr(), _stream_ptr(stream))
+                                lse.data_ptr(), wp, wn, _stream_ptr(stream))
     _raise_on(rc)
     return O, lse
 
@@ -278,7 +321,8 @@ class BoundLayer:
     make the bare C calls (ssba_build_mask, ssba_forward) with no per-call checks, so
     that host overhead stays far below the kernels' run time in tight loops."""
 
-    def __init__(self, desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O, lse, workspace, stream=None):
+    def __init__(self, desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O, lse, workspace, stream=None,
+                 fwd_workspace="default"):
         lib = load_library()
         self._lib = lib
         self._d = desc.c()
@@ -292,13 +336,18 @@ class BoundLayer:
         need = mask_workspace_bytes(desc)
         if workspace.numel() * workspace.element_size() < need:
             raise SsbaError(SSBA_ERR_WORKSPACE, f"workspace needs {need} bytes")
-        self.tensors = (Q, K, V, kv_idx, kv_cnt, O, lse, workspace)  # keep alive
+        if isinstance(fwd_workspace, str):
+            fwd_workspace = default_forward_workspace(desc, Q.device) if desc.dtype == torch.bfloat16 else None
+        fwp, fwn = _ws_args(fwd_workspace)
+        if fwp is not None and fwn < forward_workspace_bytes(desc):
+            raise SsbaError(SSBA_ERR_WORKSPACE, f"forward workspace needs {forward_workspace_bytes(desc)} bytes")
+        self.tensors = (Q, K, V, kv_idx, kv_cnt, O, lse, workspace, fwd_workspace)  # keep alive
         st = _stream_ptr(stream)
         self._mask_args = (ctypes.byref(self._d), Q.data_ptr(), K.data_ptr(), kv_idx.data_ptr(),
                            kv_cnt.data_ptr(), None, workspace.data_ptr(),
                            workspace.numel() * workspace.element_size(), st)
         self._fwd_args = (ctypes.byref(self._d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), kv_idx.data_ptr(),
-                          kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), st)
+                          kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), fwp, fwn, st)
 
     def mask(self) -> None:
         rc = self._lib.ssba_build_mask(*self._mask_args)

@@ -156,8 +156,17 @@ int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K, int32_t
     return launch_select(*desc, g, keep, qb, kb, kv_idx, kv_cnt, scores_opt, st);
 }
 
+size_t ssba_forward_workspace_bytes(const ssba_desc* desc)
+{
+    Grid g;
+    int keep;
+    if (check_desc(desc, "ssba_forward_workspace_bytes", &g, &keep) != SSBA_OK) return 0;
+    if (desc->dtype != SSBA_BF16) return 0;
+    return attn_tc_workspace_bytes();
+}
+
 int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void* V, const int32_t* kv_idx,
-                 const int32_t* kv_cnt, void* O, float* lse, void* stream)
+                 const int32_t* kv_cnt, void* O, float* lse, void* workspace, size_t ws_bytes, void* stream)
 {
     Grid g;
     int keep;
@@ -172,17 +181,21 @@ int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void
         set_error("ssba_forward: Q, K, V, O must be 16-byte aligned; lse, kv_idx, kv_cnt 4-byte aligned");
         return SSBA_ERR_INVALID;
     }
+    if (workspace && !aligned(workspace, 16)) {
+        set_error("ssba_forward: workspace must be 16-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
     const float scale = resolve_scale(desc);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (desc->dtype == SSBA_FP32)
         return launch_attn_simt_f32(*desc, g, keep, scale, static_cast<const float*>(Q),
                                     static_cast<const float*>(K), static_cast<const float*>(V), kv_idx, kv_cnt,
                                     static_cast<float*>(O), lse, st);
-    return launch_attn_tc_bf16(*desc, g, keep, scale, Q, K, V, kv_idx, kv_cnt, O, lse, st);
+    return launch_attn_tc_bf16(*desc, g, keep, scale, Q, K, V, kv_idx, kv_cnt, O, lse, workspace, ws_bytes, st);
 }
 
 int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, const void* V, void* O, float* lse,
-                       void* stream)
+                       void* workspace, size_t ws_bytes, void* stream)
 {
     Grid g;
     int keep;
@@ -196,11 +209,15 @@ int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, cons
         set_error("ssba_forward_dense: Q, K, V, O must be 16-byte aligned; lse 4-byte aligned");
         return SSBA_ERR_INVALID;
     }
+    if (workspace && !aligned(workspace, 16)) {
+        set_error("ssba_forward_dense: workspace must be 16-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
     if (desc->dtype != SSBA_BF16) {
         set_error("ssba_forward_dense: bf16 only");
         return SSBA_ERR_UNSUPPORTED;
     }
-    return launch_dense_tc_bf16(*desc, resolve_scale(desc), Q, K, V, O, lse,
+    return launch_dense_tc_bf16(*desc, resolve_scale(desc), Q, K, V, O, lse, workspace, ws_bytes,
                                 static_cast<cudaStream_t>(stream));
 }
 

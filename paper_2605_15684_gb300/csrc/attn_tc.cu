@@ -63,7 +63,10 @@ constexpr uint32_t kTileBytes = kRows * kD * 2;  // 8 KB
 enum BoxShape { kBox8x8 = 0, kBox8c4r = 1, kBox4c8r = 2, kBox4x4 = 3 };
 constexpr uint64_t kBudgetNs = 2000000000ull;    // 2 s per wait
 constexpr float kRescaleLog2 = 8.0f;
-constexpr int kLabelCap = 256;  // labels staged per producer warp; longer lists are read per block
+constexpr int kLabelCap = 128;  // labels staged per producer warp and piece; the rest are read per block
+constexpr int kCntCap = 64;     // phase-B item counts of a pipeline held in shared memory
+constexpr int kCntA = 3;        // phase-A pieces of one pipeline: at most three
+constexpr int kSplitMinKeep = 24;  // shortest list for which items are cut to balance the pipelines
 
 // QK: M=64 N=64, A (Q) and B (K) K-major. PV: M=64 N=64, A (P) K-major, B (V) MN-major.
 constexpr uint32_t kIdescQK = idesc_bf16_f32(64, 64, false, false);
@@ -88,7 +91,10 @@ struct __align__(1024) SlotSmem {
     uint64_t o_full;
     uint64_t o_free;
     uint64_t drain[2];
-    int32_t labels[2][kLabelCap];  // key-block labels of the current item, per producer warp
+    int32_t labels[2][kLabelCap];     // [producer warp] key-block labels of the current piece
+    int32_t cnts[kCntCap];            // counts of the first phase-B items, in walk order
+    int4 pieceA[kCntA];               // phase-A pieces in walk order: item, tb, nb, part
+    int nA, nB, M;                    // phase-A pieces, phase-B items, phase-A items (all pipelines)
 };
 
 struct __align__(1024) SmemLayout {
@@ -112,6 +118,41 @@ struct TcParams {
     int num_items;
     float scale_log2;  // softmax scale * log2(e)
     int* status;       // device status word
+    // Split-merge workspace (null when the caller gave none; then split = 0).
+    int split;         // 1: pipelines take equal ranges of blocks, items may be cut in two
+    int* ws_cnt;       // [boundaries][4] arrival counters, zero between launches
+    float2* ws_st;     // [boundaries][2][64] row (max in log2 units, sum) of each part
+    float* ws_o;       // [boundaries][2][64][64] unnormalised O of each part, fp32
+};
+
+// Work schedule, for V pipelines (two per CTA).
+//   split = 0: whole items round-robin, item v + r V for pipeline v (neighbouring pipelines
+//     work on neighbouring items, so the K/V tiles of a few heads are shared through L2).
+//   split = 1 (a workspace was given and items is not a multiple of V, items >= V): the
+//     first M = items - (floor(items / V) - 1) V items (V <= M < 2V) form phase A, the rest
+//     phase B. Phase A counts in units (item, key block), item u / keep, block u % keep (a
+//     block past the item's count is an empty unit); pipeline v takes the units
+//     [floor(M keep v / V), floor(M keep (v+1) / V)), at least keep of them, so an item is
+//     cut at most once: at boundary v, into a first part (the last item of pipeline v-1)
+//     and a second part (the first item of pipeline v). Each part writes its unnormalised
+//     O and row statistics to the workspace, and the part that arrives second at the
+//     boundary's counter merges the two (two partial softmax sums combine by rescaling
+//     each by 2^(m_part - m), m the larger maximum, and adding) and resets the counter.
+//     Phase B is whole items round-robin, item M + v + r V. Every pipeline then has the
+//     same number of key blocks, give or take one.
+// A pipeline runs phase A first and, in it, its cut last item first, so that both parts
+// of every cut item finish early and the merges (a few global-memory round trips)
+// overlap later work instead of lengthening the end of the kernel.
+__device__ __forceinline__ int split_items(const TcParams& p, int V)
+{
+    return p.split ? p.num_items - (p.num_items / V - 1) * V : 0;
+}
+
+struct Piece {
+    int item;  // (batch, head) * Tb + query-block label
+    int tb;    // first block (position in the item's list)
+    int nb;    // blocks of this piece (0 for an empty piece)
+    int part;  // -1 whole item, 0 first part (boundary v + 1), 1 second part (boundary v)
 };
 
 __device__ __forceinline__ float fast_exp2(float x)
@@ -149,17 +190,6 @@ __device__ __forceinline__ void tmem_st_16x32bx2_x16_off32(uint32_t taddr, const
 
 __device__ __forceinline__ int clamp_label(int j, int Tb) { return j < 0 ? 0 : (j >= Tb ? Tb - 1 : j); }
 
-// Key blocks of an item: the listed ones (count clamped to [0, keep]), or, in dense
-// mode (no list), every block of the head.
-__device__ __forceinline__ int item_nblk(const TcParams& p, int item)
-{
-    return p.idx ? min(max(__ldg(p.cnt + item), 0), p.keep) : p.keep;
-}
-
-__device__ __forceinline__ int item_label(const TcParams& p, int item, int t, int Tb)
-{
-    return p.idx ? clamp_label(__ldg(p.idx + (size_t)item * p.keep + t), Tb) : t;
-}
 
 // Origin (row, col) of the shifted 8x8 window `label` in the unshifted grid. With block
 // 8 and a shift that is a multiple of 4, a window either fits (origin <= size - 8) or is
@@ -219,6 +249,63 @@ __device__ __forceinline__ int tile_row_pos(const Grid& g, int label, int r)
     return (4 * (q >> 1) + a) * 8 + 4 * (q & 1) + b;
 }
 
+// Piece k of pipeline v (V pipelines) from the schedule in shared memory.
+__device__ __forceinline__ Piece get_piece(const TcParams& p, const SlotSmem& sm, int k, int v, int V)
+{
+    Piece pc;
+    if (k < sm.nA) {
+        const int4 e = sm.pieceA[k];
+        pc.item = e.x;
+        pc.tb = e.y;
+        pc.nb = e.z;
+        pc.part = e.w;
+    } else {
+        const int r = k - sm.nA;
+        pc.item = sm.M + v + r * V;
+        pc.tb = 0;
+        pc.part = -1;
+        pc.nb = p.keep;
+        if (p.idx) pc.nb = min(max(r < kCntCap ? sm.cnts[r] : __ldg(p.cnt + pc.item), 0), p.keep);
+    }
+    return pc;
+}
+
+// Fills the schedule of pipeline v (thread t of its nthr threads); see the work-schedule
+// comment above.
+__device__ void build_schedule(const TcParams& p, SlotSmem& sm, int v, int V, int t, int nthr)
+{
+    const int M = split_items(p, V);
+    const int rest = p.num_items - M - v;
+    const int nB = rest > 0 ? (rest + V - 1) / V : 0;
+    if (p.idx)
+        for (int r = t; r < nB && r < kCntCap; r += nthr) sm.cnts[r] = __ldg(p.cnt + M + v + r * V);
+    if (t != 0) return;
+    int nA = 0;
+    if (M > 0) {
+        const long long u0 = (long long)M * p.keep * v / V, u1 = (long long)M * p.keep * (v + 1) / V;
+        const long long cut = u1 / p.keep * p.keep;  // start of the item holding unit u1 - 1
+        auto add = [&](long long a, long long b) {   // piece over units [a, b) of one item
+            const int item = (int)(a / p.keep);
+            const int tb = (int)(a - (long long)item * p.keep), te = (int)(b - (long long)item * p.keep);
+            const int n = p.idx ? min(max(__ldg(p.cnt + item), 0), p.keep) : p.keep;
+            sm.pieceA[nA++] = make_int4(item, tb, max(0, min(te, n) - tb), tb > 0 ? 1 : (te < p.keep ? 0 : -1));
+        };
+        long long uend = u1;
+        if (u1 % p.keep != 0 && cut > u0) {  // the cut last item goes first
+            add(cut, u1);
+            uend = cut;
+        }
+        for (long long u = u0; u < uend;) {
+            const long long next = min((u / p.keep + 1) * p.keep, uend);
+            add(u, next);
+            u = next;
+        }
+    }
+    sm.nA = nA;
+    sm.nB = nB;
+    sm.M = M;
+}
+
 __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ TileMaps maps,
                                                                     const TcParams p)
 {
@@ -230,8 +317,10 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     const int warp = gwarp % kSlotWarps;   // role within the pipeline
     SlotSmem& sm = cs.slot[slot];
     volatile int* abortf = &cs.abort_flag;
-    // pipeline `slot` of CTA b is virtual CTA 2b + slot of a grid of 2 * gridDim.x
-    const int vcta = blockIdx.x * kSlots + slot;
+    // pipeline `slot` of CTA b is pipeline b + slot * gridDim.x of 2 * gridDim.x: the items
+    // left over after whole rounds go to the first pipelines, one per CTA, and the other
+    // pipeline of such a CTA finishes first and leaves it the SM
+    const int vcta = slot * gridDim.x + blockIdx.x;
     const int vgrid = gridDim.x * kSlots;
     const Grid g = p.g;
     const int Tb = g.Tb();
@@ -262,6 +351,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         mbar_init(smem_u32(&sm.drain[1]), 1);
         fence_mbar_init();
     }
+    build_schedule(p, sm, vcta, vgrid, threadIdx.x % (kSlotWarps * 32), kSlotWarps * 32);
     if (gwarp == 0 && lane < 12) tma_prefetch_desc(lane < 4 ? &maps.q[lane] : (lane < 8 ? &maps.k[lane - 4] : &maps.v[lane - 8]));
     if (gwarp == 1) {
         tmem_alloc(smem_u32(&cs.tmem_base), kTmemCols);
@@ -281,15 +371,18 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         // rings do not wait on each other, and the two issuing threads overlap their TMA
         // issue latency (about 140 cycles per box per thread).
         const bool is_k = warp == 0;
-        int32_t* lab = sm.labels[is_k ? 0 : 1];
         uint32_t g = 0, nq = 0;
-        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nq) {
-            const int bh = item / Tb, label = item - bh * Tb;
-            const int nblk = item_nblk(p, item);
-            const int32_t* list = p.idx ? p.idx + (size_t)item * p.keep : nullptr;
-            // all lanes fetch the item's labels in one round; lane 0 then issues the copies
+        const int npieces = sm.nA + sm.nB;
+        for (int k = 0; !dead && k < npieces; ++k, ++nq) {
+            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+            const int bh = pc.item / Tb, label = pc.item - bh * Tb;
+            const int nblk = pc.nb;
+            const int32_t* list = p.idx ? p.idx + (size_t)pc.item * p.keep + pc.tb : nullptr;
+            // all lanes fetch the piece's labels in one round; lane 0 then issues the copies
+            // (measured: faster than prefetching them one piece ahead with cp.async)
+            int32_t* lab = sm.labels[is_k ? 0 : 1];
             if (list)
-                for (int t = lane; t < nblk && t < kLabelCap; t += 32) lab[t] = clamp_label(__ldg(list + t), Tb);
+                for (int t = lane; t < nblk && t < kLabelCap; t += 32) lab[t] = __ldg(list + t);
             __syncwarp();
             if (lane == 0) {
                 if (is_k) {
@@ -301,7 +394,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     }
                 }
                 for (int t = 0; t < nblk && !dead; ++t, ++g) {
-                    const int j = !list ? t : (t < kLabelCap ? lab[t] : clamp_label(__ldg(list + t), Tb));
+                    const int j = !list ? pc.tb + t : clamp_label(t < kLabelCap ? lab[t] : __ldg(list + t), Tb);
                     const uint32_t slot = g % kStages;
                     uint64_t* empty = is_k ? &sm.k_empty[slot] : &sm.v_empty[slot];
                     uint64_t* full = is_k ? &sm.k_full[slot] : &sm.v_full[slot];
@@ -333,8 +426,10 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         const bool leader = elect_one_sync();
         uint32_t gblk = 0, nloc = 0;
         const uint32_t kbase = smem_u32(&sm.k[0][0]);
-        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
-            const int nblk = item_nblk(p, item);
+        const int npieces = sm.nA + sm.nB;
+        for (int k = 0; !dead && k < npieces; ++k, ++nloc) {
+            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+            const int nblk = pc.nb;
             const uint32_t qb = nloc & 1;
             const uint32_t qaddr = smem_u32(&sm.q[qb][0]);
             if (!mbar_wait(smem_u32(&sm.q_full[qb]), (nloc >> 1) & 1, abortf, kBudgetNs)) {
@@ -380,8 +475,10 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         const bool leader = elect_one_sync();
         uint32_t gblk = 0, nloc = 0;
         const uint32_t vbase = smem_u32(&sm.v[0][0]);
-        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
-            const int nblk = item_nblk(p, item);
+        const int npieces = sm.nA + sm.nB;
+        for (int k = 0; !dead && k < npieces; ++k, ++nloc) {
+            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+            const int nblk = pc.nb;
             for (int t = 0; t < nblk; ++t) {
                 const uint32_t gb = gblk + t, sb = gb % kSBuf, slot = gb % kStages;
                 if (!mbar_wait(smem_u32(&sm.p_full[sb]), (gb / kSBuf) & 1, abortf, kBudgetNs)) {
@@ -433,8 +530,10 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
         const float c = p.scale_log2;
         uint32_t gblk = 0, nloc = 0;
-        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
-            const int nblk = item_nblk(p, item);
+        const int npieces = sm.nA + sm.nB;
+        for (int k = 0; !dead && k < npieces; ++k, ++nloc) {
+            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+            const int nblk = pc.nb;
             float m_used = 0.f, l = 0.f;
             for (int t = 0; t < nblk; ++t) {
                 const uint32_t gb = gblk + t, sb = gb % kSBuf;
@@ -531,8 +630,10 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         const int row = quad * 16 + (lane & 15);
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
         uint32_t nloc = 0;
-        for (int item = vcta; item < p.num_items && !dead; item += vgrid, ++nloc) {
-            const int bh = item / Tb, label = item - bh * Tb;
+        const int npieces = sm.nA + sm.nB;
+        for (int k = 0; !dead && k < npieces; ++k, ++nloc) {
+            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+            const int bh = pc.item / Tb, label = pc.item - bh * Tb;
             const uint32_t eb = nloc & 1;
             if (!mbar_wait(smem_u32(&sm.o_full), nloc & 1, abortf, kBudgetNs)) {
                 dead = true;
@@ -550,9 +651,47 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 dead = true;
                 break;
             }
-            const float2 st = sm.stats[eb][row];
+            float2 st = sm.stats[eb][row];
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&sm.stats_free[eb]));
+
+            if (pc.part >= 0) {
+                // a cut item: publish this part, and if the other part is already there,
+                // merge (each warp owns 16 rows, so the hand-off is per warp)
+                const int bidx = pc.part == 1 ? vcta : vcta + 1;
+                const size_t mine = (size_t)bidx * 2 + pc.part, other = mine ^ 1;
+                float4* wo = reinterpret_cast<float4*>(p.ws_o + (mine * kRows + row) * kD + half * 32);
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    wo[i] = make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]),
+                                        __uint_as_float(o[4 * i + 2]), __uint_as_float(o[4 * i + 3]));
+                if (half == 0) p.ws_st[mine * kRows + row] = st;
+                __threadfence();
+                __syncwarp();
+                int arrived = 0;
+                if (lane == 0) arrived = atomicAdd(p.ws_cnt + bidx * 4 + quad, 1);
+                arrived = __shfl_sync(0xffffffffu, arrived, 0);
+                if (arrived == 0) continue;  // first here: the other part merges
+                if (lane == 0) atomicExch(p.ws_cnt + bidx * 4 + quad, 0);  // ready for the next launch
+                __threadfence();
+                const float2 os = __ldcg(p.ws_st + other * kRows + row);
+                const float4* oo = reinterpret_cast<const float4*>(p.ws_o + (other * kRows + row) * kD + half * 32);
+                // an empty part (sum 0) contributes nothing; its O was never written
+                const bool a_ok = st.y > 0.f, b_ok = os.y > 0.f;
+                const float m = a_ok ? (b_ok ? fmaxf(st.x, os.x) : st.x) : os.x;
+                const float wa = a_ok ? fast_exp2(st.x - m) : 0.f, wb = b_ok ? fast_exp2(os.x - m) : 0.f;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float4 x = __ldcg(oo + i);
+                    const float xb[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float a = a_ok ? __uint_as_float(o[4 * i + e]) * wa : 0.f;
+                        o[4 * i + e] = __float_as_uint(b_ok ? fmaf(xb[e], wb, a) : a);
+                    }
+                }
+                st = make_float2(m, (a_ok ? st.y * wa : 0.f) + (b_ok ? os.y * wb : 0.f));
+            }
 
             const bool ok = st.y > 0.f;
             const float inv = ok ? 1.f / st.y : 0.f;
@@ -620,27 +759,47 @@ bool encode_window_maps(CUtensorMap* m4, const void* base, int BH, int H, int W)
     return true;
 }
 
+// SM count of the current device (1 when it cannot be read; not cached then).
 int num_sms()
 {
     static int n = 0;
-    if (!n) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        if (n <= 0) n = 1;
+    if (n > 0) return n;
+    int dev = 0, m = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&m, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || m <= 0) {
+        cudaGetLastError();
+        return 1;
     }
+    n = m;
     return n;
 }
 
 }  // namespace
 
+// Split-merge workspace: counters, then row statistics, then O parts, for one boundary
+// per pipeline of the largest grid this device runs (two per SM) plus one.
+namespace {
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+int max_grid() { return num_sms(); }
+size_t ws_boundaries() { return (size_t)kSlots * max_grid() + 1; }
+size_t ws_cnt_bytes() { return align256(ws_boundaries() * 4 * sizeof(int)); }
+size_t ws_st_bytes() { return align256(ws_boundaries() * 2 * kRows * sizeof(float2)); }
+size_t ws_o_bytes() { return ws_boundaries() * 2 * kRows * kD * sizeof(float); }
+}  // namespace
+
+size_t attn_tc_workspace_bytes() { return ws_cnt_bytes() + ws_st_bytes() + ws_o_bytes(); }
+
 int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
-                        const void* V, const int32_t* idx, const int32_t* cnt, void* O, float* lse,
-                        cudaStream_t st)
+                        const void* V, const int32_t* idx, const int32_t* cnt, void* O, float* lse, void* ws,
+                        size_t ws_bytes, cudaStream_t st)
 {
     if (d.head_dim != kD || g.blk != 8 || (g.sr % 4) || (g.sc % 4)) {
         set_error("ssba_forward (bf16): needs head_dim=64, block=8 and shifts that are multiples of 4");
         return SSBA_ERR_UNSUPPORTED;
+    }
+    if (ws && ws_bytes < attn_tc_workspace_bytes()) {
+        set_error("ssba_forward (bf16): workspace of %zu bytes, %zu needed", ws_bytes, attn_tc_workspace_bytes());
+        return SSBA_ERR_WORKSPACE;
     }
     const int BH = d.B * d.heads;
     TileMaps maps;
@@ -674,7 +833,23 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
     // A kernel that uses tensor memory gets one CTA per SM, so each CTA runs kSlots
     // pipelines; the persistent grid has one CTA per SM (fewer for small problems).
     const int want = (p.num_items + kSlots - 1) / kSlots;
-    const int grid = want < num_sms() ? want : num_sms();
+    const int grid = want < max_grid() ? want : max_grid();
+    p.split = 0;
+    p.ws_cnt = nullptr;
+    p.ws_st = nullptr;
+    p.ws_o = nullptr;
+    if (ws) {
+        char* w = static_cast<char*>(ws);
+        p.ws_cnt = reinterpret_cast<int*>(w);
+        p.ws_st = reinterpret_cast<float2*>(w + ws_cnt_bytes());
+        p.ws_o = reinterpret_cast<float*>(w + ws_cnt_bytes() + ws_st_bytes());
+        // Equal shares of blocks only pay when some pipeline would otherwise take one item
+        // more than another, and when items are long: a merge costs a few global-memory
+        // round trips (about 5 us under load, measured), which 11-block items do not
+        // earn back but 64-block items (dense) do (173 vs 190 us at 1024 px, 24 heads).
+        p.split = (keep >= kSplitMinKeep && p.num_items >= kSlots * grid && p.num_items % (kSlots * grid) != 0)
+                      ? 1 : 0;
+    }
     ssba_attn_tc_kernel<<<grid, kThreads, smem, st>>>(maps, p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
@@ -687,7 +862,7 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
 // Dense attention from the same kernel: no list, every key block visited in label
 // order with query tiles of one 8x8 block each (unshifted grid).
 int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V, void* O,
-                         float* lse, cudaStream_t st)
+                         float* lse, void* ws, size_t ws_bytes, cudaStream_t st)
 {
     if (d.head_dim != kD || d.H_tok % 8 || d.W_tok % 8) {
         set_error("ssba_forward_dense: needs head_dim=64 and H_tok, W_tok multiples of 8");
@@ -700,7 +875,7 @@ int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const v
     g.sr = 0;
     g.sc = 0;
     g.bw = d.W_tok / 8;
-    return launch_attn_tc_bf16(d, g, g.Tb(), scale, Q, K, V, nullptr, nullptr, O, lse, st);
+    return launch_attn_tc_bf16(d, g, g.Tb(), scale, Q, K, V, nullptr, nullptr, O, lse, ws, ws_bytes, st);
 }
 
 }  // namespace ssba

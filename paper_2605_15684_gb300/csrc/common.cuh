@@ -45,9 +45,11 @@ int launch_attn_simt_f32(const ssba_desc& d, const Grid& g, int keep, float scal
                          float* lse, cudaStream_t st);
 int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q,
                         const void* K, const void* V, const int32_t* idx, const int32_t* cnt, void* O,
-                        float* lse, cudaStream_t st);
+                        float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
 int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V,
-                         void* O, float* lse, cudaStream_t st);
+                         void* O, float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
+// Bytes of the split-merge workspace of the bf16 forward on the current device.
+size_t attn_tc_workspace_bytes();
 
 // Thread-local error text for ssba_last_error().
 void set_error(const char* fmt, ...);

@@ -71,7 +71,7 @@ def test_workspace_bytes(lib):
 def test_invalid_descriptors_are_rejected(lib, bad):
     d = desc(**bad)
     assert lib.ssba_keep_count(ctypes.byref(d)) == -1
-    rc = lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None)
+    rc = lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, 0, None)
     assert rc == api.SSBA_ERR_INVALID
     assert lib.ssba_last_error()
 
@@ -87,9 +87,9 @@ def test_null_and_misaligned_pointers(lib):
         api.SSBA_ERR_WORKSPACE
     assert lib.ssba_build_mask(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, None, None, ws, None) == \
         api.SSBA_ERR_WORKSPACE
-    assert lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, None) == \
+    assert lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, None, 0, None) == \
         api.SSBA_ERR_INVALID
-    assert lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE + 8, FAKE, FAKE, FAKE, FAKE, None) == \
+    assert lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE + 8, FAKE, FAKE, FAKE, FAKE, None, 0, None) == \
         api.SSBA_ERR_INVALID
     assert b"aligned" in lib.ssba_last_error()
 
@@ -99,9 +99,25 @@ def test_null_and_misaligned_pointers(lib):
 def test_tensor_core_path_rejects_unsupported_shapes(lib, bad):
     """The bf16 path needs head_dim 64, 8x8 blocks and 4-aligned shifts; it says so before launching."""
     d = desc(**bad)
-    rc = lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None)
+    rc = lib.ssba_forward(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, 0, None)
     assert rc == api.SSBA_ERR_UNSUPPORTED
     assert b"multiples of 4" in lib.ssba_last_error()
+
+
+def test_forward_workspace_rules(lib):
+    """The optional forward workspace: sized by the library, checked for size and
+    alignment before any launch, and not needed by the fp32 path."""
+    d = desc()
+    need = lib.ssba_forward_workspace_bytes(ctypes.byref(d))
+    assert need > 0 and need % 16 == 0
+    assert lib.ssba_forward_workspace_bytes(ctypes.byref(desc(dtype=api.SSBA_FP32))) == 0
+    assert lib.ssba_forward_workspace_bytes(ctypes.byref(desc(H_tok=12))) == 0
+    args = (ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE)
+    assert lib.ssba_forward(*args, FAKE, need - 16, None) == api.SSBA_ERR_WORKSPACE
+    assert b"workspace" in lib.ssba_last_error()
+    assert lib.ssba_forward(*args, FAKE + 8, need, None) == api.SSBA_ERR_INVALID
+    assert lib.ssba_forward_dense(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 16, None) == \
+        api.SSBA_ERR_WORKSPACE
 
 
 def test_build_mask_rejects_unsupported_head_dim(lib):

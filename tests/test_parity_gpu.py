@@ -181,3 +181,95 @@ def test_end_to_end_layer_with_gpu_mask():
 def test_status_word_reads_ok():
     torch.cuda.synchronize()
     assert api.get_status() == api.SSBA_OK
+
+
+# ----------------------------------------------------------------------------- split schedule
+# With a forward workspace and lists of at least 24 blocks, the bf16 kernel gives each of
+# its pipelines (two per SM) an equal share of key blocks and cuts the query blocks that
+# straddle two shares, merging the two parts. 5 heads of a 64x64 grid are 320 query
+# blocks: more than 2 x 152 pipelines and not a multiple of them, so shares end inside
+# query blocks. rho = 0.5 keeps 32 of 64 blocks.
+G = 64
+
+
+def _split_inputs(seed, heads=5, rho=0.5, shift=(4, 4)):
+    q, k, v, qd, kd, vd = _inputs(1, heads, G, G, torch.bfloat16, seed)
+    desc = api.SsbaDesc(1, heads, G, G, shift_r=shift[0], shift_c=shift[1], rho=rho)
+    idx_o, cnt_o = oracle.build_mask(q, k, G, G, 8, shift, rho)
+    return desc, (q, k, v, qd, kd, vd), idx_o, cnt_o
+
+
+def test_forward_split_and_whole_shares_agree_with_oracle():
+    desc, (q, k, v, qd, kd, vd), idx_o, cnt_o = _split_inputs(0)
+    assert idx_o.shape[-1] == 32
+    O_o, lse_o = oracle.forward(q, k, v, idx_o, G, G, 8, (4, 4))
+    idx_d, cnt_d = torch.from_numpy(idx_o).cuda(), torch.from_numpy(cnt_o).cuda()
+    ws = torch.zeros(api.forward_workspace_bytes(desc), dtype=torch.uint8, device="cuda")
+    for w in (ws, None):
+        O, lse = api.forward(desc, qd, kd, vd, idx_d, cnt_d, workspace=w)
+        torch.cuda.synchronize()
+        check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
+def test_forward_split_workspace_reused_across_calls():
+    """Calls in a row on one workspace, each on new inputs: the boundary counters must
+    be back at zero after every call, or a later call would merge stale parts."""
+    ws = None
+    for seed in (1, 2, 3):
+        desc, (q, k, v, qd, kd, vd), idx_o, cnt_o = _split_inputs(seed, shift=(0, 0) if seed == 2 else (4, 4))
+        if ws is None:
+            ws = torch.zeros(api.forward_workspace_bytes(desc), dtype=torch.uint8, device="cuda")
+        O, lse = api.forward(desc, qd, kd, vd, torch.from_numpy(idx_o).cuda(), torch.from_numpy(cnt_o).cuda(),
+                             workspace=ws)
+        torch.cuda.synchronize()
+        O_o, lse_o = oracle.forward(q, k, v, idx_o, G, G, 8, (desc.shift_r, desc.shift_c))
+        check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+    nsm = torch.cuda.get_device_properties(0).multi_processor_count
+    counters = ws[: (2 * nsm + 1) * 16].view(torch.int32)
+    assert int(counters.abs().sum()) == 0
+
+
+def test_forward_split_ragged_counts():
+    """Counts below the list length: many cut query blocks have an empty part (no block
+    of the part's range is below the count), which must contribute nothing to the merge.
+    The expected rows come from the oracle run on the lists truncated to each count."""
+    desc, (q, k, v, qd, kd, vd), idx_o, _ = _split_inputs(4)
+    keep = idx_o.shape[-1]
+    Tb = G * G // 64
+    choices = np.array([1, 9, 17, 25, keep], dtype=np.int32)
+    items = np.arange(desc.B * desc.heads * Tb).reshape(desc.B, desc.heads, Tb)
+    cnt = choices[(items * 7) % len(choices)]
+    O, lse = api.forward(desc, qd, kd, vd, torch.from_numpy(idx_o).cuda(), torch.from_numpy(cnt).cuda())
+    torch.cuda.synchronize()
+    lab = oracle.partition(G, G, 8, (4, 4))
+    O_ref = np.empty((desc.B, desc.heads, G * G, 64))
+    lse_ref = np.empty((desc.B, desc.heads, G * G))
+    for c in choices:
+        O_c, lse_c = oracle.forward(q, k, v, np.ascontiguousarray(idx_o[..., :c]), G, G, 8, (4, 4))
+        sel = cnt[:, :, lab] == c  # [B, heads, N]: rows whose query block has count c
+        O_ref[sel] = O_c[sel]
+        lse_ref[sel] = lse_c[sel]
+    check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_ref, lse_ref, "bf16")
+
+
+def test_forward_dense_split_schedule():
+    q, k, v, qd, kd, vd = _inputs(1, 5, G, G, torch.bfloat16, seed=5)
+    desc = api.SsbaDesc(1, 5, G, G)
+    O_o, lse_o = oracle.dense_forward(q, k, v)
+    for w in ("default", None):
+        O, lse = api.forward_dense(desc, qd, kd, vd, workspace=w)
+        torch.cuda.synchronize()
+        check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
+def test_forward_headline_whole_shares():
+    """1024 px headline with and without a workspace (11-block lists: whole query blocks
+    either way)."""
+    q, k, v, qd, kd, vd = _inputs(1, 24, 64, 64, torch.bfloat16)
+    desc = api.SsbaDesc(1, 24, 64, 64, shift_r=4, shift_c=4, rho=0.8416)
+    idx_o, cnt_o = oracle.build_mask(q, k, 64, 64, 8, (4, 4), 0.8416)
+    O, lse = api.forward(desc, qd, kd, vd, torch.from_numpy(idx_o).cuda(), torch.from_numpy(cnt_o).cuda(),
+                         workspace=None)
+    torch.cuda.synchronize()
+    O_o, lse_o = oracle.forward(q, k, v, idx_o, 64, 64, 8, (4, 4))
+    check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
