@@ -5,7 +5,7 @@
 // Work item = one query block (64 tokens, an 8x8 window of the shifted grid) of one
 // (batch, head); it visits only the key blocks listed for it. Persistent CTAs, one per SM
 // (a kernel that uses tensor memory gets one CTA per SM), each running two independent
-// pipelines of 12 warps (768 threads), warp-specialised:
+// pipelines of 12 warps (768 threads), warp-specialised by warpgroup:
 //   warp 0      TMA producer (Q, K). Q of each item and K, V of each listed key block arrive as
 //               8 KB tiles cut from [B*heads, H, W, d] tensor maps (128-byte swizzle): one
 //               8x8-token box when the shifted window does not cross the grid edge, else two
@@ -13,28 +13,32 @@
 //               window splits 4 + 4: no gather pass and no out-of-range fill. Q is
 //               double-buffered; K and V have separate 5-stage rings (a K slot frees when
 //               its QK is done, a V slot when its PV is done).
-//   warp 10     TMA producer of the V ring (warp 0 keeps Q and K), so that two threads
-//               share the per-box issue latency.
 //   warp 1      QK issuer (one elected lane; warp 1 of the CTA also owns the TMEM allocation):
 //                 S_t = Q K_t^T   tcgen05.mma kind::f16, M=64 N=64, A = Q tile and
 //                                 B = K tile from shared memory (K-major, SW128)
-//               S is triple-buffered: QK of block t waits until PV of block t-3 has read
-//               the P it overwrites.
-//   warp 11     PV issuer (one elected lane):
-//                 O  += P_t V_t   tcgen05.mma kind::f16, M=64 N=64, A = P from TMEM
-//                                 (written over S_t), B = V tile (MN-major, SW128)
-//               Two issuing threads keep one's barrier waits (about 100 cycles per query)
-//               off the other's issue path.
-//   warps 2-5   softmax, one TMEM lane quadrant each. The M=64 data path puts tile row r
+//               S is double-buffered in TMEM: QK of block t waits only until the softmax
+//               has loaded S_{t-2} into registers.
+//   warp 2      TMA producer of the V ring (warp 0 keeps Q and K), so that two threads
+//               share the per-box issue latency.
+//   warp 3      PV issuer (one elected lane):
+//                 O  += P_t V_t   tcgen05.mma kind::f16, M=64 N=64, A = P from TMEM,
+//                                 B = V tile (MN-major, SW128)
+//               P has its own two TMEM buffers (bf16 pairs, 32 columns each), so an S
+//               buffer is not held while its P waits for the PV. TMEM of a pipeline:
+//               S 2 x 64 + P 2 x 32 + O 64 = 256 columns. Two issuing threads keep one's
+//               barrier waits (about 100 cycles per query) off the other's issue path.
+//   warps 4-7   softmax, one TMEM lane quadrant each. The M=64 data path puts tile row r
 //               at lane 32*(r/16) + r%16, so two threads share a row (16x32bx2 TMEM
 //               loads), each holding 32 of its 64 scores. Online softmax in fp32 with exp2
 //               in the log2-scaled domain; the running max is only raised when it grows by
-//               more than 2^8 (then O is rescaled in TMEM), which keeps P <= 256 in bf16.
-//               At the end of an item the row statistics (max, sum) go to shared memory.
-//   warps 6-9   epilogue: O / l in bf16 and lse, overlapping the next item's softmax.
-// Tile rows follow the TMA box order of the window (tile_row_pos). All mbarrier waits are bounded (globaltimer budget + CTA abort
-// flag); a timeout is reported in the device status word and the CTA drains its
-// in-flight copies and MMAs before it exits.
+//               more than 2^8, which keeps P <= 256 in bf16; O is then rescaled in TMEM
+//               after P_t is stored, so that S and O never share the registers (80 per
+//               thread: 768 threads on one SM). At the end of an item the row statistics
+//               (max, sum) go to shared memory.
+//   warps 8-11  epilogue: O / l in bf16 and lse, overlapping the next item's softmax.
+// Tile rows follow the TMA box order of the window (tile_row_pos). All mbarrier waits are
+// bounded (globaltimer budget + CTA abort flag); a timeout is reported in the device status
+// word and the CTA drains its in-flight copies and MMAs before it exits.
 #include <cuda.h>
 #include <cstdio>
 
@@ -49,14 +53,17 @@ using namespace ptx;
 
 constexpr int kD = 64;
 constexpr int kRows = 64;  // query rows per item = tokens per block
-constexpr int kStages = 5;
-constexpr int kSBuf = 3;
+constexpr int kKStages = 5;  // K ring
+constexpr int kVStages = 5;  // V ring
+constexpr int kSBuf = 2;     // S buffers in TMEM (fp32, 64 columns each)
+constexpr int kPBuf = 2;     // P buffers in TMEM (bf16 pairs, 32 columns each)
 constexpr int kSlotWarps = 12;                // warps of one pipeline (see the role map above)
 constexpr int kSlots = 2;                     // independent pipelines per CTA
 constexpr int kThreads = kSlots * kSlotWarps * 32;
 constexpr uint32_t kSlotCols = 256;           // TMEM columns of one pipeline
 constexpr uint32_t kTmemCols = kSlots * kSlotCols;
-constexpr uint32_t kColS = 0;    // S/P buffers: [0,64), [64,128), [128,192)
+constexpr uint32_t kColS = 0;    // S buffers: [0,64), [64,128)
+constexpr uint32_t kColP = 128;  // P buffers: [128,160), [160,192)
 constexpr uint32_t kColO = 192;  // O accumulator: [192,256)
 constexpr uint32_t kTileBytes = kRows * kD * 2;  // 8 KB
 // Tensor-map box shapes (d x cols x rows) used to cut a shifted 8x8 window out of the grid.
@@ -73,19 +80,20 @@ constexpr uint32_t kIdescQK = idesc_bf16_f32(64, 64, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(64, 64, false, true);
 
 struct __align__(1024) SlotSmem {
-    uint8_t k[kStages][kTileBytes];
-    uint8_t v[kStages][kTileBytes];
+    uint8_t k[kKStages][kTileBytes];
+    uint8_t v[kVStages][kTileBytes];
     uint8_t q[2][kTileBytes];
     float2 stats[2][kRows];  // (max in log2 units, row sum) per item parity
-    uint64_t k_full[kStages];
-    uint64_t k_empty[kStages];
-    uint64_t v_full[kStages];
-    uint64_t v_empty[kStages];
+    uint64_t k_full[kKStages];
+    uint64_t k_empty[kKStages];
+    uint64_t v_full[kVStages];
+    uint64_t v_empty[kVStages];
     uint64_t q_full[2];
     uint64_t q_empty[2];
     uint64_t s_full[kSBuf];
-    uint64_t p_full[kSBuf];
-    uint64_t pv_done[kSBuf];
+    uint64_t s_free[kSBuf];   // the softmax has loaded S_t: QK_{t+2} may overwrite it
+    uint64_t p_full[kPBuf];
+    uint64_t p_empty[kPBuf];  // PV_t has finished (it read P_t; O holds it)
     uint64_t stats_full[2];
     uint64_t stats_free[2];
     uint64_t o_full;
@@ -328,16 +336,21 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
 
     if (threadIdx.x % (kSlotWarps * 32) == 0) {
         if (slot == 0) cs.abort_flag = 0;
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kKStages; ++s) {
             mbar_init(smem_u32(&sm.k_full[s]), 1);
             mbar_init(smem_u32(&sm.k_empty[s]), 1);
+        }
+        for (int s = 0; s < kVStages; ++s) {
             mbar_init(smem_u32(&sm.v_full[s]), 1);
             mbar_init(smem_u32(&sm.v_empty[s]), 1);
         }
         for (int b = 0; b < kSBuf; ++b) {
             mbar_init(smem_u32(&sm.s_full[b]), 1);
+            mbar_init(smem_u32(&sm.s_free[b]), 4);
+        }
+        for (int b = 0; b < kPBuf; ++b) {
             mbar_init(smem_u32(&sm.p_full[b]), 4);
-            mbar_init(smem_u32(&sm.pv_done[b]), 1);
+            mbar_init(smem_u32(&sm.p_empty[b]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&sm.q_full[b]), 1);
@@ -363,18 +376,18 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     const uint32_t tbase = cs.tmem_base + slot * kSlotCols;
     bool dead = false;
 
-    if (warp == 0 || warp == 10) {
+    if (warp == 0 || warp == 2) {
         // ------------------------------------------------------------ TMA producers
         // Warp 0 loads each item's Q tile and the K tiles of its key blocks into the K ring,
-        // warp 10 the V tiles into the V ring; one elected lane each, blocking (suspending)
+        // warp 2 the V tiles into the V ring; one elected lane each, blocking (suspending)
         // waits. A K slot frees when its QK is done and a V slot when its PV is done, so the
         // rings do not wait on each other, and the two issuing threads overlap their TMA
         // issue latency (about 140 cycles per box per thread).
         const bool is_k = warp == 0;
         uint32_t g = 0, nq = 0;
         const int npieces = sm.nA + sm.nB;
-        for (int k = 0; !dead && k < npieces; ++k, ++nq) {
-            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+        for (int pi = 0; !dead && pi < npieces; ++pi, ++nq) {
+            const Piece pc = get_piece(p, sm, pi, vcta, vgrid);
             const int bh = pc.item / Tb, label = pc.item - bh * Tb;
             const int nblk = pc.nb;
             const int32_t* list = p.idx ? p.idx + (size_t)pc.item * p.keep + pc.tb : nullptr;
@@ -395,10 +408,10 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 }
                 for (int t = 0; t < nblk && !dead; ++t, ++g) {
                     const int j = !list ? pc.tb + t : clamp_label(t < kLabelCap ? lab[t] : __ldg(list + t), Tb);
-                    const uint32_t slot = g % kStages;
+                    const uint32_t nst = is_k ? kKStages : kVStages, slot = g % nst;
                     uint64_t* empty = is_k ? &sm.k_empty[slot] : &sm.v_empty[slot];
                     uint64_t* full = is_k ? &sm.k_full[slot] : &sm.v_full[slot];
-                    if (!mbar_wait(smem_u32(empty), ((g / kStages) & 1) ^ 1, abortf, kBudgetNs)) {
+                    if (!mbar_wait(smem_u32(empty), ((g / nst) & 1) ^ 1, abortf, kBudgetNs)) {
                         dead = true;
                         break;
                     }
@@ -412,8 +425,9 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         }
         if (dead && lane == 0) {
             // drain: wait for the copies this thread issued that may still be in flight
-            for (uint32_t x = g > (uint32_t)kStages ? g - kStages : 0; x < g; ++x)
-                wait_raw(smem_u32(is_k ? &sm.k_full[x % kStages] : &sm.v_full[x % kStages]), (x / kStages) & 1);
+            const uint32_t nst = is_k ? kKStages : kVStages;
+            for (uint32_t x = g > nst ? g - nst : 0; x < g; ++x)
+                wait_raw(smem_u32(is_k ? &sm.k_full[x % nst] : &sm.v_full[x % nst]), (x / nst) & 1);
             if (is_k)
                 for (uint32_t n = nq > 1 ? nq - 1 : 0; n <= nq; ++n)
                     wait_raw(smem_u32(&sm.q_full[n & 1]), (n >> 1) & 1);
@@ -421,14 +435,13 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------------------ QK issuer
-        // S_t = Q K_t^T into S buffer t % 3. The buffer still holds P_{t-3} until PV_{t-3}
-        // has finished reading it, so QK_t waits for that PV's completion (pv_done).
+        // S_t = Q K_t^T into S buffer t % 3, once the softmax has loaded S_{t-3} from it.
         const bool leader = elect_one_sync();
         uint32_t gblk = 0, nloc = 0;
         const uint32_t kbase = smem_u32(&sm.k[0][0]);
         const int npieces = sm.nA + sm.nB;
-        for (int k = 0; !dead && k < npieces; ++k, ++nloc) {
-            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+        for (int pi = 0; !dead && pi < npieces; ++pi, ++nloc) {
+            const Piece pc = get_piece(p, sm, pi, vcta, vgrid);
             const int nblk = pc.nb;
             const uint32_t qb = nloc & 1;
             const uint32_t qaddr = smem_u32(&sm.q[qb][0]);
@@ -438,13 +451,13 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             }
             if (nblk == 0 && leader) mma_commit(smem_u32(&sm.q_empty[qb]));
             for (int t = 0; t < nblk; ++t) {
-                const uint32_t gb = gblk + t, slot = gb % kStages, sb = gb % kSBuf;
+                const uint32_t gb = gblk + t, slot = gb % kKStages, sb = gb % kSBuf;
                 if (gb >= (uint32_t)kSBuf &&
-                    !mbar_wait(smem_u32(&sm.pv_done[sb]), ((gb / kSBuf) - 1) & 1, abortf, kBudgetNs)) {
+                    !mbar_wait(smem_u32(&sm.s_free[sb]), ((gb / kSBuf) - 1) & 1, abortf, kBudgetNs)) {
                     dead = true;
                     break;
                 }
-                if (!mbar_wait(smem_u32(&sm.k_full[slot]), (gb / kStages) & 1, abortf, kBudgetNs)) {
+                if (!mbar_wait(smem_u32(&sm.k_full[slot]), (gb / kKStages) & 1, abortf, kBudgetNs)) {
                     dead = true;
                     break;
                 }
@@ -468,20 +481,20 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             mma_commit(smem_u32(&sm.drain[0]));
             wait_raw(smem_u32(&sm.drain[0]), 0);
         }
-    } else if (warp == 11) {
+    } else if (warp == 3) {
         // ------------------------------------------------------------ PV issuer
-        // O += P_t V_t once the softmax has written P_t and V_t has landed; PVs of a pipeline
-        // are issued by this one thread, so they accumulate into O in order.
+        // O += P_t V_t once the softmax has written P_t to shared memory and V_t has landed;
+        // PVs of a pipeline are issued by this one thread, so they accumulate into O in order.
         const bool leader = elect_one_sync();
         uint32_t gblk = 0, nloc = 0;
         const uint32_t vbase = smem_u32(&sm.v[0][0]);
         const int npieces = sm.nA + sm.nB;
-        for (int k = 0; !dead && k < npieces; ++k, ++nloc) {
-            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+        for (int pi = 0; !dead && pi < npieces; ++pi, ++nloc) {
+            const Piece pc = get_piece(p, sm, pi, vcta, vgrid);
             const int nblk = pc.nb;
             for (int t = 0; t < nblk; ++t) {
-                const uint32_t gb = gblk + t, sb = gb % kSBuf, slot = gb % kStages;
-                if (!mbar_wait(smem_u32(&sm.p_full[sb]), (gb / kSBuf) & 1, abortf, kBudgetNs)) {
+                const uint32_t gb = gblk + t, pb = gb % kPBuf, slot = gb % kVStages;
+                if (!mbar_wait(smem_u32(&sm.p_full[pb]), (gb / kPBuf) & 1, abortf, kBudgetNs)) {
                     dead = true;
                     break;
                 }
@@ -490,20 +503,20 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     dead = true;
                     break;
                 }
-                if (!mbar_wait(smem_u32(&sm.v_full[slot]), (gb / kStages) & 1, abortf, kBudgetNs)) {
+                if (!mbar_wait(smem_u32(&sm.v_full[slot]), (gb / kVStages) & 1, abortf, kBudgetNs)) {
                     dead = true;
                     break;
                 }
                 tc_fence_after();
                 if (leader) {
                     const uint64_t vdesc = sdesc_sw128(vbase + slot * kTileBytes, 8192, 1024);
-                    const uint32_t pcol = tbase + kColS + sb * 64;
+                    const uint32_t pcol = tbase + kColP + pb * 32;
 #pragma unroll
                     for (int k = 0; k < 4; ++k)
                         mma_ts(tbase + kColO, pcol + k * 8, vdesc + (uint64_t)(k * 128), kIdescPV,
                                (t > 0 || k > 0) ? 1u : 0u);
                     mma_commit(smem_u32(&sm.v_empty[slot]));
-                    mma_commit(smem_u32(&sm.pv_done[sb]));
+                    mma_commit(smem_u32(&sm.p_empty[pb]));
                 }
                 __syncwarp();
             }
@@ -522,7 +535,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             mma_commit(smem_u32(&sm.drain[1]));
             wait_raw(smem_u32(&sm.drain[1]), 0);
         }
-    } else if (warp < 6) {
+    } else if (warp >= 4 && warp < 8) {
         // ------------------------------------------------------------ softmax
         const int quad = gwarp & 3;  // TMEM lane quadrant of this warp
         const int half = lane >> 4;
@@ -531,8 +544,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         const float c = p.scale_log2;
         uint32_t gblk = 0, nloc = 0;
         const int npieces = sm.nA + sm.nB;
-        for (int k = 0; !dead && k < npieces; ++k, ++nloc) {
-            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+        for (int pi = 0; !dead && pi < npieces; ++pi, ++nloc) {
+            const Piece pc = get_piece(p, sm, pi, vcta, vgrid);
             const int nblk = pc.nb;
             float m_used = 0.f, l = 0.f;
             for (int t = 0; t < nblk; ++t) {
@@ -547,6 +560,10 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 tmem_ld_16x32bx2_x16_off32(scol, *reinterpret_cast<uint32_t(*)[16]>(&sr[0]));
                 tmem_ld_16x32bx2_x16_off32(scol + 16, *reinterpret_cast<uint32_t(*)[16]>(&sr[16]));
                 tmem_wait_ld();
+                // S_t is in registers: QK_{t+2} may overwrite its buffer
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&sm.s_free[sb]));
                 float mx;
                 {
                     float t8[8];
@@ -560,34 +577,19 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 }
                 mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
                 const float mx2 = mx * c;
+                // lazy rescale: the running max is raised only when it grows by more than
+                // 2^kRescaleLog2; O is then rescaled below, after P_t is stored (so that O
+                // and S are never held in registers at the same time)
+                bool rescale = false;
+                float alpha = 1.f;
                 if (t == 0) {
                     m_used = mx2;
                 } else {
                     const bool need = mx2 > m_used + kRescaleLog2;
-                    if (__any_sync(0xffffffffu, need)) {
-                        // O must hold every earlier PV before it is rescaled
-                        const uint32_t pb = (gb - 1) % kSBuf;
-                        if (!mbar_wait(smem_u32(&sm.pv_done[pb]), ((gb - 1) / kSBuf) & 1, abortf, kBudgetNs)) {
-                            dead = true;
-                            break;
-                        }
-                        tc_fence_after();
-                        const float alpha = need ? fast_exp2(m_used - mx2) : 1.f;
-                        const uint32_t ocol = tbase + lane_off + kColO;
-                        uint32_t o[16];
-#pragma unroll
-                        for (int h2 = 0; h2 < 2; ++h2) {
-                            tmem_ld_16x32bx2_x16_off32(ocol + h2 * 16, o);
-                            tmem_wait_ld();
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                            tmem_st_16x32bx2_x16_off32(ocol + h2 * 16, o);
-                        }
-                        tmem_wait_st();
-                        if (need) {
-                            l *= alpha;
-                            m_used = mx2;
-                        }
+                    rescale = __any_sync(0xffffffffu, need);
+                    if (need) {
+                        alpha = fast_exp2(m_used - mx2);
+                        m_used = mx2;
                     }
                 }
                 // x = s * c - m and the row sums in packed fp32x2 arithmetic (two lanes per op)
@@ -603,12 +605,38 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     pk[i] = pack_bf16(pp.x, pp.y);
                 }
                 const float2 lsum = __fadd2_rn(ls2[0], ls2[1]);
-                l += lsum.x + lsum.y;
-                tmem_st_16x32bx2_x16_off16(tbase + lane_off + kColS + sb * 64, pk);
+                l = fmaf(l, alpha, lsum.x + lsum.y);
+                // P_t (bf16 pairs) into its TMEM buffer once PV_{t-2} has finished reading it
+                const uint32_t pb = gb % kPBuf;
+                if (gb >= (uint32_t)kPBuf &&
+                    !mbar_wait(smem_u32(&sm.p_empty[pb]), ((gb / kPBuf) - 1) & 1, abortf, kBudgetNs)) {
+                    dead = true;
+                    break;
+                }
+                tmem_st_16x32bx2_x16_off16(tbase + lane_off + kColP + pb * 32, pk);
+                if (rescale) {
+                    // O must hold every earlier PV before it is rescaled; PV_t waits for p_full
+                    const uint32_t qb = (gb - 1) % kPBuf;
+                    if (!mbar_wait(smem_u32(&sm.p_empty[qb]), ((gb - 1) / kPBuf) & 1, abortf, kBudgetNs)) {
+                        dead = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t ocol = tbase + lane_off + kColO;
+                    uint32_t o[16];
+#pragma unroll
+                    for (int h2 = 0; h2 < 2; ++h2) {
+                        tmem_ld_16x32bx2_x16_off32(ocol + h2 * 16, o);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                        tmem_st_16x32bx2_x16_off32(ocol + h2 * 16, o);
+                    }
+                }
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&sm.p_full[sb]));
+                if (lane == 0) mbar_arrive(smem_u32(&sm.p_full[pb]));
             }
             if (dead) break;
             // hand the row statistics to the epilogue warps
@@ -631,8 +659,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
         uint32_t nloc = 0;
         const int npieces = sm.nA + sm.nB;
-        for (int k = 0; !dead && k < npieces; ++k, ++nloc) {
-            const Piece pc = get_piece(p, sm, k, vcta, vgrid);
+        for (int pi = 0; !dead && pi < npieces; ++pi, ++nloc) {
+            const Piece pc = get_piece(p, sm, pi, vcta, vgrid);
             const int bh = pc.item / Tb, label = pc.item - bh * Tb;
             const uint32_t eb = nloc & 1;
             if (!mbar_wait(smem_u32(&sm.o_full), nloc & 1, abortf, kBudgetNs)) {
@@ -846,7 +874,7 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
         // Equal shares of blocks only pay when some pipeline would otherwise take one item
         // more than another, and when items are long: a merge costs a few global-memory
         // round trips (about 5 us under load, measured), which 11-block items do not
-        // earn back but 64-block items (dense) do (173 vs 190 us at 1024 px, 24 heads).
+        // earn back but 64-block items (dense) do (179 vs 198 us at 1024 px, 24 heads).
         p.split = (keep >= kSplitMinKeep && p.num_items >= kSlots * grid && p.num_items % (kSlots * grid) != 0)
                       ? 1 : 0;
     }
