@@ -151,6 +151,8 @@ int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K, int32_t
     float* qb = static_cast<float*>(workspace);
     float* kb = reinterpret_cast<float*>(static_cast<char*>(workspace) + need / 2);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    rc = launch_mask_fused(*desc, g, keep, Q, K, kv_idx, kv_cnt, scores_opt, st);
+    if (rc != SSBA_ERR_UNSUPPORTED) return rc;
     rc = launch_pool(*desc, g, Q, K, qb, kb, st);
     if (rc != SSBA_OK) return rc;
     return launch_select(*desc, g, keep, qb, kb, kv_idx, kv_cnt, scores_opt, st);

@@ -40,6 +40,10 @@ int launch_pool(const ssba_desc& d, const Grid& g, const void* Q, const void* K,
                 cudaStream_t st);
 int launch_select(const ssba_desc& d, const Grid& g, int keep, const float* qb, const float* kb,
                   int32_t* idx, int32_t* cnt, float* scores, cudaStream_t st);
+// Pool + affinity + selection in one launch (head_dim 64, 8x8 blocks, Tb <= 256); returns
+// SSBA_ERR_UNSUPPORTED without launching for other shapes.
+int launch_mask_fused(const ssba_desc& d, const Grid& g, int keep, const void* Q, const void* K, int32_t* idx,
+                      int32_t* cnt, float* scores, cudaStream_t st);
 int launch_attn_simt_f32(const ssba_desc& d, const Grid& g, int keep, float scale, const float* Q,
                          const float* K, const float* V, const int32_t* idx, const int32_t* cnt, float* O,
                          float* lse, cudaStream_t st);

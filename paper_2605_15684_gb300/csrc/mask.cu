@@ -11,6 +11,12 @@
 //                       the total order (S descending, label ascending), i.e. the k_drop
 //                       smallest are dropped and ties keep the lower label; the kept labels
 //                       are written in ascending order.
+//   ssba_mask_fused_kernel  both steps in one launch for head_dim 64, 8x8 blocks and at
+//                       most 256 blocks: a cluster of 8 CTAs per (batch, head) pools its
+//                       blocks into shared memory, reads the head's k_b from the other CTAs
+//                       of the cluster (distributed shared memory), and selects its rows. No
+//                       q_b/k_b round trip through global memory and no second launch.
+#include <cooperative_groups.h>
 #include <cstdio>
 
 #include "common.cuh"
@@ -286,6 +292,148 @@ __global__ void __launch_bounds__(kSelWarps * 32) ssba_select_kernel(const float
     if (lane == 0) cnt[rowoff] = keep;
 }
 
+
+constexpr int kFuseCluster = 8;    // CTAs per (batch, head)
+constexpr int kFuseWarps = 8;
+constexpr int kFuseMaxTb = 256;
+
+// One cluster of kFuseCluster CTAs per (batch*head); CTA r of the cluster owns the blocks
+// [r * bpc, (r + 1) * bpc) ∩ [0, Tb).
+// smem: qown [bpc][64] | kown [bpc][64] | kbT [64][Tb + 1] | S keys [kFuseWarps][Tb]
+//   1. pool: warp w takes (block, tensor) units w, w + 8, ... of its CTA; lane l covers
+//      16-byte chunk l % CPR of rows l / CPR + RPI * i, summed in row order, then across
+//      lanes by shuffles (fixed order); the mean goes to qown / kown.
+//   2. cluster barrier; every CTA copies the head's k_b (transposed) from the owners'
+//      kown into its kbT; cluster barrier again (no CTA leaves while another reads it).
+//   3. one warp per owned query block: S row by four interleaved partial sums over d,
+//      then the exact rank selection of ssba_select_kernel.
+template <typename T>
+__global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const T* __restrict__ Q,
+                                                                          const T* __restrict__ K, Grid g,
+                                                                          int keep, int bpc,
+                                                                          int32_t* __restrict__ idx,
+                                                                          int32_t* __restrict__ cnt,
+                                                                          float* __restrict__ scores)
+{
+    namespace cg = cooperative_groups;
+    constexpr int kD = 64;
+    constexpr int VE = Vec<T>::kElems;
+    constexpr int CPR = kD / VE;      // 16-byte chunks per token row
+    constexpr int RPI = 32 / CPR;     // rows per warp instruction
+    constexpr int LOADS = 64 / RPI;   // loads per lane per (block, tensor)
+    constexpr int BATCH = LOADS < 16 ? LOADS : 16;  // loads in flight per lane
+    cg::cluster_group cluster = cg::this_cluster();
+    extern __shared__ float smf[];
+    const int Tb = g.Tb();
+    const int rank = (int)cluster.block_rank();
+    const int bh = blockIdx.y;
+    const int b0 = rank * bpc;
+    const int nb = max(0, min(bpc, Tb - b0));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int N = g.H * g.W;
+    float* qown = smf;
+    float* kown = qown + bpc * kD;
+    const int ld = Tb + 1;
+    float* kbT = kown + bpc * kD;
+    uint32_t* Skey = reinterpret_cast<uint32_t*>(kbT + kD * ld);
+
+    // 1. pool the owned blocks
+    const int col = lane % CPR, r0 = lane / CPR;
+    for (int u = warp; u < 2 * nb; u += kFuseWarps) {
+        const int which = u & 1, k = u >> 1, label = b0 + k;
+        const T* X = (which ? K : Q) + (size_t)bh * N * kD + col * VE;
+        // window origin in the rolled frame, once per unit; rows and columns of the 8x8
+        // window then follow by shifts (the same map as Grid::token with blk = 8)
+        const int br = label / g.bw, bc = label - br * g.bw;
+        const int rb = br * 8 - g.sr, cb = bc * 8 - g.sc;
+        float acc[VE];
+#pragma unroll
+        for (int e = 0; e < VE; ++e) acc[e] = 0.f;
+#pragma unroll
+        for (int i0 = 0; i0 < LOADS; i0 += BATCH) {
+            uint4 v[BATCH];
+#pragma unroll
+            for (int i = 0; i < BATCH; ++i) {
+                const int pos = r0 + (i0 + i) * RPI;
+                int r = rb + (pos >> 3), c = cb + (pos & 7);
+                r += r < 0 ? g.H : 0;
+                c += c < 0 ? g.W : 0;
+                v[i] = __ldg(reinterpret_cast<const uint4*>(X + (size_t)(r * g.W + c) * kD));
+            }
+#pragma unroll
+            for (int i = 0; i < BATCH; ++i) {
+                float f[VE];
+                Vec<T>::to_f32(v[i], f);
+#pragma unroll
+                for (int e = 0; e < VE; ++e) acc[e] += f[e];
+            }
+        }
+#pragma unroll
+        for (int o = CPR; o < 32; o <<= 1)
+#pragma unroll
+            for (int e = 0; e < VE; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+        if (r0 == 0) {
+            float* dst = (which ? kown : qown) + k * kD + col * VE;
+#pragma unroll
+            for (int e = 0; e < VE; ++e) dst[e] = acc[e] * (1.0f / 64.0f);
+        }
+    }
+    cluster.sync();
+
+    // 2. gather the head's k_b, transposed: kbT[c][j] = k_b[j][c] (four remote loads in
+    //    flight per thread and round)
+    constexpr int kG = 4;
+    for (int base = 0; base < Tb * (kD / 4); base += kG * kFuseWarps * 32) {
+        float4 v[kG];
+#pragma unroll
+        for (int r = 0; r < kG; ++r) {
+            const int e4 = base + r * kFuseWarps * 32 + threadIdx.x;
+            if (e4 < Tb * (kD / 4)) {
+                const int j = e4 / (kD / 4), c = (e4 - j * (kD / 4)) * 4;
+                const int owner = j / bpc, jl = j - owner * bpc;
+                v[r] = *reinterpret_cast<const float4*>(cluster.map_shared_rank(kown, owner) + jl * kD + c);
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < kG; ++r) {
+            const int e4 = base + r * kFuseWarps * 32 + threadIdx.x;
+            if (e4 < Tb * (kD / 4)) {
+                const int j = e4 / (kD / 4), c = (e4 - j * (kD / 4)) * 4;
+                kbT[(c + 0) * ld + j] = v[r].x;
+                kbT[(c + 1) * ld + j] = v[r].y;
+                kbT[(c + 2) * ld + j] = v[r].z;
+                kbT[(c + 3) * ld + j] = v[r].w;
+            }
+        }
+    }
+    cluster.sync();
+
+    // 3. affinity rows and selection
+    uint32_t* S = Skey + (size_t)warp * Tb;
+    for (int k = warp; k < nb; k += kFuseWarps) {
+        const size_t rowoff = (size_t)bh * Tb + b0 + k;
+        const float* q = qown + k * kD;
+        for (int j = lane; j < Tb; j += 32) {
+            float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int c = 0; c < kD; c += 4)
+#pragma unroll
+                for (int u = 0; u < 4; ++u) a[u] = fmaf(q[c + u], kbT[(c + u) * ld + j], a[u]);
+            const float acc = (a[0] + a[1]) + (a[2] + a[3]);
+            if (scores) scores[rowoff * Tb + j] = acc;
+            S[j] = order_key(acc);
+        }
+        __syncwarp();
+        int32_t* dst = idx + rowoff * keep;
+        if (Tb <= 32) rank_select<1>(S, Tb, keep, lane, dst);
+        else if (Tb <= 64) rank_select<2>(S, Tb, keep, lane, dst);
+        else if (Tb <= 128) rank_select<4>(S, Tb, keep, lane, dst);
+        else rank_select<8>(S, Tb, keep, lane, dst);
+        if (lane == 0) cnt[rowoff] = keep;
+        __syncwarp();
+    }
+}
+
 }  // namespace
 
 int launch_pool(const ssba_desc& d, const Grid& g, const void* Q, const void* K, float* qb, float* kb,
@@ -352,6 +500,50 @@ int launch_select(const ssba_desc& d, const Grid& g, int keep, const float* qb, 
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
         set_error("ssba_select_kernel launch: %s", cudaGetErrorString(e));
+        return SSBA_ERR_CUDA;
+    }
+    return SSBA_OK;
+}
+
+}  // namespace ssba
+
+namespace ssba {
+
+// The fused mask build (one launch) when the shape allows it; returns SSBA_ERR_UNSUPPORTED
+// (without launching and without setting an error) otherwise.
+int launch_mask_fused(const ssba_desc& d, const Grid& g, int keep, const void* Q, const void* K, int32_t* idx,
+                      int32_t* cnt, float* scores, cudaStream_t st)
+{
+    const int Tb = g.Tb();
+    if (d.head_dim != 64 || g.blk != 8 || Tb > kFuseMaxTb) return SSBA_ERR_UNSUPPORTED;
+    const int bpc = (Tb + kFuseCluster - 1) / kFuseCluster;
+    const size_t smem = ((size_t)2 * bpc * 64 + (size_t)64 * (Tb + 1) + (size_t)kFuseWarps * Tb) * sizeof(float);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kFuseCluster, d.B * d.heads, 1);
+    cfg.blockDim = dim3(kFuseWarps * 32, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kFuseCluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e;
+    if (d.dtype == SSBA_BF16) {
+        auto k = ssba_mask_fused_kernel<__nv_bfloat16>;
+        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        e = cudaLaunchKernelEx(&cfg, k, static_cast<const __nv_bfloat16*>(Q), static_cast<const __nv_bfloat16*>(K),
+                               g, keep, bpc, idx, cnt, scores);
+    } else {
+        auto k = ssba_mask_fused_kernel<float>;
+        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        e = cudaLaunchKernelEx(&cfg, k, static_cast<const float*>(Q), static_cast<const float*>(K), g, keep, bpc, idx,
+                               cnt, scores);
+    }
+    if (e != cudaSuccess) {
+        set_error("ssba_mask_fused_kernel launch: %s", cudaGetErrorString(e));
         return SSBA_ERR_CUDA;
     }
     return SSBA_OK;

@@ -58,6 +58,22 @@ def test_mask_full_configs(H, W, B, rho, shift):
     assert near < 0.1 * B * 24 * (H * W // 64)
 
 
+@pytest.mark.parametrize("d,H,W,dtype", [(32, 32, 32, torch.bfloat16), (128, 32, 32, torch.float32),
+                                         (64, 136, 136, torch.bfloat16)])
+def test_mask_two_kernel_path(d, H, W, dtype):
+    """Shapes outside the fused one-launch build (head_dim 64, at most 256 blocks) go
+    through the separate pooling and selection kernels: other head widths, and 289
+    blocks (radix selection)."""
+    q, k, _ = synthetic.qkv(1, 2, H * W, d, dtype, 7)
+    desc = api.SsbaDesc(1, 2, H, W, head_dim=d, shift_r=4, shift_c=4, rho=0.8, dtype=dtype)
+    idx, cnt, S = api.build_mask(desc, q.cuda(), k.cuda(), scores=True)
+    torch.cuda.synchronize()
+    idx_o, cnt_o, S_o = oracle.build_mask(q, k, H, W, 8, (4, 4), 0.8, return_scores=True)
+    keep = oracle.keep_count(H * W // 64, 0.8)
+    near = check_mask(idx.cpu().numpy(), cnt.cpu().numpy(), S.cpu().numpy(), S_o, idx_o, keep)
+    assert near < 0.1 * 2 * (H * W // 64)
+
+
 def test_mask_ties_keep_lower_label():
     """Constant Q/K make every S entry equal: each row keeps labels 0..keep-1."""
     H = W = 32
