@@ -57,6 +57,28 @@ def layer_shift(l: int):
     return (0, 0) if l % 2 == 0 else (4, 4)
 
 
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """The largest x over all ranks (the slowest rank's time); x itself on one rank."""
+    if world <= 1:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_tflops(world: int, flops_per_rank: float, seconds: float) -> float:
+    """Whole-job rate: every rank does flops_per_rank of independent work; the job takes
+    as long as its slowest rank (seconds)."""
+    return world * flops_per_rank / seconds / 1e12
+
+
+def mask_launches(head_dim: int, Tb: int, blk: int = 8) -> int:
+    """Kernels one ssba_build_mask call launches: the fused build (head_dim 64, 8x8 blocks,
+    at most 256 blocks) is one, the pooling + selection pair is two."""
+    return 1 if (head_dim == 64 and blk == 8 and Tb <= 256) else 2
+
+
 def kept_flops(B, h, Tb, keep, d, blk=8):
     """QK^T plus PV over the kept blocks only (2 * 2 * rows * keys * d)."""
     return 4.0 * B * h * Tb * keep * (blk * blk) * (blk * blk) * d
@@ -289,10 +311,7 @@ def run_ours(args, rank, world):
     time.sleep(0.1)
     clocks.stop()
     ms_total = t_start.elapsed_time(t_end)
-    if world > 1:
-        tt = torch.tensor([ms_total], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(ms_total, world, dev)
     ms_step = ms_total / K
     mask_ms = statistics.mean(evs[s][0][l].elapsed_time(evs[s][1][l]) for s in range(K) for l in range(L))
     attn_ms = statistics.mean(evs[s][1][l].elapsed_time(evs[s][2][l]) for s in range(K) for l in range(L))
@@ -301,7 +320,7 @@ def run_ours(args, rank, world):
         raise RuntimeError(f"device status {int(st[0])} after the timed region")
 
     F_layer = kept_flops(w.B, w.heads, Tb, keep, w.head_dim)
-    value = world * L * F_layer / (ms_step * 1e-3) / 1e12
+    value = whole_job_tflops(world, L * F_layer, ms_step * 1e-3)
 
     # ---- roofline of the dominant kernel (the attention kernel)
     hbm_gbs, bf16_tflops, peak_src = measured_peaks()
@@ -380,13 +399,10 @@ def run_ours(args, rank, world):
             e2e_step()
         torch.cuda.synchronize()
         e2e_s = (time.perf_counter() - t0) / args.e2e_steps
-        if world > 1:
-            tt = torch.tensor([e2e_s], device=dev)
-            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-            e2e_s = float(tt.item())
+        e2e_s = max_over_ranks(e2e_s, world, dev)
         h2d = L * 3 * w.B * w.heads * w.N * w.head_dim * 2
         d2h = L * (w.B * w.heads * w.N * w.head_dim * 2 + w.B * w.heads * w.N * 4)
-        e2e = {"value": world * L * F_layer / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+        e2e = {"value": whole_job_tflops(world, L * F_layer, e2e_s), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "steps": args.e2e_steps,
                "how": "pinned host Q/K/V -> device on a copy stream, mask + forward, O and lse -> "
                       "pinned host on a second copy stream; host wall clock around the steps"}
@@ -414,7 +430,7 @@ def run_ours(args, rank, world):
             "speedup_vs_dense": (dense_ms / attn_ms) if isinstance(dense_ms, float) else None,
             "ideal_speedup_vs_dense": Tb / keep,
             "e2e": e2e, "cpu_baseline": cpu,
-            "gpu_launches": K * L * 3,
+            "gpu_launches": K * L * (mask_launches(w.head_dim, Tb) + 1),
             "clocks": clocks.summary(wall0, wall1),
         }
         print(json.dumps(line), flush=True)

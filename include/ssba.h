@@ -175,6 +175,18 @@ SSBA_API int ssba_build_mask_noalloc(const ssba_desc* desc, const void* Q, const
                                      int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt,
                                      void* stream);
 
+/* Test hook for failure detection (the paper has no counterpart): runs the bf16 forward
+ * of ssba_forward with every barrier wait limited to budget_ns of wall time (clamped to
+ * [1 ms, 2 s]) and one K tile copy of the first pipeline announced but never issued, so
+ * that the waits on it run out. The kernel then stops all its roles, waits (bounded) for
+ * its own copies and MMAs in flight, frees its tensor memory and returns; the device
+ * status word reads SSBA_ERR_TIMEOUT (ssba_get_status, after a synchronize), O and lse
+ * are undefined, and the context stays usable. No fault, trap or endless wait is
+ * involved. Arguments as ssba_forward (workspace NULL); bf16 only. */
+SSBA_API int ssba_test_forward_timeout(const ssba_desc* desc, const void* Q, const void* K, const void* V,
+                                       const int32_t* kv_idx, const int32_t* kv_cnt, void* O, float* lse,
+                                       uint64_t budget_ns, void* stream);
+
 /* Reads and clears the device status word of the current device (SSBA_OK or
  * SSBA_ERR_TIMEOUT). Synchronous: call after the caller's stream sync. Returns
  * SSBA_OK, or SSBA_ERR_CUDA if the read failed. */

@@ -27,8 +27,8 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
                  4: "SSBA_ERR_TIMEOUT", 5: "SSBA_ERR_WORKSPACE"}
 
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
-            "ssba_forward", "ssba_forward_workspace_bytes", "ssba_forward_dense", "ssba_get_status",
-            "ssba_last_error")
+            "ssba_forward", "ssba_forward_workspace_bytes", "ssba_forward_dense", "ssba_test_forward_timeout",
+            "ssba_get_status", "ssba_last_error")
 
 
 class SsbaError(RuntimeError):
@@ -107,6 +107,8 @@ def load_library():
         lib.ssba_forward_workspace_bytes.restype = ctypes.c_size_t
         lib.ssba_forward_dense.argtypes = [DP, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_forward_dense.restype = ctypes.c_int
+        lib.ssba_test_forward_timeout.argtypes = [DP, P, P, P, P, P, P, P, ctypes.c_uint64, P]
+        lib.ssba_test_forward_timeout.restype = ctypes.c_int
         lib.ssba_get_status.argtypes = [ctypes.POINTER(ctypes.c_int32)]
         lib.ssba_get_status.restype = ctypes.c_int
         lib.ssba_last_error.argtypes = []
@@ -301,6 +303,25 @@ def forward_dense(desc: SsbaDesc, Q, K, V, O=None, lse=None, workspace="default"
                                 lse.data_ptr(), wp, wn, _stream_ptr(stream))
     _raise_on(rc)
     return O, lse
+
+
+def test_forward_timeout(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O, lse, budget_ns: int = 2_000_000,
+                         stream=None) -> None:
+    """ssba_test_forward_timeout: the failure-detection test hook (see include/ssba.h)."""
+    lib = load_library()
+    d = desc.c()
+    keep = lib.ssba_keep_count(ctypes.byref(d))
+    if keep < 0:
+        _raise_on(SSBA_ERR_INVALID)
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V"), (O, "O")):
+        _check(t, n, shp, desc.dtype)
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    _check(lse, "lse", shp[:3], torch.float32)
+    _raise_on(lib.ssba_test_forward_timeout(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(),
+                                            kv_idx.data_ptr(), kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(),
+                                            int(budget_ns), _stream_ptr(stream)))
 
 
 def get_status() -> int:

@@ -223,6 +223,32 @@ int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, cons
                                 static_cast<cudaStream_t>(stream));
 }
 
+int ssba_test_forward_timeout(const ssba_desc* desc, const void* Q, const void* K, const void* V,
+                              const int32_t* kv_idx, const int32_t* kv_cnt, void* O, float* lse, uint64_t budget_ns,
+                              void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_test_forward_timeout", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !V || !kv_idx || !kv_cnt || !O || !lse) {
+        set_error("ssba_test_forward_timeout: every pointer must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(lse, 4) ||
+        !aligned(kv_idx, 4) || !aligned(kv_cnt, 4)) {
+        set_error("ssba_test_forward_timeout: Q, K, V, O must be 16-byte aligned; lse, kv_idx, kv_cnt 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    if (desc->dtype != SSBA_BF16) {
+        set_error("ssba_test_forward_timeout: bf16 only");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    const uint64_t b = budget_ns < 1000000ull ? 1000000ull : (budget_ns > kWaitBudgetNs ? kWaitBudgetNs : budget_ns);
+    return launch_attn_tc_bf16(*desc, g, keep, resolve_scale(desc), Q, K, V, kv_idx, kv_cnt, O, lse, nullptr, 0,
+                               static_cast<cudaStream_t>(stream), b, 1);
+}
+
 int ssba_get_status(int32_t* device_status_out)
 {
     if (!device_status_out) {

@@ -47,9 +47,13 @@ int launch_mask_fused(const ssba_desc& d, const Grid& g, int keep, const void* Q
 int launch_attn_simt_f32(const ssba_desc& d, const Grid& g, int keep, float scale, const float* Q,
                          const float* K, const float* V, const int32_t* idx, const int32_t* cnt, float* O,
                          float* lse, cudaStream_t st);
+// budget_ns: wall-time limit of each barrier wait (a wait that runs out sets the device
+// status to SSBA_ERR_TIMEOUT); withhold != 0 is the failure-detection test hook.
+constexpr uint64_t kWaitBudgetNs = 2000000000ull;  // 2 s
 int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q,
                         const void* K, const void* V, const int32_t* idx, const int32_t* cnt, void* O,
-                        float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
+                        float* lse, void* ws, size_t ws_bytes, cudaStream_t st,
+                        uint64_t budget_ns = kWaitBudgetNs, int withhold = 0);
 int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V,
                          void* O, float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
 // Bytes of the split-merge workspace of the bf16 forward on the current device.
