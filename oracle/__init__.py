@@ -68,6 +68,12 @@ def _load():
                                                 _F64P, _F64P]
         lib.ssba_oracle_dense_all.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, c_int, c_double,
                                               _F64P, _F64P]
+        vp = ctypes.c_void_p
+        lib.ssba_oracle_attention_joint.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, vp, vp, c_int, _I32P,
+                                                    c_int, _I32P, c_int, c_double, _F64P, _F64P]
+        lib.ssba_oracle_forward_joint_all.argtypes = [_F64P, _F64P, _F64P, vp, vp, c_int, c_int, c_int, c_int,
+                                                      c_int, c_int, c_int, c_int, _I32P, c_int, c_double,
+                                                      _F64P, _F64P]
         lib.ssba_oracle_set_threads.argtypes = [c_int]
         lib.ssba_oracle_set_threads.restype = None
         _lib = lib
@@ -205,6 +211,45 @@ def forward(Q, K, V, idx, H: int, W: int, blk: int = 8, shift=(0, 0), scale=None
     lse = np.empty((B, h, N), dtype=np.float64)
     _check(_load().ssba_oracle_forward_all(Q, K, V, B * h, H, W, d, blk, int(shift[0]),
                                            int(shift[1]), idx, keep, scale, O, lse), "forward")
+    return O, lse
+
+
+def attention_joint(Q, K, V, Kt, Vt, block_of, idx, scale=None):
+    """Single-slice joint text + image attention (Algorithm 1 with its text segment):
+    Q, K, V [N, d] image tokens, Kt, Vt [Tt, d] text tokens; returns the image rows
+    (O [N, d], lse [N])."""
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    N, d = Q.shape
+    Kt, Vt = _f64(Kt).reshape(-1, d), _f64(Vt).reshape(-1, d)
+    Tt = Kt.shape[0]
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    Tb, keep = idx.shape
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    O = np.empty((N, d), dtype=np.float64)
+    lse = np.empty(N, dtype=np.float64)
+    _check(_load().ssba_oracle_attention_joint(Q, K, V, N, d, Kt.ctypes.data if Tt else None,
+                                               Vt.ctypes.data if Tt else None, Tt,
+                                               np.ascontiguousarray(block_of, np.int32), Tb, idx, keep, scale,
+                                               O, lse), "attention_joint")
+    return O, lse
+
+
+def forward_joint(Q, K, V, Kt, Vt, idx, H: int, W: int, blk: int = 8, shift=(0, 0), scale=None):
+    """Whole-tensor joint forward. Q, K, V: [B, heads, N, d]; Kt, Vt: [B, heads, Tt, d];
+    idx [B, heads, Tb, keep]. Returns the image rows (O [B, heads, N, d], lse)."""
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    Kt, Vt = _f64(Kt), _f64(Vt)
+    B, h, N, d = Q.shape
+    Tt = Kt.shape[2]
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    keep = idx.shape[-1]
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    O = np.empty((B, h, N, d), dtype=np.float64)
+    lse = np.empty((B, h, N), dtype=np.float64)
+    _check(_load().ssba_oracle_forward_joint_all(Q, K, V, Kt.ctypes.data if Tt else None,
+                                                 Vt.ctypes.data if Tt else None, Tt, B * h, H, W, d, blk,
+                                                 int(shift[0]), int(shift[1]), idx, keep, scale, O, lse),
+           "forward_joint")
     return O, lse
 
 

@@ -26,7 +26,9 @@
  *   - Softmax scale is 1/sqrt(d) unless given; lse is a natural log of the sum of
  *     exp(scaled score).
  *   - Inputs are taken as post-RoPE (Algorithm 1 applies RoPE before pooling).
- *   - Only image tokens: the text-token padding of M is not part of this path.
+ *   - Text tokens (the _joint functions): the padded mask makes every text key visible to
+ *     every image query; text queries are not evaluated, because Algorithm 1 returns
+ *     the image rows O[T_txt:] only.
  *
  * Pins (tests/test_oracle_*.py): closed forms, brute force over block pairs,
  * brute-force subset search for the gate, np.roll for the partition, and the
@@ -252,6 +254,78 @@ int ssba_oracle_attention_rows(const double *Q, const double *K, const double *V
     return rc;
 }
 
+/* Joint text + image attention of one image query n (Algorithm 1: the token mask is
+ * padded with ones for the T_txt text tokens, Q, K, V are the concatenations [text;
+ * image], and SparseAttention runs on the whole sequence). The keys of image query n are
+ * all Tt text keys (the padded columns) followed by the image keys of the kept blocks of
+ * block_of[n]; scores, max, lse and the weighted sum of values are formed over that one
+ * list exactly as in attend_row. */
+static int attend_row_joint(const double *Q, const double *K, const double *V, int d, int n,
+                            const double *Kt, const double *Vt, int Tt,
+                            const int32_t *block_of, int Tb, const int32_t *idx, int keep,
+                            double scale, const int *start, const int *tok, double *a, int *am,
+                            double *O_row, double *lse_n)
+{
+    const int32_t *kept = idx + (size_t)block_of[n] * keep;
+    int na = 0;
+    for (int m = 0; m < Tt; ++m) {
+        double dot = 0.0;
+        for (int c = 0; c < d; ++c) dot += Q[(size_t)n * d + c] * Kt[(size_t)m * d + c];
+        a[na] = scale * dot;
+        am[na] = -1 - m;  /* text key m */
+        na++;
+    }
+    for (int t = 0; t < keep; ++t) {
+        int j = kept[t];
+        if (j < 0 || j >= Tb) return ORC_BAD;
+        for (int u = start[j]; u < start[j + 1]; ++u) {
+            int m = tok[u];
+            double dot = 0.0;
+            for (int c = 0; c < d; ++c) dot += Q[(size_t)n * d + c] * K[(size_t)m * d + c];
+            a[na] = scale * dot;
+            am[na] = m;
+            na++;
+        }
+    }
+    double mx = -INFINITY;
+    for (int u = 0; u < na; ++u) if (a[u] > mx) mx = a[u];
+    double sum = 0.0;
+    for (int u = 0; u < na; ++u) sum += exp(a[u] - mx);
+    double l = mx + log(sum);
+    *lse_n = l;
+    for (int c = 0; c < d; ++c) O_row[c] = 0.0;
+    for (int u = 0; u < na; ++u) {
+        double p = exp(a[u] - l);
+        const double *vm = am[u] >= 0 ? V + (size_t)am[u] * d : Vt + (size_t)(-1 - am[u]) * d;
+        for (int c = 0; c < d; ++c) O_row[c] += p * vm[c];
+    }
+    return ORC_OK;
+}
+
+/* Joint attention of one slice (Algorithm 1 with its text segment, returning the image
+ * rows O[T_txt:] only): Q, K, V [N][d] image tokens, Kt, Vt [Tt][d] text tokens.
+ * Text queries are not evaluated: Algorithm 1 returns the image features only, so
+ * their rows cannot affect the result. */
+int ssba_oracle_attention_joint(const double *Q, const double *K, const double *V, int N, int d,
+                                const double *Kt, const double *Vt, int Tt,
+                                const int32_t *block_of, int Tb, const int32_t *idx, int keep,
+                                double scale, double *O, double *lse)
+{
+    if (!Q || !K || !V || !block_of || !idx || !O || !lse) return ORC_BAD;
+    if (N <= 0 || d <= 0 || Tb <= 0 || keep <= 0 || keep > Tb || Tt < 0) return ORC_BAD;
+    if (Tt > 0 && (!Kt || !Vt)) return ORC_BAD;
+    int *start = (int *)malloc(sizeof(int) * ((size_t)Tb + 1));
+    int *tok = (int *)malloc(sizeof(int) * (size_t)N);
+    double *a = (double *)malloc(sizeof(double) * ((size_t)N + (size_t)Tt));
+    int *am = (int *)malloc(sizeof(int) * ((size_t)N + (size_t)Tt));
+    int rc = (start && tok && a && am) ? block_lists(N, block_of, Tb, start, tok) : ORC_BAD;
+    for (int n = 0; n < N && rc == ORC_OK; ++n)
+        rc = attend_row_joint(Q, K, V, d, n, Kt, Vt, Tt, block_of, Tb, idx, keep, scale, start, tok, a, am,
+                              O + (size_t)n * d, lse + n);
+    free(start); free(tok); free(a); free(am);
+    return rc;
+}
+
 /* Dense softmax attention over all N keys (Table 2 "baseline 0%" sparsity). */
 int ssba_oracle_dense_attention(const double *Q, const double *K, const double *V,
                                 int N, int d, double scale, double *O, double *lse)
@@ -341,6 +415,34 @@ int ssba_oracle_forward_all(const double *Q, const double *K, const double *V, i
         bad |= ssba_oracle_attention(Q + off, K + off, V + off, N, d, block_of, Tb,
                                      idx + (size_t)s * Tb * keep, keep, scale,
                                      O + off, lse + (size_t)s * N);
+    }
+    free(block_of);
+    return bad ? ORC_BAD : ORC_OK;
+}
+
+int ssba_oracle_forward_joint_all(const double *Q, const double *K, const double *V,
+                                  const double *Kt, const double *Vt, int Tt, int BH,
+                                  int H, int W, int d, int blk, int shift_r, int shift_c,
+                                  const int32_t *idx, int keep, double scale,
+                                  double *O, double *lse)
+{
+    if (!Q || !K || !V || !idx || !O || !lse || BH <= 0 || blk <= 0 || Tt < 0) return ORC_BAD;
+    if (H % blk || W % blk) return ORC_BAD;
+    int N = H * W, Tb = N / (blk * blk);
+    int32_t *block_of = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    if (!block_of) return ORC_BAD;
+    if (ssba_oracle_partition(H, W, blk, shift_r, shift_c, block_of) != ORC_OK) {
+        free(block_of);
+        return ORC_BAD;
+    }
+    int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(|:bad)
+    for (int s = 0; s < BH; ++s) {
+        size_t off = (size_t)s * N * d, toff = (size_t)s * Tt * d;
+        bad |= ssba_oracle_attention_joint(Q + off, K + off, V + off, N, d, Tt ? Kt + toff : NULL,
+                                           Tt ? Vt + toff : NULL, Tt, block_of, Tb,
+                                           idx + (size_t)s * Tb * keep, keep, scale, O + off,
+                                           lse + (size_t)s * N);
     }
     free(block_of);
     return bad ? ORC_BAD : ORC_OK;

@@ -310,3 +310,75 @@ def test_attention_rows_matches_numpy_on_sampled_rows():
     want_O, want_lse, _ = numpy_masked_softmax_attention(Q, K, V, allowed, 1 / 8.0)
     np.testing.assert_allclose(O, want_O[rows], rtol=1e-10, atol=1e-12)
     np.testing.assert_allclose(lse, want_lse[rows], rtol=1e-12, atol=1e-12)
+
+
+# ----------------------------------------------------------------------------- text segment
+def algorithm1_joint_literal(Qt, Kt, Vt, Q, K, V, block_of, idx, scale):
+    """Algorithm 1 written out densely: G from the kept lists, M_img = ExpandMask(G),
+    M = Pad(M_img, T_txt, axis=(0, 1)) with ones, Q, K, V = [text; image], masked softmax
+    attention over the whole sequence, return the image rows O[T_txt:] (and their lse)."""
+    Tt, N = Kt.shape[0], K.shape[0]
+    Tb = idx.shape[0]
+    G = np.zeros((Tb, Tb), dtype=bool)
+    for i in range(Tb):
+        G[i, idx[i]] = True
+    M_img = G[block_of][:, block_of]
+    M = np.ones((Tt + N, Tt + N), dtype=bool)
+    M[Tt:, Tt:] = M_img
+    Qa, Ka, Va = np.vstack([Qt, Q]), np.vstack([Kt, K]), np.vstack([Vt, V])
+    a = scale * (Qa @ Ka.T)
+    a = np.where(M, a, -np.inf)
+    mx = a.max(axis=1, keepdims=True)
+    e = np.exp(a - mx)
+    s = e.sum(axis=1, keepdims=True)
+    return (e / s @ Va)[Tt:], (mx + np.log(s))[Tt:, 0]
+
+
+@pytest.mark.parametrize("Tt,shift", [(5, (4, 4)), (13, (0, 0)), (1, (3, -5))])
+def test_joint_attention_is_algorithm1_with_padded_mask(Tt, shift):
+    rng = np.random.default_rng(40 + Tt)
+    H = W = 16
+    N, d = H * W, 8
+    Q, K, V = (rng.standard_normal((N, d)) for _ in range(3))
+    Qt, Kt, Vt = (rng.standard_normal((Tt, d)) for _ in range(3))
+    lab = oracle.partition(H, W, 8, shift)
+    idx = np.array([[0, 3], [1, 2], [0, 2], [1, 3]], dtype=np.int32)
+    O, lse = oracle.attention_joint(Q, K, V, Kt, Vt, lab, idx)
+    O_ref, lse_ref = algorithm1_joint_literal(Qt, Kt, Vt, Q, K, V, lab, idx, 1 / np.sqrt(d))
+    np.testing.assert_allclose(O, O_ref, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lse, lse_ref, rtol=0, atol=1e-12)
+    # the text queries do not reach the image rows Algorithm 1 returns
+    O2, _ = algorithm1_joint_literal(Qt + 3.0, Kt, Vt, Q, K, V, lab, idx, 1 / np.sqrt(d))
+    np.testing.assert_allclose(O2, O_ref, rtol=0, atol=0)
+
+
+def test_joint_attention_reductions():
+    rng = np.random.default_rng(7)
+    H = W = 16
+    N, d, Tt = H * W, 8, 9
+    Q, K, V = (rng.standard_normal((N, d)) for _ in range(3))
+    Kt, Vt = (rng.standard_normal((Tt, d)) for _ in range(2))
+    lab = oracle.partition(H, W, 8, (4, 4))
+    idx = np.array([[1, 2], [0, 3], [2, 3], [0, 1]], dtype=np.int32)
+    # no text tokens: the image-only attention
+    O0, l0 = oracle.attention_joint(Q, K, V, Kt[:0], Vt[:0], lab, idx)
+    Oi, li = oracle.attention(Q, K, V, lab, idx)
+    np.testing.assert_array_equal(O0, Oi)
+    np.testing.assert_array_equal(l0, li)
+    # every image block kept: dense softmax over the concatenated keys [text; image]
+    full = np.tile(np.arange(4, dtype=np.int32), (4, 1))
+    Of, lf = oracle.attention_joint(Q, K, V, Kt, Vt, lab, full)
+    Od, ld, _ = numpy_masked_softmax_attention(Q, np.vstack([Kt, K]), np.vstack([Vt, V]),
+                                               np.ones((N, Tt + N), dtype=bool), 1 / np.sqrt(d))
+    np.testing.assert_allclose(Of, Od, atol=1e-12)
+    np.testing.assert_allclose(lf, ld, atol=1e-12)
+    # constant values: every output row is that constant (the weights sum to one)
+    c = rng.standard_normal(d)
+    Oc, _ = oracle.attention_joint(Q, K, np.tile(c, (N, 1)), Kt, np.tile(c, (Tt, 1)), lab, idx)
+    np.testing.assert_allclose(Oc, np.tile(c, (N, 1)), atol=1e-13)
+    # a text key far above every image score takes all the weight: O = its value
+    Kt2 = Kt.copy()
+    Q2 = np.tile(rng.standard_normal(d), (N, 1))
+    Kt2[4] = 40.0 * Q2[0]
+    Oh, _ = oracle.attention_joint(Q2, K, V, Kt2, Vt, lab, idx)
+    np.testing.assert_allclose(Oh, np.tile(Vt[4], (N, 1)), atol=1e-9)
