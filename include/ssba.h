@@ -135,6 +135,22 @@ SSBA_API int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, c
                  const int32_t* kv_idx, const int32_t* kv_cnt, void* O, float* lse,
                  void* workspace, size_t ws_bytes, void* stream);
 
+/* Joint text + image forward (Algorithm 1 with its text segment: the token mask is padded
+ * with ones for the T_txt text tokens, Q, K and V are the concatenations [text; image], and
+ * the image rows O[T_txt:] are returned). For every image query token n of block i:
+ * softmax over all T_txt text keys and the image keys of the blocks listed in
+ * kv_idx[b][h][i][0 .. kv_cnt-1]. Text queries are not evaluated, since Algorithm 1
+ * returns the image features only.
+ *   Q, K, V, kv_idx, kv_cnt, O, lse, workspace: as ssba_forward (image tokens only).
+ *   K_txt, V_txt  device, [B][heads][T_txt][head_dim] bf16, 16-byte aligned.
+ *   T_txt         number of text tokens, >= 0 (0 gives ssba_forward's result).
+ * bf16 only, with the shape limits of the bf16 ssba_forward; text keys are read in
+ * 64-token tiles, the last one masked past T_txt. */
+SSBA_API int ssba_forward_joint(const ssba_desc* desc, const void* Q, const void* K, const void* V,
+                                const void* K_txt, const void* V_txt, int32_t T_txt,
+                                const int32_t* kv_idx, const int32_t* kv_cnt, void* O, float* lse,
+                                void* workspace, size_t ws_bytes, void* stream);
+
 /* Bytes of the optional ssba_forward / ssba_forward_dense workspace for desc on the
  * current device (it scales with the device's SM count: about 10 MB on 152 SMs);
  * 0 for an fp32 or an invalid descriptor. Host only, no device work. */

@@ -27,7 +27,8 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
                  4: "SSBA_ERR_TIMEOUT", 5: "SSBA_ERR_WORKSPACE"}
 
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
-            "ssba_forward", "ssba_forward_workspace_bytes", "ssba_forward_dense", "ssba_test_forward_timeout",
+            "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
+            "ssba_test_forward_timeout",
             "ssba_get_status", "ssba_last_error")
 
 
@@ -103,6 +104,8 @@ def load_library():
         lib.ssba_build_mask_noalloc.restype = ctypes.c_int
         lib.ssba_forward.argtypes = [DP, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_forward.restype = ctypes.c_int
+        lib.ssba_forward_joint.argtypes = [DP, P, P, P, P, P, ctypes.c_int32, P, P, P, P, P, ctypes.c_size_t, P]
+        lib.ssba_forward_joint.restype = ctypes.c_int
         lib.ssba_forward_workspace_bytes.argtypes = [DP]
         lib.ssba_forward_workspace_bytes.restype = ctypes.c_size_t
         lib.ssba_forward_dense.argtypes = [DP, P, P, P, P, P, P, ctypes.c_size_t, P]
@@ -279,6 +282,42 @@ def forward(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O=None, lse=None, workspace
     wp, wn = _ws_args(workspace)
     rc = lib.ssba_forward(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), kv_idx.data_ptr(),
                           kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), wp, wn, _stream_ptr(stream))
+    _raise_on(rc)
+    return O, lse
+
+
+def forward_joint(desc: SsbaDesc, Q, K, V, K_txt, V_txt, kv_idx, kv_cnt, O=None, lse=None, workspace="default",
+                  stream=None):
+    """ssba_forward_joint: image rows of the joint [text; image] attention (Algorithm 1 with
+    its text segment). K_txt, V_txt: [B, heads, T_txt, d] bf16. Returns (O, lse) of the
+    image tokens."""
+    lib = load_library()
+    d = desc.c()
+    keep = lib.ssba_keep_count(ctypes.byref(d))
+    if keep < 0:
+        _raise_on(SSBA_ERR_INVALID)
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
+        _check(t, n, shp, desc.dtype)
+    T_txt = int(K_txt.shape[2]) if isinstance(K_txt, torch.Tensor) and K_txt.dim() == 4 else -1
+    tshp = (desc.B, desc.heads, max(T_txt, 0), desc.head_dim)
+    _check(K_txt, "K_txt", tshp, desc.dtype)
+    _check(V_txt, "V_txt", tshp, desc.dtype)
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    if O is None:
+        O = torch.empty(shp, dtype=desc.dtype, device=Q.device)
+    if lse is None:
+        lse = torch.empty(shp[:3], dtype=torch.float32, device=Q.device)
+    _check(O, "O", shp, desc.dtype)
+    _check(lse, "lse", shp[:3], torch.float32)
+    if isinstance(workspace, str):
+        workspace = default_forward_workspace(desc, Q.device) if desc.dtype == torch.bfloat16 else None
+    wp, wn = _ws_args(workspace)
+    rc = lib.ssba_forward_joint(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(),
+                                K_txt.data_ptr() if T_txt > 0 else None, V_txt.data_ptr() if T_txt > 0 else None,
+                                T_txt, kv_idx.data_ptr(), kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), wp, wn,
+                                _stream_ptr(stream))
     _raise_on(rc)
     return O, lse
 

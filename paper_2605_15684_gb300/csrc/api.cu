@@ -196,6 +196,33 @@ int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void
     return launch_attn_tc_bf16(*desc, g, keep, scale, Q, K, V, kv_idx, kv_cnt, O, lse, workspace, ws_bytes, st);
 }
 
+int ssba_forward_joint(const ssba_desc* desc, const void* Q, const void* K, const void* V, const void* K_txt,
+                       const void* V_txt, int32_t T_txt, const int32_t* kv_idx, const int32_t* kv_cnt, void* O,
+                       float* lse, void* workspace, size_t ws_bytes, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_forward_joint", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !V || !kv_idx || !kv_cnt || !O || !lse || T_txt < 0 || (T_txt > 0 && (!K_txt || !V_txt))) {
+        set_error("ssba_forward_joint: every pointer must be non-null (K_txt, V_txt when T_txt > 0) and T_txt >= 0");
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(lse, 4) ||
+        !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) || (T_txt > 0 && (!aligned(K_txt, 16) || !aligned(V_txt, 16))) ||
+        (workspace && !aligned(workspace, 16))) {
+        set_error("ssba_forward_joint: Q, K, V, K_txt, V_txt, O and the workspace must be 16-byte aligned; lse, "
+                  "kv_idx, kv_cnt 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    if (desc->dtype != SSBA_BF16) {
+        set_error("ssba_forward_joint: bf16 only");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    return launch_attn_tc_bf16(*desc, g, keep, resolve_scale(desc), Q, K, V, kv_idx, kv_cnt, O, lse, workspace,
+                               ws_bytes, static_cast<cudaStream_t>(stream), kWaitBudgetNs, 0, K_txt, V_txt, T_txt);
+}
+
 int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, const void* V, void* O, float* lse,
                        void* workspace, size_t ws_bytes, void* stream)
 {

@@ -41,6 +41,7 @@
 // word and the CTA drains its in-flight copies and MMAs before it exits.
 #include <cuda.h>
 #include <cstdio>
+#include <cstring>
 
 #include "common.cuh"
 #include "ptx.cuh"
@@ -110,9 +111,11 @@ struct __align__(1024) SmemLayout {
     int abort_flag;
 };
 
-// Four maps per tensor, one per box shape, over the [B*heads][H][W][d] bf16 view.
+// Four maps per tensor, one per box shape, over the [B*heads][H][W][d] bf16 view, and
+// the text keys and values as [B*heads][T_txt][d] (64-row boxes, zero fill past T_txt).
 struct TileMaps {
     CUtensorMap q[4], k[4], v[4];
+    CUtensorMap kt, vt;
 };
 
 struct TcParams {
@@ -121,7 +124,10 @@ struct TcParams {
     const int32_t* idx;  // null: dense mode, every block of the head
     const int32_t* cnt;
     Grid g;
-    int keep;
+    int keep;          // length of an index-list row
+    int ntxt;          // text key blocks visited first by every query block (ceil(T_txt / 64))
+    int t_txt;         // text tokens
+    int units;         // key blocks of a whole item: ntxt + keep
     int num_items;
     float scale_log2;  // softmax scale * log2(e)
     int* status;       // device status word
@@ -274,8 +280,8 @@ __device__ __forceinline__ Piece get_piece(const TcParams& p, const SlotSmem& sm
         pc.item = sm.M + v + r * V;
         pc.tb = 0;
         pc.part = -1;
-        pc.nb = p.keep;
-        if (p.idx) pc.nb = min(max(r < kCntCap ? sm.cnts[r] : __ldg(p.cnt + pc.item), 0), p.keep);
+        pc.nb = p.units;
+        if (p.idx) pc.nb = p.ntxt + min(max(r < kCntCap ? sm.cnts[r] : __ldg(p.cnt + pc.item), 0), p.keep);
     }
     return pc;
 }
@@ -292,21 +298,22 @@ __device__ void build_schedule(const TcParams& p, SlotSmem& sm, int v, int V, in
     if (t != 0) return;
     int nA = 0;
     if (M > 0) {
-        const long long u0 = (long long)M * p.keep * v / V, u1 = (long long)M * p.keep * (v + 1) / V;
-        const long long cut = u1 / p.keep * p.keep;  // start of the item holding unit u1 - 1
+        const int U = p.units;
+        const long long u0 = (long long)M * U * v / V, u1 = (long long)M * U * (v + 1) / V;
+        const long long cut = u1 / U * U;  // start of the item holding unit u1 - 1
         auto add = [&](long long a, long long b) {   // piece over units [a, b) of one item
-            const int item = (int)(a / p.keep);
-            const int tb = (int)(a - (long long)item * p.keep), te = (int)(b - (long long)item * p.keep);
-            const int n = p.idx ? min(max(__ldg(p.cnt + item), 0), p.keep) : p.keep;
-            sm.pieceA[nA++] = make_int4(item, tb, max(0, min(te, n) - tb), tb > 0 ? 1 : (te < p.keep ? 0 : -1));
+            const int item = (int)(a / U);
+            const int tb = (int)(a - (long long)item * U), te = (int)(b - (long long)item * U);
+            const int n = p.ntxt + (p.idx ? min(max(__ldg(p.cnt + item), 0), p.keep) : p.keep);
+            sm.pieceA[nA++] = make_int4(item, tb, max(0, min(te, n) - tb), tb > 0 ? 1 : (te < U ? 0 : -1));
         };
         long long uend = u1;
-        if (u1 % p.keep != 0 && cut > u0) {  // the cut last item goes first
+        if (u1 % U != 0 && cut > u0) {  // the cut last item goes first
             add(cut, u1);
             uend = cut;
         }
         for (long long u = u0; u < uend;) {
-            const long long next = min((u / p.keep + 1) * p.keep, uend);
+            const long long next = min((u / U + 1) * U, uend);
             add(u, next);
             u = next;
         }
@@ -392,12 +399,16 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             const Piece pc = get_piece(p, sm, pi, vcta, vgrid);
             const int bh = pc.item / Tb, label = pc.item - bh * Tb;
             const int nblk = pc.nb;
-            const int32_t* list = p.idx ? p.idx + (size_t)pc.item * p.keep + pc.tb : nullptr;
+            // item blocks [tb, tb + nblk): text blocks first (positions < ntxt), then the
+            // listed image blocks, list entry (position - ntxt)
+            const int ti0 = max(pc.tb, p.ntxt);
+            const int nimg = max(0, pc.tb + nblk - ti0);
+            const int32_t* list = p.idx ? p.idx + (size_t)pc.item * p.keep + (ti0 - p.ntxt) : nullptr;
             // all lanes fetch the piece's labels in one round; lane 0 then issues the copies
             // (measured: faster than prefetching them one piece ahead with cp.async)
             int32_t* lab = sm.labels[is_k ? 0 : 1];
             if (list)
-                for (int t = lane; t < nblk && t < kLabelCap; t += 32) lab[t] = __ldg(list + t);
+                for (int t = lane; t < nimg && t < kLabelCap; t += 32) lab[t] = __ldg(list + t);
             __syncwarp();
             if (lane == 0) {
                 if (is_k) {
@@ -408,9 +419,26 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                         window_boxes<false>(maps.q, smem_u32(&sm.q[qb][0]), smem_u32(&sm.q_full[qb]), p.g, label, bh);
                     }
                 }
-                for (int t = 0; t < nblk && !dead; ++t, ++g) {
-                    const int j = !list ? pc.tb + t : clamp_label(t < kLabelCap ? lab[t] : __ldg(list + t), Tb);
-                    const uint32_t nst = is_k ? kKStages : kVStages, slot = g % nst;
+                const uint32_t nst = is_k ? kKStages : kVStages;
+                // text blocks of the piece (positions below ntxt): rows [64 tt, 64 tt + 64) of
+                // the text keys / values, zero past T_txt
+                const int te_txt = min(pc.tb + nblk, p.ntxt);
+                for (int tt = pc.tb; tt < te_txt && !dead; ++tt, ++g) {
+                    const uint32_t slot = g % nst;
+                    uint64_t* empty = is_k ? &sm.k_empty[slot] : &sm.v_empty[slot];
+                    uint64_t* full = is_k ? &sm.k_full[slot] : &sm.v_full[slot];
+                    if (!mbar_wait(smem_u32(empty), ((g / nst) & 1) ^ 1, abortf, p.budget_ns)) {
+                        dead = true;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(smem_u32(full), kTileBytes);
+                    tma_load_3d(smem_u32(is_k ? &sm.k[slot][0] : &sm.v[slot][0]), is_k ? &maps.kt : &maps.vt,
+                                smem_u32(full), 0, tt * 64, bh);
+                }
+                // image blocks of the piece: list entries [ti0 - ntxt, ti0 - ntxt + nimg)
+                for (int t = 0; t < nimg && !dead; ++t, ++g) {
+                    const int j = !list ? ti0 - p.ntxt + t : clamp_label(t < kLabelCap ? lab[t] : __ldg(list + t), Tb);
+                    const uint32_t slot = g % nst;
                     uint64_t* empty = is_k ? &sm.k_empty[slot] : &sm.v_empty[slot];
                     uint64_t* full = is_k ? &sm.k_full[slot] : &sm.v_full[slot];
                     if (!mbar_wait(smem_u32(empty), ((g / nst) & 1) ^ 1, abortf, p.budget_ns)) {
@@ -568,6 +596,14 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 tmem_ld_16x32bx2_x16_off32(scol, *reinterpret_cast<uint32_t(*)[16]>(&sr[0]));
                 tmem_ld_16x32bx2_x16_off32(scol + 16, *reinterpret_cast<uint32_t(*)[16]>(&sr[16]));
                 tmem_wait_ld();
+                {
+                    // the last text block: its columns past T_txt are zero-filled keys, not keys
+                    const int tt = pc.tb + t, valid = p.t_txt - tt * 64;
+                    if (tt < p.ntxt && valid < 64)
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (half * 32 + i >= valid) sr[i] = __float_as_uint(-INFINITY);
+                }
                 // S_t is in registers: QK_{t+2} may overwrite its buffer
                 tc_fence_before();
                 __syncwarp();
@@ -796,6 +832,21 @@ bool encode_window_maps(CUtensorMap* m4, const void* base, int BH, int H, int W)
 }
 
 // SM count of the current device (1 when it cannot be read; not cached then).
+// [B*heads][T][d] bf16 as a 3-D map with 64-row boxes (128-byte swizzle); rows past T read
+// as zeros.
+bool encode_rows_map(CUtensorMap* m, const void* base, int BH, int T)
+{
+    EncodeTiledFn fn = get_encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)T, (cuuint64_t)BH};
+    cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)T * kD * 2};
+    cuuint32_t box[3] = {kD, 64, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int num_sms()
 {
     static int n = 0;
@@ -827,7 +878,8 @@ size_t attn_tc_workspace_bytes() { return ws_cnt_bytes() + ws_st_bytes() + ws_o_
 
 int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
                         const void* V, const int32_t* idx, const int32_t* cnt, void* O, float* lse, void* ws,
-                        size_t ws_bytes, cudaStream_t st, uint64_t budget_ns, int withhold)
+                        size_t ws_bytes, cudaStream_t st, uint64_t budget_ns, int withhold, const void* Kt,
+                        const void* Vt, int t_txt)
 {
     if (d.head_dim != kD || g.blk != 8 || (g.sr % 4) || (g.sc % 4)) {
         set_error("ssba_forward (bf16): needs head_dim=64, block=8 and shifts that are multiples of 4");
@@ -839,9 +891,14 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
     }
     const int BH = d.B * d.heads;
     TileMaps maps;
+    memset(&maps, 0, sizeof(maps));
     if (!encode_window_maps(maps.q, Q, BH, g.H, g.W) || !encode_window_maps(maps.k, K, BH, g.H, g.W) ||
         !encode_window_maps(maps.v, V, BH, g.H, g.W)) {
         set_error("ssba_forward (bf16): cuTensorMapEncodeTiled failed");
+        return SSBA_ERR_CUDA;
+    }
+    if (t_txt > 0 && (!encode_rows_map(&maps.kt, Kt, BH, t_txt) || !encode_rows_map(&maps.vt, Vt, BH, t_txt))) {
+        set_error("ssba_forward_joint: cuTensorMapEncodeTiled failed for the text keys/values");
         return SSBA_ERR_CUDA;
     }
     TcParams p;
@@ -851,6 +908,9 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
     p.cnt = cnt;
     p.g = g;
     p.keep = keep;
+    p.t_txt = t_txt > 0 ? t_txt : 0;
+    p.ntxt = (p.t_txt + 63) / 64;
+    p.units = p.ntxt + keep;
     p.num_items = BH * g.Tb();
     p.scale_log2 = scale * 1.4426950408889634f;
     p.budget_ns = budget_ns;
@@ -885,7 +945,7 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
         // more than another, and when items are long: a merge costs a few global-memory
         // round trips (about 5 us under load, measured), which 11-block items do not
         // earn back but 64-block items (dense) do (179 vs 198 us at 1024 px, 24 heads).
-        p.split = (keep >= kSplitMinKeep && p.num_items >= kSlots * grid && p.num_items % (kSlots * grid) != 0)
+        p.split = (p.units >= kSplitMinKeep && p.num_items >= kSlots * grid && p.num_items % (kSlots * grid) != 0)
                       ? 1 : 0;
     }
     ssba_attn_tc_kernel<<<grid, kThreads, smem, st>>>(maps, p);

@@ -53,7 +53,8 @@ constexpr uint64_t kWaitBudgetNs = 2000000000ull;  // 2 s
 int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q,
                         const void* K, const void* V, const int32_t* idx, const int32_t* cnt, void* O,
                         float* lse, void* ws, size_t ws_bytes, cudaStream_t st,
-                        uint64_t budget_ns = kWaitBudgetNs, int withhold = 0);
+                        uint64_t budget_ns = kWaitBudgetNs, int withhold = 0, const void* Kt = nullptr,
+                        const void* Vt = nullptr, int t_txt = 0);
 int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V,
                          void* O, float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
 // Bytes of the split-merge workspace of the bf16 forward on the current device.

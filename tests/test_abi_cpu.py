@@ -120,6 +120,19 @@ def test_forward_workspace_rules(lib):
         api.SSBA_ERR_WORKSPACE
 
 
+def test_forward_joint_validation(lib):
+    """The joint text + image entry point checks its text arguments before any launch."""
+    d = desc()
+    base = (FAKE, FAKE, FAKE)
+    tail = (FAKE, FAKE, FAKE, FAKE, None, 0, None)
+    assert lib.ssba_forward_joint(ctypes.byref(d), *base, None, None, 16, *tail) == api.SSBA_ERR_INVALID
+    assert lib.ssba_forward_joint(ctypes.byref(d), *base, FAKE, FAKE, -1, *tail) == api.SSBA_ERR_INVALID
+    assert lib.ssba_forward_joint(ctypes.byref(d), *base, FAKE + 8, FAKE, 16, *tail) == api.SSBA_ERR_INVALID
+    assert lib.ssba_forward_joint(ctypes.byref(desc(dtype=api.SSBA_FP32)), *base, FAKE, FAKE, 16, *tail) == \
+        api.SSBA_ERR_UNSUPPORTED
+    assert b"bf16" in lib.ssba_last_error()
+
+
 def test_build_mask_rejects_unsupported_head_dim(lib):
     d = desc(head_dim=12)  # 24 bytes per bf16 row: not a multiple of 16
     ws = lib.ssba_mask_workspace_bytes(ctypes.byref(d))

@@ -289,3 +289,36 @@ def test_forward_headline_whole_shares():
     torch.cuda.synchronize()
     O_o, lse_o = oracle.forward(q, k, v, idx_o, 64, 64, 8, (4, 4))
     check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
+# ----------------------------------------------------------------------------- text segment
+# Algorithm 1 with its text segment: every image query also attends to all T_txt text keys
+# (the token mask is padded with ones), and the image rows O[T_txt:] are returned.
+def _joint_case(H, W, h, rho, shift, T_txt, seed=21, workspace="default"):
+    q, k, v = synthetic.qkv(1, h, H * W, 64, torch.bfloat16, seed)
+    kt, vt, _ = synthetic.qkv(1, h, T_txt, 64, torch.bfloat16, seed + 1)
+    desc = api.SsbaDesc(1, h, H, W, shift_r=shift[0], shift_c=shift[1], rho=rho)
+    idx_o, cnt_o = oracle.build_mask(q, k, H, W, 8, shift, rho)
+    O, lse = api.forward_joint(desc, q.cuda(), k.cuda(), v.cuda(), kt.cuda(), vt.cuda(),
+                               torch.from_numpy(idx_o).cuda(), torch.from_numpy(cnt_o).cuda(), workspace=workspace)
+    torch.cuda.synchronize()
+    O_o, lse_o = oracle.forward_joint(q, k, v, kt, vt, idx_o, H, W, 8, shift)
+    return check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
+@pytest.mark.parametrize("T_txt,shift", [(77, (4, 4)), (256, (0, 0)), (5, (4, -4)), (0, (4, 4))])
+def test_forward_joint_text(T_txt, shift):
+    """Ragged (77 = 64 + 13), whole (256), shorter than one tile (5) and no text."""
+    _joint_case(32, 32, 4, 0.75, shift, T_txt)
+
+
+def test_forward_joint_headline_with_text():
+    """1024 px headline geometry with a 256-token text prefix."""
+    _joint_case(64, 64, 24, 0.8416, (4, 4), 256, seed=3)
+
+
+@pytest.mark.parametrize("workspace", ["default", None])
+def test_forward_joint_split_schedule(workspace):
+    """A 1024-token text prefix makes 16 + 11 = 27 key blocks per query block, so with a
+    workspace the pipelines take equal shares and cut query blocks; 320 query blocks."""
+    _joint_case(64, 64, 5, 0.8416, (4, 4), 1024, seed=5, workspace=workspace)
