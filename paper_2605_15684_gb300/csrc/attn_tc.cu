@@ -105,8 +105,11 @@ struct __align__(1024) SlotSmem {
     int nA, nB, M;                    // phase-A pieces, phase-B items, phase-A items (all pipelines)
 };
 
+constexpr int kWinCap = 1024;  // labels whose window (origin, box shape) is tabulated per CTA
+
 struct __align__(1024) SmemLayout {
     SlotSmem slot[kSlots];
+    uint32_t win[kWinCap];  // label -> r0 | c0 << 15 | box shape << 30 (see window_entry)
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -219,37 +222,47 @@ __device__ __forceinline__ void window_origin(const Grid& g, int label, int& r0,
     if (c0 < 0) c0 += g.W;
 }
 
-// Loads the 64 tokens of window `label` into an 8 KB tile with as few boxes as the grid
-// edge allows: one 8x8 box; two 8-col x 4-row boxes (split rows); two 4-col x 8-row
-// boxes (split columns); or four 4x4 boxes. The tile row order is set by the shape
-// class and decoded by tile_row_pos(); K and V of one label always share it.
-template <bool kPrefetch>
-__device__ __forceinline__ void window_boxes(const CUtensorMap* m4, uint32_t dst, uint32_t bar, const Grid& g,
-                                             int label, int bh)
+// Window of `label` packed in one word: origin row r0 (bits 0-14), origin column c0 (bits
+// 15-29) and the box shape class (bits 30-31: 0 one 8x8 box, 1 split rows, 2 split columns,
+// 3 both). Tabulated per CTA at kernel start, so that the producers' per-copy work is a
+// shared-memory load and a switch (the producers' issue loop is on the critical path).
+__device__ __forceinline__ uint32_t window_entry(const Grid& g, int label)
 {
     int r0, c0;
     window_origin(g, label, r0, c0);
-    const bool wr = r0 + 8 > g.H, wc = c0 + 8 > g.W;
-    auto box = [&](int shape, uint32_t off, int c, int r) {
-        if (kPrefetch) tma_prefetch_l2_4d(&m4[shape], 0, c, r, bh);
-        else tma_load_4d(dst + off, &m4[shape], bar, 0, c, r, bh);
-    };
-    if (!wr && !wc) {
-        box(kBox8x8, 0, c0, r0);
-    } else if (wr && !wc) {
-        box(kBox8c4r, 0, c0, r0);
-        box(kBox8c4r, 4096, c0, 0);
-    } else if (!wr && wc) {
-        box(kBox4c8r, 0, c0, r0);
-        box(kBox4c8r, 4096, 0, r0);
-    } else {
-        box(kBox4x4, 0, c0, r0);
-        box(kBox4x4, 2048, 0, r0);
-        box(kBox4x4, 4096, c0, 0);
-        box(kBox4x4, 6144, 0, 0);
+    const uint32_t wr = r0 + 8 > g.H, wc = c0 + 8 > g.W;
+    return (uint32_t)r0 | ((uint32_t)c0 << 15) | ((wr | (wc << 1)) << 30);
+}
+
+// TMA copies of a window given its packed entry (see window_boxes).
+__device__ __forceinline__ void window_boxes_e(const CUtensorMap* m4, uint32_t dst, uint32_t bar, uint32_t e, int bh)
+{
+    const int r0 = e & 0x7fff, c0 = (e >> 15) & 0x7fff;
+    switch (e >> 30) {
+        case 0:
+            tma_load_4d(dst, &m4[kBox8x8], bar, 0, c0, r0, bh);
+            break;
+        case 1:
+            tma_load_4d(dst, &m4[kBox8c4r], bar, 0, c0, r0, bh);
+            tma_load_4d(dst + 4096, &m4[kBox8c4r], bar, 0, c0, 0, bh);
+            break;
+        case 2:
+            tma_load_4d(dst, &m4[kBox4c8r], bar, 0, c0, r0, bh);
+            tma_load_4d(dst + 4096, &m4[kBox4c8r], bar, 0, 0, r0, bh);
+            break;
+        default:
+            tma_load_4d(dst, &m4[kBox4x4], bar, 0, c0, r0, bh);
+            tma_load_4d(dst + 2048, &m4[kBox4x4], bar, 0, 0, r0, bh);
+            tma_load_4d(dst + 4096, &m4[kBox4x4], bar, 0, c0, 0, bh);
+            tma_load_4d(dst + 6144, &m4[kBox4x4], bar, 0, 0, 0, bh);
+            break;
     }
 }
 
+// A window is one 8x8 box when it does not cross the grid edge, else two 8-col x 4-row boxes
+// (split rows), two 4-col x 8-row boxes (split columns) or four 4x4 boxes; the tile row
+// order is set by the shape class and decoded by tile_row_pos(); K and V of one label
+// always share it.
 // Tile row r of window `label` -> in-window position (row-major over the 8x8 window).
 __device__ __forceinline__ int tile_row_pos(const Grid& g, int label, int r)
 {
@@ -374,6 +387,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         fence_mbar_init();
     }
     build_schedule(p, sm, vcta, vgrid, threadIdx.x % (kSlotWarps * 32), kSlotWarps * 32);
+    for (int l = threadIdx.x; l < Tb && l < kWinCap; l += kThreads) cs.win[l] = window_entry(g, l);
     if (gwarp == 0 && lane < 12) tma_prefetch_desc(lane < 4 ? &maps.q[lane] : (lane < 8 ? &maps.k[lane - 4] : &maps.v[lane - 8]));
     if (gwarp == 1) {
         tmem_alloc(smem_u32(&cs.tmem_base), kTmemCols);
@@ -404,11 +418,14 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             const int ti0 = max(pc.tb, p.ntxt);
             const int nimg = max(0, pc.tb + nblk - ti0);
             const int32_t* list = p.idx ? p.idx + (size_t)pc.item * p.keep + (ti0 - p.ntxt) : nullptr;
-            // all lanes fetch the piece's labels in one round; lane 0 then issues the copies
-            // (measured: faster than prefetching them one piece ahead with cp.async)
-            int32_t* lab = sm.labels[is_k ? 0 : 1];
-            if (list)
-                for (int t = lane; t < nimg && t < kLabelCap; t += 32) lab[t] = __ldg(list + t);
+            // all lanes fetch the piece's labels in one round and stage their window entries;
+            // lane 0 then issues the copies (measured: faster than prefetching the labels one
+            // piece ahead with cp.async)
+            uint32_t* lab = reinterpret_cast<uint32_t*>(sm.labels[is_k ? 0 : 1]);
+            for (int t = lane; t < nimg && t < kLabelCap; t += 32) {
+                const int j = list ? clamp_label(__ldg(list + t), Tb) : ti0 - p.ntxt + t;
+                lab[t] = j < kWinCap ? cs.win[j] : window_entry(p.g, j);
+            }
             __syncwarp();
             if (lane == 0) {
                 if (is_k) {
@@ -416,7 +433,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     if (!mbar_wait(smem_u32(&sm.q_empty[qb]), ((nq >> 1) & 1) ^ 1, abortf, p.budget_ns)) dead = true;
                     if (!dead) {
                         mbar_arrive_expect_tx(smem_u32(&sm.q_full[qb]), kTileBytes);
-                        window_boxes<false>(maps.q, smem_u32(&sm.q[qb][0]), smem_u32(&sm.q_full[qb]), p.g, label, bh);
+                        window_boxes_e(maps.q, smem_u32(&sm.q[qb][0]), smem_u32(&sm.q_full[qb]),
+                                       label < kWinCap ? cs.win[label] : window_entry(p.g, label), bh);
                     }
                 }
                 const uint32_t nst = is_k ? kKStages : kVStages;
@@ -436,19 +454,27 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                                 smem_u32(full), 0, tt * 64, bh);
                 }
                 // image blocks of the piece: list entries [ti0 - ntxt, ti0 - ntxt + nimg)
+                const bool hold = p.withhold && is_k && vcta == 0;  // test hook: never lands
+                const uint32_t empty0 = smem_u32(is_k ? &sm.k_empty[0] : &sm.v_empty[0]);
+                const uint32_t full0 = smem_u32(is_k ? &sm.k_full[0] : &sm.v_full[0]);
+                const uint32_t tile0 = smem_u32(is_k ? &sm.k[0][0] : &sm.v[0][0]);
+                const CUtensorMap* m4 = is_k ? maps.k : maps.v;
                 for (int t = 0; t < nimg && !dead; ++t, ++g) {
-                    const int j = !list ? ti0 - p.ntxt + t : clamp_label(t < kLabelCap ? lab[t] : __ldg(list + t), Tb);
+                    uint32_t e;
+                    if (t < kLabelCap) {
+                        e = lab[t];
+                    } else {
+                        const int j = list ? clamp_label(__ldg(list + t), Tb) : ti0 - p.ntxt + t;
+                        e = j < kWinCap ? cs.win[j] : window_entry(p.g, j);
+                    }
                     const uint32_t slot = g % nst;
-                    uint64_t* empty = is_k ? &sm.k_empty[slot] : &sm.v_empty[slot];
-                    uint64_t* full = is_k ? &sm.k_full[slot] : &sm.v_full[slot];
-                    if (!mbar_wait(smem_u32(empty), ((g / nst) & 1) ^ 1, abortf, p.budget_ns)) {
+                    if (!mbar_wait(empty0 + 8 * slot, ((g / nst) & 1) ^ 1, abortf, p.budget_ns)) {
                         dead = true;
                         break;
                     }
-                    mbar_arrive_expect_tx(smem_u32(full), kTileBytes);
-                    if (p.withhold && is_k && vcta == 0 && g == 0) continue;  // test hook: never lands
-                    window_boxes<false>(is_k ? maps.k : maps.v, smem_u32(is_k ? &sm.k[slot][0] : &sm.v[slot][0]),
-                                        smem_u32(full), p.g, j, bh);
+                    mbar_arrive_expect_tx(full0 + 8 * slot, kTileBytes);
+                    if (hold && g == 0) continue;
+                    window_boxes_e(m4, tile0 + slot * kTileBytes, full0 + 8 * slot, e, bh);
                 }
             }
             dead = __shfl_sync(0xffffffffu, dead, 0);
@@ -883,6 +909,10 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
 {
     if (d.head_dim != kD || g.blk != 8 || (g.sr % 4) || (g.sc % 4)) {
         set_error("ssba_forward (bf16): needs head_dim=64, block=8 and shifts that are multiples of 4");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    if (g.H >= 32768 || g.W >= 32768) {
+        set_error("ssba_forward (bf16): H_tok and W_tok must be below 32768");
         return SSBA_ERR_UNSUPPORTED;
     }
     if (ws && ws_bytes < attn_tc_workspace_bytes()) {
