@@ -386,8 +386,12 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         mbar_init(smem_u32(&sm.drain[1]), 1);
         fence_mbar_init();
     }
-    build_schedule(p, sm, vcta, vgrid, threadIdx.x % (kSlotWarps * 32), kSlotWarps * 32);
     for (int l = threadIdx.x; l < Tb && l < kWinCap; l += kThreads) cs.win[l] = window_entry(g, l);
+    // everything above reads no input; the lists, counts and tensors may come from the grid
+    // launched just before this one (programmatic dependent launch)
+    grid_dep_wait();
+    grid_dep_launch();
+    build_schedule(p, sm, vcta, vgrid, threadIdx.x % (kSlotWarps * 32), kSlotWarps * 32);
     if (gwarp == 0 && lane < 12) tma_prefetch_desc(lane < 4 ? &maps.q[lane] : (lane < 8 ? &maps.k[lane - 4] : &maps.v[lane - 8]));
     if (gwarp == 1) {
         tmem_alloc(smem_u32(&cs.tmem_base), kTmemCols);
@@ -978,8 +982,21 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
         p.split = (p.units >= kSplitMinKeep && p.num_items >= kSlots * grid && p.num_items % (kSlots * grid) != 0)
                       ? 1 : 0;
     }
-    ssba_attn_tc_kernel<<<grid, kThreads, smem, st>>>(maps, p);
-    cudaError_t e = cudaGetLastError();
+    // programmatic dependent launch: the kernel may start (barriers, tensor memory, window
+    // table) while the previous grid on the stream finishes; it waits for that grid before
+    // reading any input
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, ssba_attn_tc_kernel, maps, p);
+    if (e == cudaSuccess) e = cudaGetLastError();
     if (e != cudaSuccess) {
         set_error("ssba_attn_tc_kernel launch: %s", cudaGetErrorString(e));
         return SSBA_ERR_CUDA;

@@ -20,6 +20,7 @@
 #include <cstdio>
 
 #include "common.cuh"
+#include "ptx.cuh"
 
 namespace ssba {
 
@@ -337,6 +338,10 @@ __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const 
     float* kbT = kown + bpc * kD;
     uint32_t* Skey = reinterpret_cast<uint32_t*>(kbT + kD * ld);
 
+    // Q and K may come from the grid launched just before this one
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
+
     // 1. pool the owned blocks
     const int col = lane % CPR, r0 = lane / CPR;
     for (int u = warp; u < 2 * nb; u += kFuseWarps) {
@@ -523,13 +528,15 @@ int launch_mask_fused(const ssba_desc& d, const Grid& g, int keep, const void* Q
     cfg.blockDim = dim3(kFuseWarps * 32, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = kFuseCluster;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_wait
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     cudaError_t e;
     if (d.dtype == SSBA_BF16) {
         auto k = ssba_mask_fused_kernel<__nv_bfloat16>;

@@ -156,6 +156,13 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const void* tmap, uint
         : "memory");
 }
 
+// Programmatic dependent launch. grid_dep_wait: wait until the grids this one depends on
+// have completed and their memory is visible (at once when there are none).
+// grid_dep_launch: allow the dependent grid to be scheduled (its blocks still wait for room
+// on the SMs and run their own grid_dep_wait before reading what this grid writes).
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // 3-D tiled load into CTA shared memory, completion counted on `bar` in bytes.
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, uint32_t bar, int c0, int c1, int c2)
 {
