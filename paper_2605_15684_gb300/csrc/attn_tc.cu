@@ -798,19 +798,30 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             const bool ok = st.y > 0.f;
             const float inv = ok ? 1.f / st.y : 0.f;
             const int tok = g.token(label, tile_row_pos(g, label, row));
-            uint4* dst = reinterpret_cast<uint4*>(p.O + ((size_t)bh * N + tok) * kD + half * 32);
+            uint4 v[4];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 float f[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e) f[e] = ok ? __uint_as_float(o[8 * i + e]) * inv : 0.f;
-                uint4 v;
-                v.x = pack_bf16(f[0], f[1]);
-                v.y = pack_bf16(f[2], f[3]);
-                v.z = pack_bf16(f[4], f[5]);
-                v.w = pack_bf16(f[6], f[7]);
-                dst[i] = v;
+                v[i].x = pack_bf16(f[0], f[1]);
+                v[i].y = pack_bf16(f[2], f[3]);
+                v[i].z = pack_bf16(f[4], f[5]);
+                v[i].w = pack_bf16(f[6], f[7]);
             }
+            // lanes l and l ^ 16 hold the two halves of one row (chunks 0-3 and 4-7): swap two
+            // chunks so that every store instruction writes whole 32-byte sectors
+            uint4 s0 = half ? v[0] : v[1], s1 = half ? v[2] : v[3], r0v, r1v;
+            r0v.x = __shfl_xor_sync(0xffffffffu, s0.x, 16); r0v.y = __shfl_xor_sync(0xffffffffu, s0.y, 16);
+            r0v.z = __shfl_xor_sync(0xffffffffu, s0.z, 16); r0v.w = __shfl_xor_sync(0xffffffffu, s0.w, 16);
+            r1v.x = __shfl_xor_sync(0xffffffffu, s1.x, 16); r1v.y = __shfl_xor_sync(0xffffffffu, s1.y, 16);
+            r1v.z = __shfl_xor_sync(0xffffffffu, s1.z, 16); r1v.w = __shfl_xor_sync(0xffffffffu, s1.w, 16);
+            uint4* rowp = reinterpret_cast<uint4*>(p.O + ((size_t)bh * N + tok) * kD);
+            // chunk written by this lane in instruction i: 2i + half
+            rowp[0 + half] = half ? r0v : v[0];
+            rowp[2 + half] = half ? r1v : v[2];
+            rowp[4 + half] = half ? v[1] : r0v;
+            rowp[6 + half] = half ? v[3] : r1v;
             if (half == 0)
                 p.lse[(size_t)bh * N + tok] = ok ? (st.x * 0.69314718055994531f + logf(st.y)) : -INFINITY;
         }
