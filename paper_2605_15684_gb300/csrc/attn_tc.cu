@@ -105,7 +105,7 @@ struct __align__(1024) SlotSmem {
     int nA, nB, M;                    // phase-A pieces, phase-B items, phase-A items (all pipelines)
 };
 
-constexpr int kWinCap = 1024;  // labels whose window (origin, box shape) is tabulated per CTA
+constexpr int kWinCap = 256;  // labels whose window (origin, box shape) is tabulated per CTA (2048 px: 256)
 
 struct __align__(1024) SmemLayout {
     SlotSmem slot[kSlots];
