@@ -68,6 +68,10 @@ def _load():
                                                 _F64P, _F64P]
         lib.ssba_oracle_dense_all.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, c_int, c_double,
                                               _F64P, _F64P]
+        lib.ssba_oracle_attention_backward.argtypes = [_F64P, _F64P, _F64P, _F64P, c_int, c_int, _I32P, c_int,
+                                                       _I32P, c_int, c_double, _F64P, _F64P, _F64P]
+        lib.ssba_oracle_backward_all.argtypes = [_F64P, _F64P, _F64P, _F64P, c_int, c_int, c_int, c_int, c_int,
+                                                 c_int, c_int, _I32P, c_int, c_double, _F64P, _F64P, _F64P]
         vp = ctypes.c_void_p
         lib.ssba_oracle_attention_joint.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, vp, vp, c_int, _I32P,
                                                     c_int, _I32P, c_int, c_double, _F64P, _F64P]
@@ -251,6 +255,32 @@ def forward_joint(Q, K, V, Kt, Vt, idx, H: int, W: int, blk: int = 8, shift=(0, 
                                                  int(shift[0]), int(shift[1]), idx, keep, scale, O, lse),
            "forward_joint")
     return O, lse
+
+
+def attention_backward(Q, K, V, dO, block_of, idx, scale=None):
+    """Single-slice gradients (dQ, dK, dV) of the sparse attention for output gradient dO."""
+    Q, K, V, dO = _f64(Q), _f64(K), _f64(V), _f64(dO)
+    N, d = Q.shape
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    Tb, keep = idx.shape
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    dQ, dK, dV = (np.empty((N, d), dtype=np.float64) for _ in range(3))
+    _check(_load().ssba_oracle_attention_backward(Q, K, V, dO, N, d, np.ascontiguousarray(block_of, np.int32),
+                                                  Tb, idx, keep, scale, dQ, dK, dV), "attention_backward")
+    return dQ, dK, dV
+
+
+def backward(Q, K, V, dO, idx, H: int, W: int, blk: int = 8, shift=(0, 0), scale=None):
+    """Whole-tensor gradients of the sparse forward. Q, K, V, dO: [B, heads, N, d]."""
+    Q, K, V, dO = _f64(Q), _f64(K), _f64(V), _f64(dO)
+    B, h, N, d = Q.shape
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    keep = idx.shape[-1]
+    scale = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    dQ, dK, dV = (np.empty((B, h, N, d), dtype=np.float64) for _ in range(3))
+    _check(_load().ssba_oracle_backward_all(Q, K, V, dO, B * h, H, W, d, blk, int(shift[0]), int(shift[1]), idx,
+                                            keep, scale, dQ, dK, dV), "backward")
+    return dQ, dK, dV
 
 
 def dense_forward(Q, K, V, scale=None):

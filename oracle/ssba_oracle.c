@@ -326,6 +326,77 @@ int ssba_oracle_attention_joint(const double *Q, const double *K, const double *
     return rc;
 }
 
+/* Gradients of the sparse attention of one slice (the backward pass of Algorithm 1's
+ * SparseAttention over the same expanded mask; the paper trains with it but does not write
+ * it out, so this is the chain rule of the forward above). Given the output gradient dO:
+ *   p_nm  = exp(a_nm - lse_n),  a_nm = scale * <Q_n, K_m>, over the allowed keys of n
+ *   D_n   = sum_m p_nm <dO_n, V_m>  (= <dO_n, O_n>)
+ *   dV_m  = sum_n p_nm dO_n
+ *   ds_nm = p_nm (<dO_n, V_m> - D_n)
+ *   dQ_n  = scale * sum_m ds_nm K_m,   dK_m = scale * sum_n ds_nm Q_n.
+ * Every sum runs over the pairs (n, m) the mask allows; query rows in token order, keys as
+ * in attend_row. */
+int ssba_oracle_attention_backward(const double *Q, const double *K, const double *V, const double *dO,
+                                   int N, int d, const int32_t *block_of, int Tb, const int32_t *idx,
+                                   int keep, double scale, double *dQ, double *dK, double *dV)
+{
+    if (!Q || !K || !V || !dO || !block_of || !idx || !dQ || !dK || !dV) return ORC_BAD;
+    if (N <= 0 || d <= 0 || Tb <= 0 || keep <= 0 || keep > Tb) return ORC_BAD;
+    int *start = (int *)malloc(sizeof(int) * ((size_t)Tb + 1));
+    int *tok = (int *)malloc(sizeof(int) * (size_t)N);
+    double *a = (double *)malloc(sizeof(double) * (size_t)N);
+    int *am = (int *)malloc(sizeof(int) * (size_t)N);
+    double *dp = (double *)malloc(sizeof(double) * (size_t)N);
+    int rc = (start && tok && a && am && dp) ? block_lists(N, block_of, Tb, start, tok) : ORC_BAD;
+    if (rc == ORC_OK) {
+        memset(dQ, 0, sizeof(double) * (size_t)N * d);
+        memset(dK, 0, sizeof(double) * (size_t)N * d);
+        memset(dV, 0, sizeof(double) * (size_t)N * d);
+    }
+    for (int n = 0; n < N && rc == ORC_OK; ++n) {
+        const int32_t *kept = idx + (size_t)block_of[n] * keep;
+        int na = 0;
+        for (int t = 0; t < keep && rc == ORC_OK; ++t) {
+            int j = kept[t];
+            if (j < 0 || j >= Tb) { rc = ORC_BAD; break; }
+            for (int u = start[j]; u < start[j + 1]; ++u) {
+                int m = tok[u];
+                double dot = 0.0;
+                for (int c = 0; c < d; ++c) dot += Q[(size_t)n * d + c] * K[(size_t)m * d + c];
+                a[na] = scale * dot;
+                am[na] = m;
+                na++;
+            }
+        }
+        if (rc != ORC_OK) break;
+        double mx = -INFINITY;
+        for (int u = 0; u < na; ++u) if (a[u] > mx) mx = a[u];
+        double sum = 0.0;
+        for (int u = 0; u < na; ++u) sum += exp(a[u] - mx);
+        const double lse = mx + log(sum);
+        double D = 0.0;
+        for (int u = 0; u < na; ++u) {
+            const double *vm = V + (size_t)am[u] * d;
+            double t = 0.0;
+            for (int c = 0; c < d; ++c) t += dO[(size_t)n * d + c] * vm[c];
+            dp[u] = t;
+            D += exp(a[u] - lse) * t;
+        }
+        for (int u = 0; u < na; ++u) {
+            const int m = am[u];
+            const double p = exp(a[u] - lse);
+            const double ds = p * (dp[u] - D);
+            for (int c = 0; c < d; ++c) {
+                dV[(size_t)m * d + c] += p * dO[(size_t)n * d + c];
+                dQ[(size_t)n * d + c] += scale * ds * K[(size_t)m * d + c];
+                dK[(size_t)m * d + c] += scale * ds * Q[(size_t)n * d + c];
+            }
+        }
+    }
+    free(start); free(tok); free(a); free(am); free(dp);
+    return rc;
+}
+
 /* Dense softmax attention over all N keys (Table 2 "baseline 0%" sparsity). */
 int ssba_oracle_dense_attention(const double *Q, const double *K, const double *V,
                                 int N, int d, double scale, double *O, double *lse)
@@ -443,6 +514,32 @@ int ssba_oracle_forward_joint_all(const double *Q, const double *K, const double
                                            Tt ? Vt + toff : NULL, Tt, block_of, Tb,
                                            idx + (size_t)s * Tb * keep, keep, scale, O + off,
                                            lse + (size_t)s * N);
+    }
+    free(block_of);
+    return bad ? ORC_BAD : ORC_OK;
+}
+
+int ssba_oracle_backward_all(const double *Q, const double *K, const double *V, const double *dO,
+                             int BH, int H, int W, int d, int blk, int shift_r, int shift_c,
+                             const int32_t *idx, int keep, double scale,
+                             double *dQ, double *dK, double *dV)
+{
+    if (!Q || !K || !V || !dO || !idx || !dQ || !dK || !dV || BH <= 0 || blk <= 0) return ORC_BAD;
+    if (H % blk || W % blk) return ORC_BAD;
+    int N = H * W, Tb = N / (blk * blk);
+    int32_t *block_of = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    if (!block_of) return ORC_BAD;
+    if (ssba_oracle_partition(H, W, blk, shift_r, shift_c, block_of) != ORC_OK) {
+        free(block_of);
+        return ORC_BAD;
+    }
+    int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(|:bad)
+    for (int s = 0; s < BH; ++s) {
+        size_t off = (size_t)s * N * d;
+        bad |= ssba_oracle_attention_backward(Q + off, K + off, V + off, dO + off, N, d, block_of, Tb,
+                                              idx + (size_t)s * Tb * keep, keep, scale,
+                                              dQ + off, dK + off, dV + off);
     }
     free(block_of);
     return bad ? ORC_BAD : ORC_OK;

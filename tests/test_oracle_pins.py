@@ -382,3 +382,68 @@ def test_joint_attention_reductions():
     Kt2[4] = 40.0 * Q2[0]
     Oh, _ = oracle.attention_joint(Q2, K, V, Kt2, Vt, lab, idx)
     np.testing.assert_allclose(Oh, np.tile(Vt[4], (N, 1)), atol=1e-9)
+
+
+# ----------------------------------------------------------------------------- backward
+def numpy_masked_attention_backward(Q, K, V, G, allowed, scale):
+    """Textbook matrix-form gradients of O = softmax(scale Q K^T, masked) V for dL/dO = G:
+    dV = P^T G, dP = G V^T, dS = P * (dP - rowsum(dP * P)), dQ = scale dS K, dK = scale dS^T Q."""
+    _, _, P = numpy_masked_softmax_attention(Q, K, V, allowed, scale)
+    dV = P.T @ G
+    dP = G @ V.T
+    dS = P * (dP - (dP * P).sum(axis=1, keepdims=True))
+    return scale * dS @ K, scale * dS.T @ Q, dV
+
+
+def _bwd_case(shift, seed):
+    rng = np.random.default_rng(seed)
+    H = W = 16
+    N, d = H * W, 8
+    Q, K, V, G = (rng.standard_normal((N, d)) for _ in range(4))
+    lab = oracle.partition(H, W, 8, shift)
+    idx = np.array([[0, 3], [1, 2], [0, 2], [1, 3]], dtype=np.int32)
+    return Q, K, V, G, lab, idx, d
+
+
+@pytest.mark.parametrize("shift", [(4, 4), (0, 0), (3, -5)])
+def test_backward_equals_matrix_form_of_masked_softmax(shift):
+    Q, K, V, G, lab, idx, d = _bwd_case(shift, 60)
+    allowed = np.zeros((Q.shape[0], Q.shape[0]), dtype=bool)
+    for n in range(Q.shape[0]):
+        allowed[n, np.isin(lab, idx[lab[n]])] = True
+    dQ, dK, dV = oracle.attention_backward(Q, K, V, G, lab, idx)
+    rQ, rK, rV = numpy_masked_attention_backward(Q, K, V, G, allowed, 1 / np.sqrt(d))
+    for a, b in ((dQ, rQ), (dK, rK), (dV, rV)):
+        np.testing.assert_allclose(a, b, rtol=0, atol=1e-12)
+
+
+def test_backward_matches_central_finite_differences():
+    """dL/dX for L = sum(G * O(Q, K, V)), at sampled entries, by central differences of the
+    forward oracle (h = 1e-5: truncation and rounding errors far below 1e-7)."""
+    Q, K, V, G, lab, idx, d = _bwd_case((4, 4), 61)
+    dQ, dK, dV = oracle.attention_backward(Q, K, V, G, lab, idx)
+
+    def loss(Qx, Kx, Vx):
+        O, _ = oracle.attention(Qx, Kx, Vx, lab, idx)
+        return float((G * O).sum())
+
+    rng = np.random.default_rng(62)
+    h = 1e-5
+    for which, grad in ((0, dQ), (1, dK), (2, dV)):
+        for _ in range(12):
+            n, c = int(rng.integers(Q.shape[0])), int(rng.integers(d))
+            args = [Q.copy(), K.copy(), V.copy()]
+            args[which][n, c] += h
+            lp = loss(*args)
+            args[which][n, c] -= 2 * h
+            lm = loss(*args)
+            assert abs((lp - lm) / (2 * h) - grad[n, c]) < 1e-7, (which, n, c)
+
+
+def test_backward_key_gradients_sum_to_zero():
+    """Each query row's ds sums to zero (sum_m p (dp - D) = D - D), so sum_m dK_m = 0; a
+    sign or normaliser error breaks it. dV sums to the column sums of dO (rows of P sum to 1)."""
+    Q, K, V, G, lab, idx, d = _bwd_case((4, 4), 63)
+    _, dK, dV = oracle.attention_backward(Q, K, V, G, lab, idx)
+    np.testing.assert_allclose(dK.sum(axis=0), 0.0, atol=1e-12)
+    np.testing.assert_allclose(dV.sum(axis=0), G.sum(axis=0), atol=1e-11)
