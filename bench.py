@@ -388,6 +388,32 @@ def run_ours(args, rank, world):
     except Exception as exc:  # reported, not fatal
         joint = f"failed: {exc}"
 
+    # ---- the backward pass (gradients over the same kept blocks) of a few layers; outside the
+    #      timed region. Algorithmic FLOPs: QK^T, dP = dO V^T, dV, dQ, dK on the kept blocks,
+    #      2.5 x the forward's
+    bwd = None
+    try:
+        gos = [synthetic.qkv(w.B, w.heads, w.N, w.head_dim, w.dtype, seed=700 + l + 1000 * rank)[0].to(dev)
+               for l in range(2)]
+        wsb = torch.empty(api.backward_workspace_bytes(descs[0]), dtype=torch.uint8, device=dev)
+        grads = [torch.empty(shp, dtype=torch.float32, device=dev) for _ in range(3)]
+        api.backward(descs[0], Qs[0], Ks[0], Vs[0], Os[0], lses[0], gos[0], idx[0], cnt[0], *grads, workspace=wsb)
+        reps = 6
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for r in range(reps):
+            l = r % 2
+            api.backward(descs[l], Qs[l], Ks[l], Vs[l], Os[l], lses[l], gos[l], idx[l], cnt[l], *grads, workspace=wsb)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        tb = e0.elapsed_time(e1) / reps
+        F_b = 2.5 * F_layer
+        bwd = {"ms_per_layer": tb, "effective_tflops": F_b / (tb * 1e-3) / 1e12, "flops_per_layer": F_b,
+               "how": "ssba_backward (CUDA cores, fp32) per layer on the layer's forward O and lse and a "
+                      "synthetic dO, CUDA events"}
+    except Exception as exc:  # reported, not fatal
+        bwd = f"failed: {exc}"
+
     # ---- end to end through the public API with host buffers (pinned), copies timed
     e2e = None
     if args.e2e_steps > 0:
@@ -459,6 +485,7 @@ def run_ours(args, rank, world):
             "roofline": roofline, "roofline_mask": mask_roof,
             "dense_attention_ms_per_layer": dense_ms,
             "text_joint": joint,
+            "backward": bwd,
             "speedup_vs_dense": (dense_ms / attn_ms) if isinstance(dense_ms, float) else None,
             "ideal_speedup_vs_dense": Tb / keep,
             "e2e": e2e, "cpu_baseline": cpu,

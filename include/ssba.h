@@ -163,6 +163,28 @@ SSBA_API size_t ssba_forward_workspace_bytes(const ssba_desc* desc);
 SSBA_API int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, const void* V,
                        void* O, float* lse, void* workspace, size_t ws_bytes, void* stream);
 
+/* Gradients of ssba_forward (the backward pass of Algorithm 1's SparseAttention over the
+ * same kept blocks; the paper trains its sparse model but does not write the backward
+ * out, so this is the chain rule of the forward). For the output gradient dO, with
+ * p_nm = exp(scale q_n.k_m - lse_n) over the pairs the lists allow:
+ *   D_n = dO_n . O_n,  dV_m = sum_n p_nm dO_n,  ds_nm = p_nm (dO_n . v_m - D_n),
+ *   dQ_n = scale sum_m ds_nm k_m,  dK_m = scale sum_n ds_nm q_n.
+ *   Q, K, V, O, dO  device, [B][heads][N][head_dim] of desc->dtype (O and lse as
+ *                   ssba_forward wrote them).
+ *   lse             device, fp32 [B][heads][N].
+ *   kv_idx, kv_cnt  the lists of the forward.
+ *   dQ, dK, dV      device out, fp32 [B][heads][N][head_dim], every element written.
+ *   workspace       device scratch of at least ssba_backward_workspace_bytes(desc) bytes
+ *                   (the D_n values), 16-byte aligned.
+ * CUDA cores in fp32 (any dtype), head_dim = 64 and block = 8; deterministic (no atomics:
+ * the key gradients are gathered per key block over the query blocks that keep it). */
+SSBA_API int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, const void* V, const void* O,
+                           const float* lse, const void* dO, const int32_t* kv_idx, const int32_t* kv_cnt,
+                           float* dQ, float* dK, float* dV, void* workspace, size_t ws_bytes, void* stream);
+
+/* Bytes of the ssba_backward workspace: B * heads * N * 4 (0 for an invalid descriptor). */
+SSBA_API size_t ssba_backward_workspace_bytes(const ssba_desc* desc);
+
 /* Size of the scratch area built into the library for ssba_build_mask_noalloc (4 MiB). */
 #define SSBA_NOALLOC_SCRATCH_BYTES (4u << 20)
 

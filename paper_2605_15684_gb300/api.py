@@ -28,7 +28,7 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
 
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
-            "ssba_test_forward_timeout",
+            "ssba_test_forward_timeout", "ssba_backward", "ssba_backward_workspace_bytes",
             "ssba_get_status", "ssba_last_error")
 
 
@@ -112,6 +112,10 @@ def load_library():
         lib.ssba_forward_dense.restype = ctypes.c_int
         lib.ssba_test_forward_timeout.argtypes = [DP, P, P, P, P, P, P, P, ctypes.c_uint64, P]
         lib.ssba_test_forward_timeout.restype = ctypes.c_int
+        lib.ssba_backward.argtypes = [DP, P, P, P, P, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
+        lib.ssba_backward.restype = ctypes.c_int
+        lib.ssba_backward_workspace_bytes.argtypes = [DP]
+        lib.ssba_backward_workspace_bytes.restype = ctypes.c_size_t
         lib.ssba_get_status.argtypes = [ctypes.POINTER(ctypes.c_int32)]
         lib.ssba_get_status.restype = ctypes.c_int
         lib.ssba_last_error.argtypes = []
@@ -361,6 +365,43 @@ def test_forward_timeout(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O, lse, budget
     _raise_on(lib.ssba_test_forward_timeout(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(),
                                             kv_idx.data_ptr(), kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(),
                                             int(budget_ns), _stream_ptr(stream)))
+
+
+def backward_workspace_bytes(desc: SsbaDesc) -> int:
+    lib = load_library()
+    d = desc.c()
+    return int(lib.ssba_backward_workspace_bytes(ctypes.byref(d)))
+
+
+def backward(desc: SsbaDesc, Q, K, V, O, lse, dO, kv_idx, kv_cnt, dQ=None, dK=None, dV=None, workspace=None,
+             stream=None):
+    """ssba_backward: gradients (dQ, dK, dV) in fp32 of the sparse forward for output gradient dO."""
+    lib = load_library()
+    d = desc.c()
+    keep = lib.ssba_keep_count(ctypes.byref(d))
+    if keep < 0:
+        _raise_on(SSBA_ERR_INVALID)
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V"), (O, "O"), (dO, "dO")):
+        _check(t, n, shp, desc.dtype)
+    _check(lse, "lse", shp[:3], torch.float32)
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    outs = []
+    for t, n in ((dQ, "dQ"), (dK, "dK"), (dV, "dV")):
+        if t is None:
+            t = torch.empty(shp, dtype=torch.float32, device=Q.device)
+        _check(t, n, shp, torch.float32)
+        outs.append(t)
+    need = int(lib.ssba_backward_workspace_bytes(ctypes.byref(d)))
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=Q.device)
+    wp, wn = _ws_args(workspace)
+    rc = lib.ssba_backward(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), O.data_ptr(), lse.data_ptr(),
+                           dO.data_ptr(), kv_idx.data_ptr(), kv_cnt.data_ptr(), outs[0].data_ptr(),
+                           outs[1].data_ptr(), outs[2].data_ptr(), wp, wn, _stream_ptr(stream))
+    _raise_on(rc)
+    return tuple(outs)
 
 
 def get_status() -> int:

@@ -276,6 +276,42 @@ int ssba_test_forward_timeout(const ssba_desc* desc, const void* Q, const void* 
                                static_cast<cudaStream_t>(stream), b, 1);
 }
 
+size_t ssba_backward_workspace_bytes(const ssba_desc* desc)
+{
+    Grid g;
+    int keep;
+    if (check_desc(desc, "ssba_backward_workspace_bytes", &g, &keep) != SSBA_OK) return 0;
+    return (size_t)desc->B * desc->heads * desc->H_tok * desc->W_tok * sizeof(float);
+}
+
+int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, const void* V, const void* O, const float* lse,
+                  const void* dO, const int32_t* kv_idx, const int32_t* kv_cnt, float* dQ, float* dK, float* dV,
+                  void* workspace, size_t ws_bytes, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_backward", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !V || !O || !lse || !dO || !kv_idx || !kv_cnt || !dQ || !dK || !dV) {
+        set_error("ssba_backward: every pointer must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    const size_t es = elem_size(desc);
+    if (!aligned(Q, es) || !aligned(K, es) || !aligned(V, es) || !aligned(O, es) || !aligned(dO, es) ||
+        !aligned(lse, 4) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) || !aligned(dQ, 4) || !aligned(dK, 4) ||
+        !aligned(dV, 4)) {
+        set_error("ssba_backward: pointers must be aligned to their element size");
+        return SSBA_ERR_INVALID;
+    }
+    const size_t need = ssba_backward_workspace_bytes(desc);
+    if (!workspace || ws_bytes < need || !aligned(workspace, 16)) {
+        set_error("ssba_backward: workspace of %zu bytes (16-byte aligned) required, got %zu", need, ws_bytes);
+        return SSBA_ERR_WORKSPACE;
+    }
+    return launch_backward(*desc, g, keep, resolve_scale(desc), Q, K, V, O, lse, dO, kv_idx, kv_cnt, dQ, dK, dV,
+                           static_cast<float*>(workspace), static_cast<cudaStream_t>(stream));
+}
+
 int ssba_get_status(int32_t* device_status_out)
 {
     if (!device_status_out) {

@@ -60,6 +60,10 @@ int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const v
 // Bytes of the split-merge workspace of the bf16 forward on the current device.
 size_t attn_tc_workspace_bytes();
 
+int launch_backward(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
+                    const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
+                    const int32_t* cnt, float* dQ, float* dK, float* dV, float* Dbuf, cudaStream_t st);
+
 // Thread-local error text for ssba_last_error().
 void set_error(const char* fmt, ...);
 

@@ -133,6 +133,19 @@ def test_forward_joint_validation(lib):
     assert b"bf16" in lib.ssba_last_error()
 
 
+def test_backward_validation(lib):
+    """The backward entry point checks its workspace and shape before any launch."""
+    d = desc()
+    need = lib.ssba_backward_workspace_bytes(ctypes.byref(d))
+    assert need == 1 * 2 * 16 * 16 * 4
+    args = [ctypes.byref(d)] + [FAKE] * 11
+    assert lib.ssba_backward(*args, FAKE, need - 4, None) == api.SSBA_ERR_WORKSPACE
+    assert lib.ssba_backward(*args, None, need, None) == api.SSBA_ERR_WORKSPACE
+    bad = [ctypes.byref(d)] + [FAKE] * 5 + [None] + [FAKE] * 5
+    assert lib.ssba_backward(*bad, FAKE, need, None) == api.SSBA_ERR_INVALID
+    assert lib.ssba_backward_workspace_bytes(ctypes.byref(desc(H_tok=12))) == 0
+
+
 def test_build_mask_rejects_unsupported_head_dim(lib):
     d = desc(head_dim=12)  # 24 bytes per bf16 row: not a multiple of 16
     ws = lib.ssba_mask_workspace_bytes(ctypes.byref(d))

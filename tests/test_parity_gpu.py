@@ -322,3 +322,65 @@ def test_forward_joint_split_schedule(workspace):
     """A 1024-token text prefix makes 16 + 11 = 27 key blocks per query block, so with a
     workspace the pipelines take equal shares and cut query blocks; 320 query blocks."""
     _joint_case(64, 64, 5, 0.8416, (4, 4), 1024, seed=5, workspace=workspace)
+
+
+# ----------------------------------------------------------------------------- backward
+# Gradients of the sparse forward (fp32 outputs) against the fp64 oracle backward. The error
+# is measured relative to the largest gradient of the tensor: with fp32 arithmetic and exact
+# (fp32) O the bound is 1e-5 (measured about 1e-6); with bf16 inputs O is itself rounded to
+# bf16 (2^-9 relative), which moves D = dO . O and through it every ds, so the bound is 5e-3
+# (measured about 6e-4 at the 1024 px geometry).
+BWD_TOL = {torch.float32: 1e-5, torch.bfloat16: 5e-3}
+
+
+def _check_grads(got, ref, dtype):
+    out = {}
+    for name, g_, r in zip(("dQ", "dK", "dV"), got, ref):
+        g_ = g_.cpu().numpy().astype(np.float64)
+        assert np.all(np.isfinite(g_)), name
+        rel = float(np.abs(g_ - r).max() / max(1.0, np.abs(r).max()))
+        out[name] = rel
+        assert rel <= BWD_TOL[dtype], (name, rel)
+    return out
+
+
+def _bwd_case_gpu(B, h, H, W, rho, shift, dtype, seed):
+    q, k, v = synthetic.qkv(B, h, H * W, 64, dtype, seed)
+    go = synthetic.qkv(B, h, H * W, 64, dtype, seed + 100)[0]
+    idx_o, cnt_o = oracle.build_mask(q, k, H, W, 8, shift, rho)
+    O_o, lse_o = oracle.forward(q, k, v, idx_o, H, W, 8, shift)
+    desc = api.SsbaDesc(B, h, H, W, shift_r=shift[0], shift_c=shift[1], rho=rho, dtype=dtype)
+    grads = api.backward(desc, q.cuda(), k.cuda(), v.cuda(), torch.from_numpy(O_o).to(dtype).cuda(),
+                         torch.from_numpy(lse_o).float().cuda(), go.cuda(), torch.from_numpy(idx_o).cuda(),
+                         torch.from_numpy(cnt_o).cuda())
+    torch.cuda.synchronize()
+    ref = oracle.backward(q, k, v, go, idx_o, H, W, 8, shift)
+    return _check_grads(grads, ref, dtype)
+
+
+@pytest.mark.parametrize("shift", [(0, 0), (4, 4), (3, -5)])
+@pytest.mark.parametrize("rho", [0.75, 0.0])
+def test_backward_fp32_tiny(shift, rho):
+    _bwd_case_gpu(1, 2, 16, 16, rho, shift, torch.float32, 30)
+
+
+@pytest.mark.parametrize("H,W,h,rho,shift", [(32, 32, 4, 0.75, (4, 4)), (64, 64, 4, 0.8416, (4, 4)),
+                                            (24, 40, 3, 0.6, (4, -4))])
+def test_backward_bf16(H, W, h, rho, shift):
+    _bwd_case_gpu(1, h, H, W, rho, shift, torch.bfloat16, 31)
+
+
+def test_backward_after_gpu_forward():
+    """The training order: GPU mask, GPU forward, then the backward on the forward's own O
+    and lse, against the oracle backward on the same lists."""
+    H = W = 32
+    q, k, v = synthetic.qkv(1, 4, H * W, 64, torch.bfloat16, 32)
+    go = synthetic.qkv(1, 4, H * W, 64, torch.bfloat16, 132)[0]
+    desc = api.SsbaDesc(1, 4, H, W, shift_r=4, shift_c=4, rho=0.75)
+    qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
+    idx, cnt = api.build_mask(desc, qd, kd)
+    O, lse = api.forward(desc, qd, kd, vd, idx, cnt)
+    grads = api.backward(desc, qd, kd, vd, O, lse, go.cuda(), idx, cnt)
+    torch.cuda.synchronize()
+    ref = oracle.backward(q, k, v, go, idx.cpu().numpy(), H, W, 8, (4, 4))
+    _check_grads(grads, ref, torch.bfloat16)
