@@ -72,6 +72,8 @@ def _load():
                                                        _I32P, c_int, c_double, _F64P, _F64P, _F64P]
         lib.ssba_oracle_backward_all.argtypes = [_F64P, _F64P, _F64P, _F64P, c_int, c_int, c_int, c_int, c_int,
                                                  c_int, c_int, _I32P, c_int, c_double, _F64P, _F64P, _F64P]
+        lib.ssba_oracle_haar_dwt.argtypes = [_F64P, c_int, c_int, c_int, c_int, _F64P]
+        lib.ssba_oracle_haar_iwt.argtypes = [_F64P, c_int, c_int, c_int, c_int, _F64P]
         vp = ctypes.c_void_p
         lib.ssba_oracle_attention_joint.argtypes = [_F64P, _F64P, _F64P, c_int, c_int, vp, vp, c_int, _I32P,
                                                     c_int, _I32P, c_int, c_double, _F64P, _F64P]
@@ -291,3 +293,25 @@ def dense_forward(Q, K, V, scale=None):
     lse = np.empty((B, h, N), dtype=np.float64)
     _check(_load().ssba_oracle_dense_all(Q, K, V, B * h, N, d, scale, O, lse), "dense_forward")
     return O, lse
+
+
+def haar_dwt(x, nb: int = 4):
+    """One Haar level per channel: x [..., C, H, W] -> [..., nb * C, H/2, W/2] (LL, HL, LH, HH)."""
+    x = _f64(x)
+    *lead, C, H, W = x.shape
+    xs = x.reshape(-1, C, H, W)
+    y = np.empty((xs.shape[0], nb * C, H // 2, W // 2), dtype=np.float64)
+    for i in range(xs.shape[0]):
+        _check(_load().ssba_oracle_haar_dwt(np.ascontiguousarray(xs[i]), C, H, W, nb, y[i]), "haar_dwt")
+    return y.reshape(*lead, nb * C, H // 2, W // 2)
+
+
+def haar_iwt(y, C: int, nb: int = 4):
+    """Inverse Haar level: y [..., nb * C, h, w] -> [..., C, 2h, 2w] (HH = 0 when nb = 3)."""
+    y = _f64(y)
+    *lead, nbC, h, w = y.shape
+    ys = y.reshape(-1, nbC, h, w)
+    x = np.empty((ys.shape[0], C, 2 * h, 2 * w), dtype=np.float64)
+    for i in range(ys.shape[0]):
+        _check(_load().ssba_oracle_haar_iwt(np.ascontiguousarray(ys[i]), C, 2 * h, 2 * w, nb, x[i]), "haar_iwt")
+    return x.reshape(*lead, C, 2 * h, 2 * w)

@@ -577,3 +577,51 @@ void ssba_oracle_set_threads(int n)
     (void)n;
 #endif
 }
+
+/* ---------------------------------------------------------------- Haar wavelets (T-DVAE)
+ * One level of the 2-D Haar kernel bank F = {LL, HL, LH, HH} (Sec. 2.3 DWT-Enhanced
+ * Architecture), orthonormal, stride 2, per channel. x [C][H][W] (H, W even); for the 2 x 2
+ * window a = x[2i][2j], b = x[2i][2j+1], c = x[2i+1][2j], d = x[2i+1][2j+1]:
+ *   LL = (a + b + c + d) / 2,  HL = (a - b + c - d) / 2,
+ *   LH = (a + b - c - d) / 2,  HH = (a - b - c + d) / 2.
+ * y [nb * C][H/2][W/2], subband-major: bands LL, HL, LH (and HH when nb = 4) of every
+ * channel; nb = 3 keeps c = {LL, HL, LH} as the paper's recursion does. */
+int ssba_oracle_haar_dwt(const double *x, int C, int H, int W, int nb, double *y)
+{
+    if (!x || !y || C <= 0 || H <= 0 || W <= 0 || (H & 1) || (W & 1) || (nb != 3 && nb != 4)) return ORC_BAD;
+    const int h2 = H / 2, w2 = W / 2;
+    for (int ch = 0; ch < C; ++ch)
+        for (int i = 0; i < h2; ++i)
+            for (int j = 0; j < w2; ++j) {
+                const double *xc = x + (size_t)ch * H * W;
+                const double a = xc[(size_t)(2 * i) * W + 2 * j], b = xc[(size_t)(2 * i) * W + 2 * j + 1];
+                const double c = xc[(size_t)(2 * i + 1) * W + 2 * j], d = xc[(size_t)(2 * i + 1) * W + 2 * j + 1];
+                const double band[4] = {(a + b + c + d) / 2, (a - b + c - d) / 2, (a + b - c - d) / 2,
+                                        (a - b - c + d) / 2};
+                for (int s = 0; s < nb; ++s) y[((size_t)s * C + ch) * h2 * w2 + (size_t)i * w2 + j] = band[s];
+            }
+    return ORC_OK;
+}
+
+/* The inverse (the transpose of the orthonormal bank): y [nb * C][H/2][W/2] as above (HH
+ * taken as 0 when nb = 3), x [C][H][W]:
+ *   a = (LL + HL + LH + HH) / 2,  b = (LL - HL + LH - HH) / 2,
+ *   c = (LL + HL - LH - HH) / 2,  d = (LL - HL - LH + HH) / 2. */
+int ssba_oracle_haar_iwt(const double *y, int C, int H, int W, int nb, double *x)
+{
+    if (!x || !y || C <= 0 || H <= 0 || W <= 0 || (H & 1) || (W & 1) || (nb != 3 && nb != 4)) return ORC_BAD;
+    const int h2 = H / 2, w2 = W / 2;
+    for (int ch = 0; ch < C; ++ch)
+        for (int i = 0; i < h2; ++i)
+            for (int j = 0; j < w2; ++j) {
+                double v[4] = {0, 0, 0, 0};
+                for (int s = 0; s < nb; ++s) v[s] = y[((size_t)s * C + ch) * h2 * w2 + (size_t)i * w2 + j];
+                const double LL = v[0], HL = v[1], LH = v[2], HH = v[3];
+                double *xc = x + (size_t)ch * H * W;
+                xc[(size_t)(2 * i) * W + 2 * j] = (LL + HL + LH + HH) / 2;
+                xc[(size_t)(2 * i) * W + 2 * j + 1] = (LL - HL + LH - HH) / 2;
+                xc[(size_t)(2 * i + 1) * W + 2 * j] = (LL + HL - LH - HH) / 2;
+                xc[(size_t)(2 * i + 1) * W + 2 * j + 1] = (LL - HL - LH + HH) / 2;
+            }
+    return ORC_OK;
+}

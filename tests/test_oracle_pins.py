@@ -447,3 +447,40 @@ def test_backward_key_gradients_sum_to_zero():
     _, dK, dV = oracle.attention_backward(Q, K, V, G, lab, idx)
     np.testing.assert_allclose(dK.sum(axis=0), 0.0, atol=1e-12)
     np.testing.assert_allclose(dV.sum(axis=0), G.sum(axis=0), atol=1e-11)
+
+
+# ----------------------------------------------------------------------------- Haar wavelets
+def test_haar_hand_example_and_reconstruction():
+    """A 2 x 2 window by hand, perfect reconstruction (the bank is orthonormal), energy
+    preservation, and a constant image that has only an LL band."""
+    x = np.array([[[1.0, 2.0], [3.0, 5.0]]])  # a=1 b=2 c=3 d=5
+    y = oracle.haar_dwt(x)
+    np.testing.assert_allclose(y[:, 0, 0], [11 / 2, -3 / 2, -5 / 2, 1 / 2])  # LL HL LH HH
+    rng = np.random.default_rng(70)
+    x = rng.standard_normal((3, 6, 8))
+    y = oracle.haar_dwt(x)
+    np.testing.assert_allclose(oracle.haar_iwt(y, 3), x, atol=1e-14)
+    np.testing.assert_allclose((y ** 2).sum(), (x ** 2).sum(), rtol=1e-13)
+    yc = oracle.haar_dwt(np.full((2, 4, 4), 3.0))
+    np.testing.assert_allclose(yc[:2], 6.0)
+    np.testing.assert_allclose(yc[2:], 0.0)
+
+
+def test_haar_bands_are_separable_1d_haar():
+    """The 2-D bands equal the 1-D orthonormal Haar (sum, difference over sqrt 2) along
+    the width, then along the height: LL = low-low, HL = width-high/height-low, ..."""
+    rng = np.random.default_rng(71)
+    x = rng.standard_normal((2, 8, 6))
+    s2 = np.sqrt(2.0)
+    lo_w = (x[..., 0::2] + x[..., 1::2]) / s2
+    hi_w = (x[..., 0::2] - x[..., 1::2]) / s2
+    bands = [(lo_w[..., 0::2, :] + lo_w[..., 1::2, :]) / s2, (hi_w[..., 0::2, :] + hi_w[..., 1::2, :]) / s2,
+             (lo_w[..., 0::2, :] - lo_w[..., 1::2, :]) / s2, (hi_w[..., 0::2, :] - hi_w[..., 1::2, :]) / s2]
+    y = oracle.haar_dwt(x)
+    for s, b in enumerate(bands):
+        np.testing.assert_allclose(y[s * 2:(s + 1) * 2], b, atol=1e-14)
+    # dropping HH: the inverse of the three kept bands is x minus the HH contribution
+    y3 = oracle.haar_dwt(x, nb=3)
+    np.testing.assert_array_equal(y3, y[:6])
+    np.testing.assert_allclose(oracle.haar_iwt(y3, 2, nb=3) + oracle.haar_iwt(
+        np.concatenate([np.zeros_like(y[:6]), y[6:]]), 2), x, atol=1e-14)
