@@ -414,6 +414,42 @@ def run_ours(args, rank, world):
     except Exception as exc:  # reported, not fatal
         bwd = f"failed: {exc}"
 
+    # ---- one level of the T-DVAE's Haar bank and its inverse on a VAE-sized feature map
+    #      (128 channels of 1024 x 1024, bf16; 256 MiB each way, larger than L2); outside the
+    #      timed region. Algorithmic bytes: every input element read once, every output written once
+    haar = None
+    try:
+        hN, hC, hH, hW = 1, 128, 1024, 1024
+        hx = synthetic.feature_map(hN, hC, hH, hW, torch.bfloat16, seed=900 + rank).to(dev)
+        hy = torch.empty((hN, 4 * hC, hH // 2, hW // 2), dtype=torch.bfloat16, device=dev)
+        hy3 = torch.empty((hN, 3 * hC, hH // 2, hW // 2), dtype=torch.bfloat16, device=dev)
+        hb = torch.empty_like(hx)
+        nbytes = hx.numel() * 2
+        peak = hbm_gbs
+        out = {}
+        for name, fn, moved in (("dwt_nb4", lambda: api.haar_dwt(hx, 4, y=hy, stream=stream), 2 * nbytes),
+                                ("dwt_nb3", lambda: api.haar_dwt(hx, 3, y=hy3, stream=stream), nbytes * 7 // 4),
+                                ("iwt_nb4", lambda: api.haar_iwt(hy, hC, 4, x=hb, stream=stream), 2 * nbytes)):
+            for _ in range(3):
+                fn()
+            reps = 10
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(reps):
+                fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            t = e0.elapsed_time(e1) / reps
+            gbs = moved / (t * 1e-3) / 1e9
+            out[name] = {"us": t * 1e3, "bytes": moved, "achieved_gbs": gbs,
+                         "frac": gbs / peak}
+        haar = dict(out, shape=[hN, hC, hH, hW], dtype="bf16", peak_gbs=peak, peak_source=peak_src,
+                    how="ssba_haar_dwt / ssba_haar_iwt back to back, CUDA events around 10 launches; "
+                        "frac of the HBM copy bandwidth")
+        del hx, hy, hy3, hb
+    except Exception as exc:  # reported, not fatal
+        haar = f"failed: {exc}"
+
     # ---- end to end through the public API with host buffers (pinned), copies timed
     e2e = None
     if args.e2e_steps > 0:
@@ -486,6 +522,7 @@ def run_ours(args, rank, world):
             "dense_attention_ms_per_layer": dense_ms,
             "text_joint": joint,
             "backward": bwd,
+            "haar": haar,
             "speedup_vs_dense": (dense_ms / attn_ms) if isinstance(dense_ms, float) else None,
             "ideal_speedup_vs_dense": Tb / keep,
             "e2e": e2e, "cpu_baseline": cpu,

@@ -185,6 +185,23 @@ SSBA_API int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, 
 /* Bytes of the ssba_backward workspace: B * heads * N * 4 (0 for an invalid descriptor). */
 SSBA_API size_t ssba_backward_workspace_bytes(const ssba_desc* desc);
 
+/* One level of the T-DVAE's 2-D Haar kernel bank F = {LL, HL, LH, HH} (Sec. 2.3
+ * DWT-Enhanced Architecture), per channel, stride 2, orthonormal: for the window
+ * a = x[2i][2j], b = x[2i][2j+1], c = x[2i+1][2j], d = x[2i+1][2j+1],
+ *   LL = (a+b+c+d)/2, HL = (a-b+c-d)/2, LH = (a+b-c-d)/2, HH = (a-b-c+d)/2.
+ *   x   device, [N][C][H][W] of dtype (SSBA_BF16 or SSBA_FP32), H and W even.
+ *   y   device out, [N][nb*C][H/2][W/2] of dtype, subband-major (LL, HL, LH[, HH] of every
+ *       channel); nb = 4, or 3 to keep c = {LL, HL, LH} as the paper's recursion does.
+ * Both 16-byte aligned. fp32 arithmetic. Returns SSBA_ERR_INVALID for bad sizes or pointers,
+ * SSBA_ERR_UNSUPPORTED when one image holds 2^31 or more 16-byte units (C*H*W*size >= 64 GiB). */
+SSBA_API int ssba_haar_dwt(const void* x, void* y, int32_t N, int32_t C, int32_t H, int32_t W, int32_t nb,
+                           int32_t dtype, void* stream);
+
+/* The inverse level (the transpose of the orthonormal bank): y [N][nb*C][H/2][W/2] -> x
+ * [N][C][H][W]; with nb = 3 the HH band is taken as zero. Same layouts and rules. */
+SSBA_API int ssba_haar_iwt(const void* y, void* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t nb,
+                           int32_t dtype, void* stream);
+
 /* Size of the scratch area built into the library for ssba_build_mask_noalloc (4 MiB). */
 #define SSBA_NOALLOC_SCRATCH_BYTES (4u << 20)
 

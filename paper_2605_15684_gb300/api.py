@@ -28,7 +28,8 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
 
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
-            "ssba_test_forward_timeout", "ssba_backward", "ssba_backward_workspace_bytes",
+            "ssba_test_forward_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
+            "ssba_haar_iwt",
             "ssba_get_status", "ssba_last_error")
 
 
@@ -116,6 +117,10 @@ def load_library():
         lib.ssba_backward.restype = ctypes.c_int
         lib.ssba_backward_workspace_bytes.argtypes = [DP]
         lib.ssba_backward_workspace_bytes.restype = ctypes.c_size_t
+        I = ctypes.c_int32
+        for fn in ("ssba_haar_dwt", "ssba_haar_iwt"):
+            getattr(lib, fn).argtypes = [P, P, I, I, I, I, I, I, P]
+            getattr(lib, fn).restype = ctypes.c_int
         lib.ssba_get_status.argtypes = [ctypes.POINTER(ctypes.c_int32)]
         lib.ssba_get_status.restype = ctypes.c_int
         lib.ssba_last_error.argtypes = []
@@ -402,6 +407,42 @@ def backward(desc: SsbaDesc, Q, K, V, O, lse, dO, kv_idx, kv_cnt, dQ=None, dK=No
                            outs[1].data_ptr(), outs[2].data_ptr(), wp, wn, _stream_ptr(stream))
     _raise_on(rc)
     return tuple(outs)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return SSBA_BF16
+    if t.dtype == torch.float32:
+        return SSBA_FP32
+    raise SsbaError(SSBA_ERR_INVALID, f"unsupported dtype {t.dtype}")
+
+
+def haar_dwt(x: torch.Tensor, nb: int = 4, y=None, stream=None) -> torch.Tensor:
+    """ssba_haar_dwt: x [N, C, H, W] -> [N, nb*C, H/2, W/2] (LL, HL, LH[, HH] bands)."""
+    lib = load_library()
+    if not isinstance(x, torch.Tensor) or x.dim() != 4:
+        raise SsbaError(SSBA_ERR_INVALID, "x must be a 4-D tensor [N, C, H, W]")
+    N, C, H, W = x.shape
+    _check(x, "x", (N, C, H, W), x.dtype)
+    if y is None:
+        y = torch.empty((N, nb * C, H // 2, W // 2), dtype=x.dtype, device=x.device)
+    _check(y, "y", (N, nb * C, H // 2, W // 2), x.dtype)
+    _raise_on(lib.ssba_haar_dwt(x.data_ptr(), y.data_ptr(), N, C, H, W, nb, _dtype_code(x), _stream_ptr(stream)))
+    return y
+
+
+def haar_iwt(y: torch.Tensor, C: int, nb: int = 4, x=None, stream=None) -> torch.Tensor:
+    """ssba_haar_iwt: y [N, nb*C, h, w] -> [N, C, 2h, 2w]."""
+    lib = load_library()
+    if not isinstance(y, torch.Tensor) or y.dim() != 4:
+        raise SsbaError(SSBA_ERR_INVALID, "y must be a 4-D tensor [N, nb*C, h, w]")
+    N, nbC, h, w = y.shape
+    _check(y, "y", (N, nb * C, h, w), y.dtype)
+    if x is None:
+        x = torch.empty((N, C, 2 * h, 2 * w), dtype=y.dtype, device=y.device)
+    _check(x, "x", (N, C, 2 * h, 2 * w), y.dtype)
+    _raise_on(lib.ssba_haar_iwt(y.data_ptr(), x.data_ptr(), N, C, 2 * h, 2 * w, nb, _dtype_code(y), _stream_ptr(stream)))
+    return x
 
 
 def get_status() -> int:

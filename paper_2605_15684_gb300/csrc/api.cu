@@ -312,6 +312,37 @@ int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, const voi
                            static_cast<float*>(workspace), static_cast<cudaStream_t>(stream));
 }
 
+static int haar_args(const char* who, const void* in, const void* out, int N, int C, int H, int W, int nb,
+                     int dtype)
+{
+    if (!in || !out || N <= 0 || C <= 0 || H <= 0 || W <= 0 || (H & 1) || (W & 1) || (nb != 3 && nb != 4) ||
+        (dtype != SSBA_BF16 && dtype != SSBA_FP32)) {
+        set_error("%s: needs non-null buffers, positive sizes, even H and W, nb 3 or 4 and a known dtype", who);
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(in, 16) || !aligned(out, 16)) {
+        set_error("%s: buffers must be 16-byte aligned", who);
+        return SSBA_ERR_INVALID;
+    }
+    return SSBA_OK;
+}
+
+int ssba_haar_dwt(const void* x, void* y, int32_t N, int32_t C, int32_t H, int32_t W, int32_t nb, int32_t dtype,
+                  void* stream)
+{
+    int rc = haar_args("ssba_haar_dwt", x, y, N, C, H, W, nb, dtype);
+    if (rc != SSBA_OK) return rc;
+    return launch_haar(false, x, y, N, C, H, W, nb, dtype, static_cast<cudaStream_t>(stream));
+}
+
+int ssba_haar_iwt(const void* y, void* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t nb, int32_t dtype,
+                  void* stream)
+{
+    int rc = haar_args("ssba_haar_iwt", y, x, N, C, H, W, nb, dtype);
+    if (rc != SSBA_OK) return rc;
+    return launch_haar(true, y, x, N, C, H, W, nb, dtype, static_cast<cudaStream_t>(stream));
+}
+
 int ssba_get_status(int32_t* device_status_out)
 {
     if (!device_status_out) {

@@ -64,6 +64,9 @@ int launch_backward(const ssba_desc& d, const Grid& g, int keep, float scale, co
                     const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
                     const int32_t* cnt, float* dQ, float* dK, float* dV, float* Dbuf, cudaStream_t st);
 
+int launch_haar(bool inverse, const void* in, void* out, int N, int C, int H, int W, int nb, int dtype,
+                cudaStream_t st);
+
 // Thread-local error text for ssba_last_error().
 void set_error(const char* fmt, ...);
 

@@ -65,3 +65,11 @@ def qkv(B: int, heads: int, N: int, d: int, dtype=torch.bfloat16, seed: int = 0,
 
 def workload_qkv(w: Workload, seed: int = 0):
     return qkv(w.B, w.heads, w.N, w.head_dim, w.dtype, seed, w.std)
+
+
+def feature_map(N: int, C: int, H: int, W: int, dtype=torch.float32, seed: int = 0):
+    """A VAE feature map on the CPU, [N, C, H, W], i.i.d. N(0, 1) drawn in fp32 from one seeded
+    stream, then cast to ``dtype``."""
+    g = torch.Generator(device="cpu")
+    g.manual_seed(int(seed))
+    return torch.randn((N, C, H, W), generator=g, dtype=torch.float32).to(dtype).contiguous()

@@ -146,6 +146,21 @@ def test_backward_validation(lib):
     assert lib.ssba_backward_workspace_bytes(ctypes.byref(desc(H_tok=12))) == 0
 
 
+def test_haar_validation(lib):
+    """The Haar entry points check sizes, band count, dtype and alignment before any launch."""
+    ok = (1, 3, 8, 8, 4, api.SSBA_FP32, None)
+    for fn in (lib.ssba_haar_dwt, lib.ssba_haar_iwt):
+        assert fn(FAKE, FAKE, 1, 3, 7, 8, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID  # odd H
+        assert fn(FAKE, FAKE, 1, 3, 8, 9, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID  # odd W
+        assert fn(FAKE, FAKE, 1, 3, 8, 8, 2, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID  # nb not 3 or 4
+        assert fn(FAKE, FAKE, 0, 3, 8, 8, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID  # empty batch
+        assert fn(FAKE, FAKE, 1, 3, 8, 8, 4, 7, None) == api.SSBA_ERR_INVALID  # unknown dtype
+        assert fn(None, FAKE, *ok) == api.SSBA_ERR_INVALID
+        assert fn(FAKE + 4, FAKE, *ok) == api.SSBA_ERR_INVALID  # misaligned input
+        assert fn(FAKE, FAKE + 8, *ok) == api.SSBA_ERR_INVALID  # misaligned output
+    assert b"ssba_haar_iwt" in lib.ssba_last_error()
+
+
 def test_build_mask_rejects_unsupported_head_dim(lib):
     d = desc(head_dim=12)  # 24 bytes per bf16 row: not a multiple of 16
     ws = lib.ssba_mask_workspace_bytes(ctypes.byref(d))
