@@ -315,3 +315,31 @@ def haar_iwt(y, C: int, nb: int = 4):
     for i in range(ys.shape[0]):
         _check(_load().ssba_oracle_haar_iwt(np.ascontiguousarray(ys[i]), C, 2 * h, 2 * w, nb, x[i]), "haar_iwt")
     return x.reshape(*lead, C, 2 * h, 2 * w)
+
+
+def haar_dwt_pyramid(x, levels: int, nb: int = 4):
+    """The encoder's recursion (Sec. 2.3, Eq. for W^(l)) without the convolutions between
+    levels: level 1 is the bank applied to x, level l the bank applied to the LL band of level
+    l - 1. Returns [W^(1), ..., W^(levels)], W^(l) [..., nb * C, H / 2^l, W / 2^l]."""
+    x = _f64(x)
+    C = x.shape[-3]
+    out, cur = [], x
+    for _ in range(levels):
+        y = haar_dwt(cur, nb)
+        out.append(y)
+        cur = y[..., :C, :, :]  # the LL band of every channel
+    return out
+
+
+def haar_iwt_pyramid(ys, C: int, nb: int = 4):
+    """The decoder's inverse pyramid (Sec. 2.3) without the refinements between levels: the
+    deepest level is inverted whole, and each shallower level is inverted with its LL band
+    replaced by the level below's reconstruction. Only LL of the deepest level and the detail
+    bands are read. Returns x [..., C, H, W]."""
+    cur = None
+    for y in reversed([_f64(t) for t in ys]):
+        if cur is not None:
+            y = y.copy()
+            y[..., :C, :, :] = cur
+        cur = haar_iwt(y, C, nb)
+    return cur

@@ -484,3 +484,43 @@ def test_haar_bands_are_separable_1d_haar():
     np.testing.assert_array_equal(y3, y[:6])
     np.testing.assert_allclose(oracle.haar_iwt(y3, 2, nb=3) + oracle.haar_iwt(
         np.concatenate([np.zeros_like(y[:6]), y[6:]]), 2), x, atol=1e-14)
+
+
+def test_haar_pyramid_closed_forms():
+    """Level L of the pyramid: LL is the sum over each 2^L x 2^L tile divided by 2^L (each
+    orthonormal level doubles a constant); energy splits exactly over LL_L and the detail bands
+    of every level; a constant image has no detail at any level."""
+    rng = np.random.default_rng(72)
+    x = rng.standard_normal((2, 3, 16, 24))
+    L = 3
+    ys = oracle.haar_dwt_pyramid(x, L)
+    assert [y.shape for y in ys] == [(2, 12, 8, 12), (2, 12, 4, 6), (2, 12, 2, 3)]
+    tile = x.reshape(2, 3, 2, 8, 3, 8).sum(axis=(3, 5)) / 2 ** L
+    np.testing.assert_allclose(ys[-1][:, :3], tile, atol=1e-13)
+    energy = (ys[-1][:, :3] ** 2).sum() + sum((y[:, 3:] ** 2).sum() for y in ys)
+    np.testing.assert_allclose(energy, (x ** 2).sum(), rtol=1e-13)
+    yc = oracle.haar_dwt_pyramid(np.full((1, 2, 8, 8), -1.5), 3)
+    for y in yc:
+        np.testing.assert_allclose(y[:, 2:], 0.0, atol=1e-15)
+    np.testing.assert_allclose(yc[-1][:, :2], -1.5 * 8, atol=1e-14)
+
+
+def test_haar_pyramid_inverse_reads_only_deepest_ll_and_details():
+    """The inverse pyramid gives x back, and the LL bands of the shallower levels (which the
+    decoder recomputes) do not enter it; with nb = 3 it loses exactly the HH bands."""
+    rng = np.random.default_rng(73)
+    x = rng.standard_normal((2, 4, 16, 8))
+    ys = oracle.haar_dwt_pyramid(x, 3)
+    np.testing.assert_allclose(oracle.haar_iwt_pyramid(ys, 4), x, atol=1e-13)
+    spoiled = [y.copy() for y in ys]
+    for y in spoiled[:-1]:
+        y[:, :4] = 1e6
+    np.testing.assert_allclose(oracle.haar_iwt_pyramid(spoiled, 4), x, atol=1e-13)
+    y3 = oracle.haar_dwt_pyramid(x, 2, nb=3)
+    np.testing.assert_array_equal(y3[0], ys[0][:, :12])
+    # HH removed at both levels: the inverse equals the full inverse with those bands zeroed
+    zeroed = [ys[0].copy(), ys[1].copy()]
+    zeroed[0][:, 12:] = 0.0
+    zeroed[1][:, 12:] = 0.0
+    np.testing.assert_allclose(oracle.haar_iwt_pyramid(y3, 4, nb=3), oracle.haar_iwt_pyramid(zeroed, 4),
+                               atol=1e-13)
