@@ -424,12 +424,18 @@ def run_ours(args, rank, world):
         hy = torch.empty((hN, 4 * hC, hH // 2, hW // 2), dtype=torch.bfloat16, device=dev)
         hy3 = torch.empty((hN, 3 * hC, hH // 2, hW // 2), dtype=torch.bfloat16, device=dev)
         hb = torch.empty_like(hx)
+        hp = [torch.empty((hN, 4 * hC, hH >> l, hW >> l), dtype=torch.bfloat16, device=dev) for l in (1, 2, 3)]
         nbytes = hx.numel() * 2
+        pyr_bytes = nbytes + 4 * sum(nbytes >> (2 * l) for l in (1, 2, 3))  # x once, 4 bands per level
         peak = hbm_gbs
         out = {}
         for name, fn, moved in (("dwt_nb4", lambda: api.haar_dwt(hx, 4, y=hy, stream=stream), 2 * nbytes),
                                 ("dwt_nb3", lambda: api.haar_dwt(hx, 3, y=hy3, stream=stream), nbytes * 7 // 4),
-                                ("iwt_nb4", lambda: api.haar_iwt(hy, hC, 4, x=hb, stream=stream), 2 * nbytes)):
+                                ("iwt_nb4", lambda: api.haar_iwt(hy, hC, 4, x=hb, stream=stream), 2 * nbytes),
+                                ("dwt_pyramid3", lambda: api.haar_dwt_pyramid(hx, 3, 4, ys=hp, stream=stream),
+                                 pyr_bytes),
+                                ("iwt_pyramid3", lambda: api.haar_iwt_pyramid(hp, hC, 4, x=hb, stream=stream),
+                                 nbytes + 3 * sum(nbytes >> (2 * l) for l in (1, 2, 3)) + (nbytes >> 6))):
             for _ in range(3):
                 fn()
             reps = 10
@@ -444,9 +450,11 @@ def run_ours(args, rank, world):
             out[name] = {"us": t * 1e3, "bytes": moved, "achieved_gbs": gbs,
                          "frac": gbs / peak}
         haar = dict(out, shape=[hN, hC, hH, hW], dtype="bf16", peak_gbs=peak, peak_source=peak_src,
-                    how="ssba_haar_dwt / ssba_haar_iwt back to back, CUDA events around 10 launches; "
-                        "frac of the HBM copy bandwidth")
-        del hx, hy, hy3, hb
+                    how="ssba_haar_dwt / ssba_haar_iwt (one level) and the 3-level pyramids, back to back, "
+                        "CUDA events around 10 launches; bytes: each input element read once, each output "
+                        "element written once (the inverse pyramid reads LL of level 3 and the detail "
+                        "bands); frac of the HBM copy bandwidth")
+        del hx, hy, hy3, hb, hp
     except Exception as exc:  # reported, not fatal
         haar = f"failed: {exc}"
 

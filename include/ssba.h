@@ -202,6 +202,23 @@ SSBA_API int ssba_haar_dwt(const void* x, void* y, int32_t N, int32_t C, int32_t
 SSBA_API int ssba_haar_iwt(const void* y, void* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t nb,
                            int32_t dtype, void* stream);
 
+/* The encoder's Haar recursion (Sec. 2.3, the equation for W^(l)) without the stride-2
+ * convolutions between levels, 1 <= levels <= SSBA_HAAR_MAX_LEVELS: level 1 is the bank on x,
+ * level l the bank on the LL band of level l-1, all levels in one pass over x.
+ *   x     device, [N][C][H][W] of dtype; H and W multiples of 2^levels.
+ *   y     HOST array of `levels` device pointers; y[l-1] is [N][nb*C][H/2^l][W/2^l] of dtype,
+ *         the layout of ssba_haar_dwt (nb = 3 leaves out HH; LL is always written).
+ * All device buffers 16-byte aligned. Returns SSBA_ERR_INVALID for bad sizes or pointers. */
+#define SSBA_HAAR_MAX_LEVELS 3
+SSBA_API int ssba_haar_dwt_pyramid(const void* x, void* const* y, int32_t N, int32_t C, int32_t H, int32_t W,
+                                   int32_t levels, int32_t nb, int32_t dtype, void* stream);
+
+/* The decoder's inverse pyramid (Sec. 2.3) without the refinements between levels: the deepest
+ * level's four bands (HH = 0 when nb = 3) and the detail bands HL, LH (, HH) of every shallower
+ * level give x back; the LL bands of the shallower levels are not read. Same layouts. */
+SSBA_API int ssba_haar_iwt_pyramid(void* const* y, void* x, int32_t N, int32_t C, int32_t H, int32_t W,
+                                   int32_t levels, int32_t nb, int32_t dtype, void* stream);
+
 /* Size of the scratch area built into the library for ssba_build_mask_noalloc (4 MiB). */
 #define SSBA_NOALLOC_SCRATCH_BYTES (4u << 20)
 

@@ -29,7 +29,7 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
             "ssba_test_forward_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
-            "ssba_haar_iwt",
+            "ssba_haar_iwt", "ssba_haar_dwt_pyramid", "ssba_haar_iwt_pyramid",
             "ssba_get_status", "ssba_last_error")
 
 
@@ -121,6 +121,11 @@ def load_library():
         for fn in ("ssba_haar_dwt", "ssba_haar_iwt"):
             getattr(lib, fn).argtypes = [P, P, I, I, I, I, I, I, P]
             getattr(lib, fn).restype = ctypes.c_int
+        PP = ctypes.POINTER(ctypes.c_void_p)
+        lib.ssba_haar_dwt_pyramid.argtypes = [P, PP, I, I, I, I, I, I, I, P]
+        lib.ssba_haar_dwt_pyramid.restype = ctypes.c_int
+        lib.ssba_haar_iwt_pyramid.argtypes = [PP, P, I, I, I, I, I, I, I, P]
+        lib.ssba_haar_iwt_pyramid.restype = ctypes.c_int
         lib.ssba_get_status.argtypes = [ctypes.POINTER(ctypes.c_int32)]
         lib.ssba_get_status.restype = ctypes.c_int
         lib.ssba_last_error.argtypes = []
@@ -442,6 +447,52 @@ def haar_iwt(y: torch.Tensor, C: int, nb: int = 4, x=None, stream=None) -> torch
         x = torch.empty((N, C, 2 * h, 2 * w), dtype=y.dtype, device=y.device)
     _check(x, "x", (N, C, 2 * h, 2 * w), y.dtype)
     _raise_on(lib.ssba_haar_iwt(y.data_ptr(), x.data_ptr(), N, C, 2 * h, 2 * w, nb, _dtype_code(y), _stream_ptr(stream)))
+    return x
+
+
+HAAR_MAX_LEVELS = 3
+
+
+def _ptr_array(ts):
+    return (ctypes.c_void_p * len(ts))(*[t.data_ptr() for t in ts])
+
+
+def haar_dwt_pyramid(x: torch.Tensor, levels: int, nb: int = 4, ys=None, stream=None):
+    """ssba_haar_dwt_pyramid: x [N, C, H, W] -> [W1, ..., W_levels], W_l [N, nb*C, H/2^l, W/2^l]."""
+    lib = load_library()
+    if not isinstance(x, torch.Tensor) or x.dim() != 4:
+        raise SsbaError(SSBA_ERR_INVALID, "x must be a 4-D tensor [N, C, H, W]")
+    N, C, H, W = x.shape
+    _check(x, "x", (N, C, H, W), x.dtype)
+    if not 1 <= levels <= HAAR_MAX_LEVELS:
+        raise SsbaError(SSBA_ERR_INVALID, f"levels must be 1..{HAAR_MAX_LEVELS}")
+    shapes = [(N, nb * C, H >> l, W >> l) for l in range(1, levels + 1)]
+    if ys is None:
+        ys = [torch.empty(shp, dtype=x.dtype, device=x.device) for shp in shapes]
+    if len(ys) != levels:
+        raise SsbaError(SSBA_ERR_INVALID, f"ys must hold {levels} tensors")
+    for l, (t, shp) in enumerate(zip(ys, shapes)):
+        _check(t, f"ys[{l}]", shp, x.dtype)
+    _raise_on(lib.ssba_haar_dwt_pyramid(x.data_ptr(), _ptr_array(ys), N, C, H, W, levels, nb, _dtype_code(x),
+                                        _stream_ptr(stream)))
+    return ys
+
+
+def haar_iwt_pyramid(ys, C: int, nb: int = 4, x=None, stream=None) -> torch.Tensor:
+    """ssba_haar_iwt_pyramid: [W1, ..., W_levels] -> x [N, C, H, W] (W1 is [N, nb*C, H/2, W/2])."""
+    lib = load_library()
+    levels = len(ys)
+    if not 1 <= levels <= HAAR_MAX_LEVELS or not all(isinstance(t, torch.Tensor) and t.dim() == 4 for t in ys):
+        raise SsbaError(SSBA_ERR_INVALID, f"ys must be 1..{HAAR_MAX_LEVELS} 4-D tensors")
+    N, _, h, w = ys[0].shape
+    H, W = 2 * h, 2 * w
+    for l, t in enumerate(ys):
+        _check(t, f"ys[{l}]", (N, nb * C, H >> (l + 1), W >> (l + 1)), ys[0].dtype)
+    if x is None:
+        x = torch.empty((N, C, H, W), dtype=ys[0].dtype, device=ys[0].device)
+    _check(x, "x", (N, C, H, W), ys[0].dtype)
+    _raise_on(lib.ssba_haar_iwt_pyramid(_ptr_array(ys), x.data_ptr(), N, C, H, W, levels, nb, _dtype_code(x),
+                                        _stream_ptr(stream)))
     return x
 
 

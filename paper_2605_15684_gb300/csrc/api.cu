@@ -343,6 +343,42 @@ int ssba_haar_iwt(const void* y, void* x, int32_t N, int32_t C, int32_t H, int32
     return launch_haar(true, y, x, N, C, H, W, nb, dtype, static_cast<cudaStream_t>(stream));
 }
 
+static int pyramid_args(const char* who, const void* x, void* const* y, int N, int C, int H, int W, int levels,
+                        int nb, int dtype)
+{
+    if (levels < 1 || levels > SSBA_HAAR_MAX_LEVELS || !y) {
+        set_error("%s: levels must be 1..%d and y a host array of device pointers", who, SSBA_HAAR_MAX_LEVELS);
+        return SSBA_ERR_INVALID;
+    }
+    const int m = 1 << levels;
+    if (H <= 0 || W <= 0 || H % m || W % m) {
+        set_error("%s: H and W must be positive multiples of 2^levels", who);
+        return SSBA_ERR_INVALID;
+    }
+    for (int l = 0; l < levels; ++l) {
+        int rc = haar_args(who, x, y[l], N, C, H >> l, W >> l, nb, dtype);
+        if (rc != SSBA_OK) return rc;
+    }
+    return SSBA_OK;
+}
+
+int ssba_haar_dwt_pyramid(const void* x, void* const* y, int32_t N, int32_t C, int32_t H, int32_t W, int32_t levels,
+                          int32_t nb, int32_t dtype, void* stream)
+{
+    int rc = pyramid_args("ssba_haar_dwt_pyramid", x, y, N, C, H, W, levels, nb, dtype);
+    if (rc != SSBA_OK) return rc;
+    return launch_haar_pyramid(false, const_cast<void*>(x), y, N, C, H, W, levels, nb, dtype,
+                               static_cast<cudaStream_t>(stream));
+}
+
+int ssba_haar_iwt_pyramid(void* const* y, void* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t levels,
+                          int32_t nb, int32_t dtype, void* stream)
+{
+    int rc = pyramid_args("ssba_haar_iwt_pyramid", x, y, N, C, H, W, levels, nb, dtype);
+    if (rc != SSBA_OK) return rc;
+    return launch_haar_pyramid(true, x, y, N, C, H, W, levels, nb, dtype, static_cast<cudaStream_t>(stream));
+}
+
 int ssba_get_status(int32_t* device_status_out)
 {
     if (!device_status_out) {

@@ -66,6 +66,9 @@ int launch_backward(const ssba_desc& d, const Grid& g, int keep, float scale, co
 
 int launch_haar(bool inverse, const void* in, void* out, int N, int C, int H, int W, int nb, int dtype,
                 cudaStream_t st);
+// Levels 1..SSBA_HAAR_MAX_LEVELS; ys holds one device pointer per level (host array).
+int launch_haar_pyramid(bool inverse, void* x, void* const* ys, int N, int C, int H, int W, int L, int nb, int dtype,
+                        cudaStream_t st);
 
 // Thread-local error text for ssba_last_error().
 void set_error(const char* fmt, ...);

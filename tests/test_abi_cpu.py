@@ -161,6 +161,21 @@ def test_haar_validation(lib):
     assert b"ssba_haar_iwt" in lib.ssba_last_error()
 
 
+def test_haar_pyramid_validation(lib):
+    """Level count, divisibility by 2^levels and every level's pointer are checked first."""
+    import ctypes as ct
+    ys = (ct.c_void_p * 3)(FAKE, FAKE, FAKE)
+    for fn, first in ((lib.ssba_haar_dwt_pyramid, (FAKE, ys)), (lib.ssba_haar_iwt_pyramid, (ys, FAKE))):
+        assert fn(*first, 1, 2, 16, 16, 4, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID  # 4 levels
+        assert fn(*first, 1, 2, 16, 16, 0, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID  # 0 levels
+        assert fn(*first, 1, 2, 12, 16, 3, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID  # 12 % 8
+        assert fn(*first, 1, 2, 16, 20, 3, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID  # 20 % 8
+    bad = (ct.c_void_p * 3)(FAKE, FAKE + 4, FAKE)
+    assert lib.ssba_haar_dwt_pyramid(FAKE, bad, 1, 2, 16, 16, 3, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID
+    assert lib.ssba_haar_dwt_pyramid(FAKE, None, 1, 2, 16, 16, 3, 4, api.SSBA_FP32, None) == api.SSBA_ERR_INVALID
+    assert b"ssba_haar_dwt_pyramid" in lib.ssba_last_error()
+
+
 def test_build_mask_rejects_unsupported_head_dim(lib):
     d = desc(head_dim=12)  # 24 bytes per bf16 row: not a multiple of 16
     ws = lib.ssba_mask_workspace_bytes(ctypes.byref(d))

@@ -106,3 +106,47 @@ def test_into_caller_buffers_and_stream():
     s.synchronize()
     xd = x.double().cpu().numpy()
     _check(y, oracle.haar_dwt(xd, 3), _mag_dwt(xd, 3), torch.float32)
+
+
+PYR_SHAPES = [(1, 1, 8, 8), (2, 3, 16, 24), (1, 5, 24, 40), (2, 2, 32, 12), (1, 16, 256, 264), (1, 4, 4, 4)]
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("nb", [4, 3])
+@pytest.mark.parametrize("levels", [1, 2, 3])
+@pytest.mark.parametrize("shape", PYR_SHAPES)
+def test_pyramid_matches_oracle(shape, levels, nb, dtype):
+    N, C, H, W = shape
+    if H % (1 << levels) or W % (1 << levels):
+        pytest.skip("sizes not divisible by 2^levels")
+    x = _x(shape, dtype, seed=31 * sum(shape) + levels)
+    ys = api.haar_dwt_pyramid(x.cuda(), levels, nb=nb)
+    torch.cuda.synchronize()
+    refs = oracle.haar_dwt_pyramid(x.double().numpy(), levels, nb)
+    # level l's rounding bound: the sum of |x| over its 2^l x 2^l tile, halved l times, with one
+    # rounding per level on the way (bf16 rounds the LL it passes down only in the output)
+    xa = np.abs(x.double().numpy())
+    for l, (got, ref) in enumerate(zip(ys, refs), start=1):
+        t = 1 << l
+        tile = xa.reshape(N, C, H // t, t, W // t, t).sum(axis=(3, 5)) / 2 ** l
+        mag = np.concatenate([tile] * nb, axis=1) * (1 + 2 * l)
+        _check(got, ref, mag, dtype)
+    # the inverse pyramid on the oracle's bands (rounded to dtype)
+    yin = [torch.from_numpy(r).to(dtype) for r in refs]
+    back = api.haar_iwt_pyramid([t.cuda() for t in yin], C, nb=nb)
+    torch.cuda.synchronize()
+    ydn = [t.double().numpy() for t in yin]
+    ref_back = oracle.haar_iwt_pyramid(ydn, C, nb)
+    mag = sum(np.repeat(np.repeat(0.5 * np.abs(y).reshape(N, nb, C, *y.shape[2:]).sum(axis=1), 1 << l, axis=2),
+                        1 << l, axis=3) for l, y in enumerate(ydn, start=1)) * 4
+    _check(back, ref_back, mag, dtype)
+
+
+def test_pyramid_round_trip_fp32_and_ignored_ll():
+    x = _x((2, 6, 64, 48), torch.float32, seed=9).cuda()
+    ys = api.haar_dwt_pyramid(x, 3)
+    ys[0][:, :6] = 1e6  # shallower LL bands are not read by the inverse
+    ys[1][:, :6] = -1e6
+    back = api.haar_iwt_pyramid(ys, 6)
+    torch.cuda.synchronize()
+    assert torch.allclose(back, x, rtol=0, atol=64 * U * float(x.abs().max()))
