@@ -343,3 +343,55 @@ def haar_iwt_pyramid(ys, C: int, nb: int = 4):
             y[..., :C, :, :] = cur
         cur = haar_iwt(y, C, nb)
     return cur
+
+
+ROPE_BASE = 10000.0
+
+
+def rope_2d(x, H: int, W: int, base: float = ROPE_BASE):
+    """Rotary position embedding of image tokens (Algorithm 1, first step), 2-D axial
+    reading: x [..., N, d] with N = H*W tokens in row-major grid order; the first d/2
+    dimensions rotate with the token's row r, the last d/2 with its column c. Within each
+    half, the pair (2i, 2i+1) turns by pos * theta_i, theta_i = base^(-i / (d/4))."""
+    x = _f64(x)
+    N, d = x.shape[-2], x.shape[-1]
+    if N != H * W or d % 4:
+        raise ValueError("rope_2d: N must equal H*W and d be a multiple of 4")
+    half, nf = d // 2, d // 4
+    theta = base ** (-np.arange(nf, dtype=np.float64) / nf)
+    n = np.arange(N)
+    out = x.copy()
+    for off, pos in ((0, n // W), (half, n % W)):
+        ang = pos[:, None].astype(np.float64) * theta[None, :]
+        cos, sin = np.cos(ang), np.sin(ang)
+        even = x[..., off:off + half:2]
+        odd = x[..., off + 1:off + half:2]
+        out[..., off:off + half:2] = even * cos - odd * sin
+        out[..., off + 1:off + half:2] = even * sin + odd * cos
+    return out
+
+
+def qkv_rope(X, Wqkv, bias, heads: int, H: int, W: int, d: int = 64):
+    """The QKV projection and RoPE that precede the mask build (Algorithm 1): X [B, N, Dm],
+    Wqkv [3 * heads * d, Dm] (rows: Q heads, then K heads, then V heads), bias [3 * heads * d]
+    or None. Returns Q, K, V [B, heads, N, d] with RoPE applied to Q and K."""
+    X, Wqkv = _f64(X), _f64(Wqkv)
+    B, N, Dm = X.shape
+    Y = X @ Wqkv.T
+    if bias is not None:
+        Y = Y + _f64(bias)
+    Y = Y.reshape(B, N, 3, heads, d).transpose(2, 0, 3, 1, 4)  # [3, B, heads, N, d]
+    return rope_2d(Y[0], H, W), rope_2d(Y[1], H, W), np.ascontiguousarray(Y[2])
+
+
+def pooled_blocks(X, H: int, W: int, blk: int = 8, shift=(0, 0)):
+    """Block means of every (batch, head): X [B, heads, N, d] -> [B, heads, Tb, d]."""
+    X = _f64(X)
+    B, h, N, d = X.shape
+    lab = partition(H, W, blk, shift)
+    Tb = N // (blk * blk)
+    out = np.empty((B, h, Tb, d), dtype=np.float64)
+    for b in range(B):
+        for i in range(h):
+            out[b, i] = pool(X[b, i], lab, Tb)
+    return out

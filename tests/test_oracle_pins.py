@@ -524,3 +524,72 @@ def test_haar_pyramid_inverse_reads_only_deepest_ll_and_details():
     zeroed[1][:, 12:] = 0.0
     np.testing.assert_allclose(oracle.haar_iwt_pyramid(y3, 4, nb=3), oracle.haar_iwt_pyramid(zeroed, 4),
                                atol=1e-13)
+
+
+# ----------------------------------------------------------------------------- RoPE + QKV
+def test_rope_hand_values_and_axes():
+    """theta_0 = 1 rad: a unit vector on dimension 0 at row 1 turns to (cos 1, sin 1); on
+    dimension 32 at column 2 to (cos 2, sin 2); dimension 2 turns by 10000^(-1/16) per row;
+    a row displacement leaves the column half alone and vice versa; token (0, 0) is unchanged."""
+    H, W, d = 3, 4, 64
+    x = np.zeros((H * W, d))
+    x[:, 0] = 1.0
+    x[:, 2] = 1.0
+    x[:, 32] = 1.0
+    y = oracle.rope_2d(x, H, W)
+    t = 1 * W + 0  # row 1, column 0
+    np.testing.assert_allclose(y[t, :2], [np.cos(1.0), np.sin(1.0)], atol=1e-15)
+    th1 = 10000.0 ** (-1 / 16)
+    np.testing.assert_allclose(y[t, 2:4], [np.cos(th1), np.sin(th1)], atol=1e-15)
+    np.testing.assert_allclose(y[t, 32:34], [1.0, 0.0], atol=1e-15)  # column 0: no turn
+    t = 0 * W + 2  # row 0, column 2
+    np.testing.assert_allclose(y[t, 32:34], [np.cos(2.0), np.sin(2.0)], atol=1e-15)
+    np.testing.assert_allclose(y[t, :4], [1.0, 0.0, 1.0, 0.0], atol=1e-15)
+    np.testing.assert_array_equal(y[0], x[0])
+
+
+def test_rope_is_a_rotation_with_relative_positions():
+    """Norms are kept pair by pair, and <R q(p1), R k(p2)> depends only on p1 - p2 on each axis."""
+    rng = np.random.default_rng(80)
+    H, W, d = 6, 7, 64
+    q, k = rng.standard_normal(d), rng.standard_normal(d)
+    Rq = oracle.rope_2d(np.tile(q, (H * W, 1)), H, W)
+    Rk = oracle.rope_2d(np.tile(k, (H * W, 1)), H, W)
+    np.testing.assert_allclose((Rq.reshape(-1, 32, 2) ** 2).sum(-1), np.tile((q.reshape(32, 2) ** 2).sum(-1), (H * W, 1)),
+                               rtol=1e-13)
+    tok = lambda r, c: r * W + c
+    for (r1, c1), (r2, c2), (dr, dc) in (((1, 2), (0, 0), (2, 3)), ((4, 1), (2, 5), (1, 1)), ((0, 6), (3, 0), (2, 0))):
+        a = Rq[tok(r1, c1)] @ Rk[tok(r2, c2)]
+        b = Rq[tok(r1 + dr, c1 + dc)] @ Rk[tok(r2 + dr, c2 + dc)]
+        np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-12)
+    # and does change with the offset
+    assert abs(Rq[tok(1, 2)] @ Rk[tok(0, 0)] - Rq[tok(1, 3)] @ Rk[tok(0, 0)]) > 1e-6
+
+
+def test_qkv_projection_layout_and_bias():
+    """With Wqkv = [I; 2I; 3I] the projection is X, 2X, 3X cut into heads of 64 consecutive
+    channels (Q rows first, then K, then V); the bias is added once; RoPE turns Q and K only."""
+    rng = np.random.default_rng(81)
+    B, H, W, heads, d = 2, 4, 4, 3, 64
+    Dm = heads * d
+    X = rng.standard_normal((B, H * W, Dm))
+    Wqkv = np.concatenate([np.eye(Dm), 2 * np.eye(Dm), 3 * np.eye(Dm)])
+    Q, K, V = oracle.qkv_rope(X, Wqkv, None, heads, H, W)
+    heads_of = lambda Y: Y.reshape(B, H * W, heads, d).transpose(0, 2, 1, 3)
+    np.testing.assert_allclose(Q, oracle.rope_2d(heads_of(X), H, W), atol=1e-14)
+    np.testing.assert_allclose(K, oracle.rope_2d(heads_of(2 * X), H, W), atol=1e-14)
+    np.testing.assert_allclose(V, heads_of(3 * X), atol=1e-14)
+    bias = rng.standard_normal(3 * Dm)
+    Q2, K2, V2 = oracle.qkv_rope(X, Wqkv, bias, heads, H, W)
+    np.testing.assert_allclose(V2 - V, np.broadcast_to(bias[2 * Dm:].reshape(heads, 1, d), V.shape), atol=1e-14)
+    np.testing.assert_allclose(Q2[:, :, 0] - Q[:, :, 0], np.broadcast_to(bias[:Dm].reshape(heads, d), (B, heads, d)),
+                               atol=1e-14)  # token (0, 0): RoPE is the identity there
+
+
+def test_pooled_blocks_matches_pool_of_each_head():
+    rng = np.random.default_rng(82)
+    X = rng.standard_normal((1, 2, 16 * 16, 64))
+    P = oracle.pooled_blocks(X, 16, 16, 8, (4, 4))
+    lab = oracle.partition(16, 16, 8, (4, 4))
+    for b in range(4):
+        np.testing.assert_allclose(P[0, 1, b], X[0, 1][lab == b].mean(axis=0), atol=1e-14)
