@@ -79,8 +79,8 @@ typedef struct {
  * Returns -1 for an invalid descriptor. */
 SSBA_API int ssba_keep_count(const ssba_desc* desc);
 
-/* Bytes of device workspace ssba_build_mask needs (the pooled block sums of Q
- * and K in fp32, 2 * B * heads * Tb * head_dim * 4 bytes, 256-byte aligned).
+/* Bytes of device workspace ssba_build_mask needs (the block means of Q and K
+ * in fp32, 2 * B * heads * Tb * head_dim * 4 bytes, 256-byte aligned).
  * Returns 0 for an invalid descriptor. */
 SSBA_API size_t ssba_mask_workspace_bytes(const ssba_desc* desc);
 
@@ -218,6 +218,29 @@ SSBA_API int ssba_haar_dwt_pyramid(const void* x, void* const* y, int32_t N, int
  * level give x back; the LL bands of the shallower levels are not read. Same layouts. */
 SSBA_API int ssba_haar_iwt_pyramid(void* const* y, void* x, int32_t N, int32_t C, int32_t H, int32_t W,
                                    int32_t levels, int32_t nb, int32_t dtype, void* stream);
+
+/* The steps of Algorithm 1 before the mask, fused: the QKV projection of the image tokens,
+ * RoPE on Q and K (Algorithm 1, first step; 2-D axial: dimensions [0, 32) turn with the
+ * token's row, [32, 64) with its column, pair (2i, 2i+1) by pos * 10000^(-i/16)), and the
+ * block compression of Sec. 2.2 (block means of Q and K over the layer's shifted 8x8 windows).
+ *   X       device, bf16 [B][N][Dm], Dm = heads * 64, tokens in grid order (n = r * W_tok + c).
+ *   Wqkv    device, bf16 [3 * Dm][Dm] (output channel-major: Q heads, then K, then V).
+ *   bias    device fp32 [3 * Dm], or NULL.
+ *   Q, K, V device out, bf16 [B][heads][N][64] (RoPE applied to Q and K).
+ *   qb, kb  device out, fp32 [B][heads][Tb][64]: means of the bf16 Q and K over each block of
+ *           the shifted grid (the layout ssba_select_mask reads); both NULL to skip them.
+ * desc: dtype SSBA_BF16, head_dim 64, block 8, shifts multiples of 4. All device pointers
+ * 16-byte aligned. fp32 accumulation. Returns SSBA_ERR_UNSUPPORTED for other shapes. */
+SSBA_API int ssba_qkv_rope_pool(const ssba_desc* desc, const void* X, const void* Wqkv, const float* bias, void* Q,
+                                void* K, void* V, float* qb, float* kb, void* stream);
+
+/* The mask from block means already computed (Sec. 2.2 Affinity Matrix and Top-k Gating;
+ * Algorithm 1 from "S <- q_b k_b^T" on): the second half of ssba_build_mask, for callers that
+ * pooled in the projection (ssba_qkv_rope_pool).
+ *   qb, kb  device, fp32 [B][heads][Tb][head_dim], 16-byte aligned.
+ *   kv_idx, kv_cnt, scores_opt as for ssba_build_mask. Ties keep the lower label. */
+SSBA_API int ssba_select_mask(const ssba_desc* desc, const float* qb, const float* kb, int32_t* kv_idx,
+                              int32_t* kv_cnt, float* scores_opt, void* stream);
 
 /* Size of the scratch area built into the library for ssba_build_mask_noalloc (4 MiB). */
 #define SSBA_NOALLOC_SCRATCH_BYTES (4u << 20)

@@ -29,7 +29,8 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
             "ssba_test_forward_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
-            "ssba_haar_iwt", "ssba_haar_dwt_pyramid", "ssba_haar_iwt_pyramid",
+            "ssba_haar_iwt", "ssba_haar_dwt_pyramid", "ssba_haar_iwt_pyramid", "ssba_qkv_rope_pool",
+            "ssba_select_mask",
             "ssba_get_status", "ssba_last_error")
 
 
@@ -103,6 +104,10 @@ def load_library():
         lib.ssba_build_mask.restype = ctypes.c_int
         lib.ssba_build_mask_noalloc.argtypes = [DP, P, P, P, P, P, P]
         lib.ssba_build_mask_noalloc.restype = ctypes.c_int
+        lib.ssba_qkv_rope_pool.argtypes = [DP, P, P, P, P, P, P, P, P, P]
+        lib.ssba_qkv_rope_pool.restype = ctypes.c_int
+        lib.ssba_select_mask.argtypes = [DP, P, P, P, P, P, P]
+        lib.ssba_select_mask.restype = ctypes.c_int
         lib.ssba_forward.argtypes = [DP, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_forward.restype = ctypes.c_int
         lib.ssba_forward_joint.argtypes = [DP, P, P, P, P, P, ctypes.c_int32, P, P, P, P, P, ctypes.c_size_t, P]
@@ -236,6 +241,65 @@ def build_mask(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=None, kv
                              workspace.data_ptr(), workspace.numel() * workspace.element_size(),
                              _stream_ptr(stream))
     _raise_on(rc)
+    return (kv_idx, kv_cnt, S) if S is not None else (kv_idx, kv_cnt)
+
+
+def qkv_rope_pool(desc: SsbaDesc, X: torch.Tensor, Wqkv: torch.Tensor, bias=None, pooled: bool = True,
+                  out=None, stream=None):
+    """ssba_qkv_rope_pool: X [B, N, heads*64] -> (Q, K, V [B, heads, N, 64] bf16 with RoPE on Q
+    and K, qb, kb [B, heads, Tb, 64] fp32 block means, or None when pooled is False)."""
+    lib = load_library()
+    d = desc.c()
+    Dm = desc.heads * desc.head_dim
+    _check(X, "X", (desc.B, desc.N, Dm), torch.bfloat16)
+    _check(Wqkv, "Wqkv", (3 * Dm, Dm), torch.bfloat16)
+    if bias is not None:
+        _check(bias, "bias", (3 * Dm,), torch.float32)
+    dev = X.device
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    pshp = (desc.B, desc.heads, desc.Tb, desc.head_dim)
+    if out is None:
+        out = [torch.empty(shp, dtype=torch.bfloat16, device=dev) for _ in range(3)]
+        out += [torch.empty(pshp, dtype=torch.float32, device=dev) for _ in range(2)] if pooled else [None, None]
+    Q, K, V, qb, kb = out
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
+        _check(t, n, shp, torch.bfloat16)
+    for t, n in ((qb, "qb"), (kb, "kb")):
+        if t is not None:
+            _check(t, n, pshp, torch.float32)
+    _raise_on(lib.ssba_qkv_rope_pool(ctypes.byref(d), X.data_ptr(), Wqkv.data_ptr(),
+                                     bias.data_ptr() if bias is not None else None, Q.data_ptr(), K.data_ptr(),
+                                     V.data_ptr(), qb.data_ptr() if qb is not None else None,
+                                     kb.data_ptr() if kb is not None else None, _stream_ptr(stream)))
+    return Q, K, V, qb, kb
+
+
+def select_mask(desc: SsbaDesc, qb: torch.Tensor, kb: torch.Tensor, kv_idx=None, kv_cnt=None,
+                scores: bool | torch.Tensor = False, stream=None):
+    """ssba_select_mask: block means -> (kv_idx, kv_cnt[, S]) as build_mask returns them."""
+    lib = load_library()
+    d = desc.c()
+    keep = lib.ssba_keep_count(ctypes.byref(d))
+    if keep < 0:
+        _raise_on(SSBA_ERR_INVALID)
+    pshp = (desc.B, desc.heads, desc.Tb, desc.head_dim)
+    _check(qb, "qb", pshp, torch.float32)
+    _check(kb, "kb", pshp, torch.float32)
+    dev = qb.device
+    if kv_idx is None:
+        kv_idx = torch.empty((desc.B, desc.heads, desc.Tb, keep), dtype=torch.int32, device=dev)
+    if kv_cnt is None:
+        kv_cnt = torch.empty((desc.B, desc.heads, desc.Tb), dtype=torch.int32, device=dev)
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    S = None
+    if isinstance(scores, torch.Tensor):
+        S = scores
+        _check(S, "scores", (desc.B, desc.heads, desc.Tb, desc.Tb), torch.float32)
+    elif scores:
+        S = torch.empty((desc.B, desc.heads, desc.Tb, desc.Tb), dtype=torch.float32, device=dev)
+    _raise_on(lib.ssba_select_mask(ctypes.byref(d), qb.data_ptr(), kb.data_ptr(), kv_idx.data_ptr(),
+                                   kv_cnt.data_ptr(), S.data_ptr() if S is not None else None, _stream_ptr(stream)))
     return (kv_idx, kv_cnt, S) if S is not None else (kv_idx, kv_cnt)
 
 

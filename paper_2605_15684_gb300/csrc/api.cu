@@ -158,6 +158,48 @@ int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K, int32_t
     return launch_select(*desc, g, keep, qb, kb, kv_idx, kv_cnt, scores_opt, st);
 }
 
+int ssba_qkv_rope_pool(const ssba_desc* desc, const void* X, const void* Wqkv, const float* bias, void* Q, void* K,
+                       void* V, float* qb, float* kb, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_qkv_rope_pool", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!X || !Wqkv || !Q || !K || !V || (!qb) != (!kb)) {
+        set_error("ssba_qkv_rope_pool: X, Wqkv, Q, K, V must be non-null, and qb, kb both set or both NULL");
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(X, 16) || !aligned(Wqkv, 16) || !aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) ||
+        (bias && !aligned(bias, 16)) || (qb && (!aligned(qb, 16) || !aligned(kb, 16)))) {
+        set_error("ssba_qkv_rope_pool: every device pointer must be 16-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    return launch_qkv_rope_pool(*desc, g, X, Wqkv, bias, Q, K, V, qb, kb, static_cast<cudaStream_t>(stream));
+}
+
+int ssba_select_mask(const ssba_desc* desc, const float* qb, const float* kb, int32_t* kv_idx, int32_t* kv_cnt,
+                     float* scores_opt, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_select_mask", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!qb || !kb || !kv_idx || !kv_cnt) {
+        set_error("ssba_select_mask: qb, kb, kv_idx and kv_cnt must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    if (desc->head_dim % 4 || desc->head_dim > 256) {
+        set_error("ssba_select_mask: head_dim must be a multiple of 4 and at most 256");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    if (!aligned(qb, 16) || !aligned(kb, 16) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) ||
+        (scores_opt && !aligned(scores_opt, 4))) {
+        set_error("ssba_select_mask: qb and kb must be 16-byte aligned, outputs 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    return launch_select(*desc, g, keep, qb, kb, kv_idx, kv_cnt, scores_opt, static_cast<cudaStream_t>(stream));
+}
+
 size_t ssba_forward_workspace_bytes(const ssba_desc* desc)
 {
     Grid g;

@@ -66,6 +66,10 @@ int launch_backward(const ssba_desc& d, const Grid& g, int keep, float scale, co
 
 int launch_haar(bool inverse, const void* in, void* out, int N, int C, int H, int W, int nb, int dtype,
                 cudaStream_t st);
+int launch_qkv_rope_pool(const ssba_desc& d, const Grid& g, const void* X, const void* Wqkv, const float* bias,
+                         void* Q, void* K, void* V, float* qb, float* kb, cudaStream_t st,
+                         uint64_t budget_ns = kWaitBudgetNs);
+
 // Levels 1..SSBA_HAAR_MAX_LEVELS; ys holds one device pointer per level (host array).
 int launch_haar_pyramid(bool inverse, void* x, void* const* ys, int N, int C, int H, int W, int L, int nb, int dtype,
                         cudaStream_t st);

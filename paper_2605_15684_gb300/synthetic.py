@@ -73,3 +73,15 @@ def feature_map(N: int, C: int, H: int, W: int, dtype=torch.float32, seed: int =
     g = torch.Generator(device="cpu")
     g.manual_seed(int(seed))
     return torch.randn((N, C, H, W), generator=g, dtype=torch.float32).to(dtype).contiguous()
+
+
+def projection_inputs(B: int, N: int, Dm: int, seed: int = 0):
+    """Image-token activations and a QKV projection, on the CPU, drawn in this order from one
+    seeded stream: X [B, N, Dm] ~ N(0, 1) cast to bf16, Wqkv [3 Dm, Dm] ~ N(0, 1/Dm) cast to
+    bf16 (so that every projected channel has unit variance), bias [3 Dm] ~ N(0, 0.1^2) fp32."""
+    g = torch.Generator(device="cpu")
+    g.manual_seed(int(seed))
+    X = torch.randn((B, N, Dm), generator=g, dtype=torch.float32).to(torch.bfloat16).contiguous()
+    Wqkv = (torch.randn((3 * Dm, Dm), generator=g, dtype=torch.float32) / Dm ** 0.5).to(torch.bfloat16).contiguous()
+    bias = (0.1 * torch.randn((3 * Dm,), generator=g, dtype=torch.float32)).contiguous()
+    return X, Wqkv, bias

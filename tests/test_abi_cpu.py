@@ -176,6 +176,35 @@ def test_haar_pyramid_validation(lib):
     assert b"ssba_haar_dwt_pyramid" in lib.ssba_last_error()
 
 
+def test_qkv_and_select_validation(lib):
+    """The fused projection and the selection check pointers, pairing and shape first."""
+    d = desc()
+    good = [FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE]  # X W bias Q K V qb kb
+    args = lambda v: [ct_byref(d)] + v + [None]
+    bad = list(good)
+    bad[6] = None  # qb without kb
+    assert lib.ssba_qkv_rope_pool(*args(bad)) == api.SSBA_ERR_INVALID
+    bad = list(good)
+    bad[0] = None
+    assert lib.ssba_qkv_rope_pool(*args(bad)) == api.SSBA_ERR_INVALID
+    bad = list(good)
+    bad[3] = FAKE + 8
+    assert lib.ssba_qkv_rope_pool(*args(bad)) == api.SSBA_ERR_INVALID
+    d32 = desc(dtype=api.SSBA_FP32)
+    assert lib.ssba_qkv_rope_pool(ct_byref(d32), *good, None) == api.SSBA_ERR_UNSUPPORTED
+    dsh = desc(shift_r=3)
+    assert lib.ssba_qkv_rope_pool(ct_byref(dsh), *good, None) == api.SSBA_ERR_UNSUPPORTED
+    assert b"multiples of 4" in lib.ssba_last_error()
+    assert lib.ssba_select_mask(ct_byref(d), None, FAKE, FAKE, FAKE, None, None) == api.SSBA_ERR_INVALID
+    assert lib.ssba_select_mask(ct_byref(d), FAKE + 4, FAKE, FAKE, FAKE, None, None) == api.SSBA_ERR_INVALID
+    assert lib.ssba_select_mask(ct_byref(desc(head_dim=66)), FAKE, FAKE, FAKE, FAKE, None, None) == \
+        api.SSBA_ERR_UNSUPPORTED
+
+
+def ct_byref(d):
+    return ctypes.byref(d)
+
+
 def test_build_mask_rejects_unsupported_head_dim(lib):
     d = desc(head_dim=12)  # 24 bytes per bf16 row: not a multiple of 16
     ws = lib.ssba_mask_workspace_bytes(ctypes.byref(d))
