@@ -30,6 +30,7 @@
 // All mbarrier waits are bounded (globaltimer budget + CTA abort flag); a timeout is written
 // to the device status word and the CTA drains its in-flight copies and MMAs before exiting.
 #include <cuda.h>
+#include <cstddef>
 #include <cstring>
 
 #include "common.cuh"
@@ -88,11 +89,18 @@ struct __align__(1024) QkvSmem {
     uint64_t acc_full[2], acc_empty[2];
     uint64_t drain;
     uint64_t pool_full[2], pool_free[2];  // per head pair: the quadrants' sums written / taken
+    uint64_t bias_full[2];                // per accumulator: the tile's bias has landed
+    alignas(16) float bias[2][kBN];       // per accumulator: the tile's 256 biases (bulk-copy target)
     float part[2][4][2][2][2][32];        // [head pair][quadrant][head][chunk][window][column]
     float2 rope[kNumFreq][kRopeCap];  // (cos, sin) of pos * theta_i
     uint32_t tmem_base;
     int abort_flag;
 };
+
+// every TMA / bulk-copy destination starts on the alignment its copy needs
+static_assert(offsetof(QkvSmem, a) % 1024 == 0 && offsetof(QkvSmem, b) % 1024 == 0, "stage alignment");
+static_assert(kABytes % 1024 == 0 && kBBytes % 1024 == 0, "stage size");
+static_assert(offsetof(QkvSmem, bias) % 16 == 0 && (kBN * sizeof(float)) % 16 == 0, "bias alignment");
 
 // A tile's rows: the pair of windows (window row wr, windows 2 pp and 2 pp + 1) of one image,
 // a 16 x 8 region of the rolled grid (8 x 8 when the row has an odd last window). Its origin
@@ -173,6 +181,14 @@ __device__ __forceinline__ void tile_rc(const TileGeo& o, int rho, int& a, int& 
     }
 }
 
+// One bulk copy global -> shared (16-byte aligned, size a multiple of 16), counted on bar.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
 __device__ __forceinline__ uint32_t pack2(float lo, float hi)
 {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -219,6 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
         for (int hp = 0; hp < 2; ++hp) {
             mbar_init(smem_u32(&sm.pool_full[hp]), 4);
             mbar_init(smem_u32(&sm.pool_free[hp]), 1);
+            mbar_init(smem_u32(&sm.bias_full[hp]), 1);
         }
         fence_mbar_init();
     }
@@ -270,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         const bool leader = elect_one_sync();
-        uint32_t gstep = 0, it = 0;
+        uint32_t gstep = 0, it = 0, nbias = 0;
         const uint32_t a0 = smem_u32(&sm.a[0][0]), b0 = smem_u32(&sm.b[0][0]);
         for (int t = blockIdx.x; t < p.tiles && !dead; t += gridDim.x, ++it) {
             const uint32_t acc = it & 1;
@@ -279,6 +296,15 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
                 break;
             }
             tc_fence_after();
+            if (p.bias && lane == 0) {
+                // the tile's biases, for the epilogue, into the buffer of this accumulator
+                const int c0 = (t % p.n_tiles) * kBN;
+                const uint32_t bytes = (uint32_t)min(kBN, 3 * p.Dm - c0) * 4;
+                mbar_arrive_expect_tx(smem_u32(&sm.bias_full[acc]), bytes);
+                bulk_load(smem_u32(&sm.bias[acc][0]), p.bias + c0, bytes, smem_u32(&sm.bias_full[acc]));
+                ++nbias;
+            }
+            __syncwarp();
             const uint32_t d = tbase + acc * kBN;
             for (int ks = 0; ks < ksteps; ++ks, ++gstep) {
                 const uint32_t s = gstep % kStages;
@@ -303,6 +329,11 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
             mma_commit(smem_u32(&sm.drain));
             wait_raw_q(smem_u32(&sm.drain), 0, p.budget_ns);
         }
+        if (dead && lane == 0 && nbias > 0) {
+            // the last bias copy issued may still be in flight
+            const uint32_t last = nbias - 1;  // every tile issues one copy: this is its tile count
+            wait_raw_q(smem_u32(&sm.bias_full[last & 1]), (last >> 1) & 1, p.budget_ns);
+        }
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
@@ -319,6 +350,15 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
             const bool valid = rho < 8 * o.wd;
             const int tok = valid ? g.token(o.L0 + win, ra * 8 + (rc & 7)) : 0;
             const int tpos[2] = {tok / g.W, tok % g.W};  // RoPE positions: row, column
+            // stores go out transposed within groups of four lanes (see below): the tokens and
+            // validity of the group's rows
+            int tokm[4];
+            bool validm[4];
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+                tokm[m] = __shfl_sync(0xffffffffu, tok, (lane & ~3) | m);
+                validm[m] = __shfl_sync(0xffffffffu, (int)valid, (lane & ~3) | m) != 0;
+            }
             const bool regular = o.wd == 16 && o.w1 == 0;  // window = bit 3 of the lane
             const int b = o.b, nt = o.nt;
             const uint32_t acc = it & 1;
@@ -327,6 +367,8 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
                 break;
             }
             tc_fence_after();
+            if (p.bias && !mbar_wait(smem_u32(&sm.bias_full[acc]), (it >> 1) & 1, abortf, p.budget_ns)) dead = true;
+            const float* bias_t = sm.bias[acc];
             // the warp's heads pool when they hold Q or K (the same for the four quadrants of a
             // head pair, so that their handshake counts agree)
             const int col0 = nt * kBN + hp * 2 * kD;
@@ -342,16 +384,19 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
                 if (dead || col >= 3 * p.Dm) continue;
                 const int which = col / p.Dm, head = (col - which * p.Dm) / kD;
                 __nv_bfloat16* outp = which == 0 ? p.q : (which == 1 ? p.k : p.v);
-                uint4* dst = reinterpret_cast<uint4*>(outp + (((size_t)b * p.heads + head) * N + tok) * kD);
+                __nv_bfloat16* headp = outp + ((size_t)b * p.heads + head) * N * kD;
+                // both chunks of the head from TMEM behind one wait
+                uint32_t rr[2][32];
+                {
+                    const uint32_t taddr = tbase + ((uint32_t)(32 * quad) << 16) + acc * kBN + (col - nt * kBN);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        tmem_ld_32x32b_x16(taddr + 16 * j, *reinterpret_cast<uint32_t(*)[16]>(&rr[j >> 1][16 * (j & 1)]));
+                    tmem_wait_ld();
+                }
 #pragma unroll
                 for (int ch = 0; ch < 2; ++ch) {  // chunk 0: dims [0, 32) turn with the row, chunk 1 with the column
-                    // bias and cos/sin first: the TMEM wait below is a compiler barrier, and
-                    // loads issued after it expose their whole latency
-                    float4 bb[8];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        bb[e] = p.bias ? __ldg(reinterpret_cast<const float4*>(p.bias + col + 32 * ch) + e)
-                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+                    const uint32_t(&r)[32] = rr[ch];
                     float2 cs[kNumFreq];
                     if (which < 2) {
                         const int pos = tpos[ch];
@@ -363,11 +408,11 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
                                 sincosf((float)pos * p.theta[i], &cs[i].y, &cs[i].x);
                         }
                     }
-                    uint32_t r[32];
-                    const uint32_t taddr = tbase + ((uint32_t)(32 * quad) << 16) + acc * kBN + (col - nt * kBN) + 32 * ch;
-                    tmem_ld_32x32b_x16(taddr, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-                    tmem_ld_32x32b_x16(taddr + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-                    tmem_wait_ld();
+                    float4 bb[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        bb[e] = p.bias ? reinterpret_cast<const float4*>(bias_t + (col - nt * kBN) + 32 * ch)[e]
+                                       : make_float4(0.f, 0.f, 0.f, 0.f);
                     float v[32];
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
@@ -387,10 +432,39 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
                     uint32_t o[16];
 #pragma unroll
                     for (int i = 0; i < 16; ++i) o[i] = pack2(v[2 * i], v[2 * i + 1]);
-                    if (valid) {
+                    {
+                        // 4 x 4 transpose of 16-byte pieces within each group of four lanes, so
+                        // that store m writes 64 contiguous bytes of row (group + m) from four
+                        // lanes: 8 lines per store instead of 32 (measured: the 32-line stores
+                        // held the next chunk's shared-memory loads for ~2800 cycles)
+                        uint4 X[4];
 #pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            dst[4 * ch + i] = make_uint4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+                        for (int i = 0; i < 4; ++i) X[i] = make_uint4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+                        const int k4 = lane & 3;
+#pragma unroll
+                        for (int stage = 0; stage < 2; ++stage) {
+                            const int bit = 1 << stage;
+                            const bool hi = k4 & bit;
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                if (q & bit) continue;  // slot pairs (q, q + bit)
+                                const uint4 send = hi ? X[q] : X[q + bit];
+                                uint4 recv;
+                                recv.x = __shfl_xor_sync(0xffffffffu, send.x, bit);
+                                recv.y = __shfl_xor_sync(0xffffffffu, send.y, bit);
+                                recv.z = __shfl_xor_sync(0xffffffffu, send.z, bit);
+                                recv.w = __shfl_xor_sync(0xffffffffu, send.w, bit);
+                                if (hi)
+                                    X[q] = recv;
+                                else
+                                    X[q + bit] = recv;
+                            }
+                        }
+                        // X[m] = piece k4 of row (group + m)
+#pragma unroll
+                        for (int m = 0; m < 4; ++m)
+                            if (validm[m])
+                                *reinterpret_cast<uint4*>(headp + (size_t)tokm[m] * kD + 32 * ch + 8 * k4) = X[m];
                     }
                     if (pool_tile && which < 2) {
                         // column sums of the rounded values over the quadrant's rows, per window
