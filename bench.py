@@ -458,6 +458,74 @@ def run_ours(args, rank, world):
     except Exception as exc:  # reported, not fatal
         haar = f"failed: {exc}"
 
+    def events_ms(fn, reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    # ---- layer-aware sparsity: the same 24 layers with the synthetic per-layer schedule
+    #      (edge layers at 75 %, the middle sparser, 84.16 % on average); outside the timed region
+    layer_aware = None
+    try:
+        from paper_2605_15684_gb300 import schedule
+        rhos = schedule.layer_rhos(L, Tb)
+        ldescs = [api.SsbaDesc(w.B, w.heads, w.H_tok, w.W_tok, w.head_dim, 8, *layer_shift(l), rhos[l], w.dtype)
+                  for l in range(L)]
+        lkeep = [api.keep_count(d) for d in ldescs]
+        lidx = [torch.empty((w.B, w.heads, Tb, k), dtype=torch.int32, device=dev) for k in lkeep]
+        llayers = [api.BoundLayer(ldescs[l], Qs[l], Ks[l], Vs[l], lidx[l], cnt[l], Os[l], lses[l], ws, stream)
+                   for l in range(L)]
+
+        def lstep():
+            for ly in llayers:
+                ly.mask()
+                ly.attend()
+
+        for _ in range(3):
+            lstep()
+        tl = events_ms(lstep, 5)
+        F_l = sum(kept_flops(w.B, w.heads, Tb, k, w.head_dim) for k in lkeep)
+        layer_aware = {"ms_per_step": tl, "effective_tflops": F_l / (tl * 1e-3) / 1e12,
+                       "mean_sparsity": 1.0 - sum(lkeep) / (L * Tb), "keep_per_layer": lkeep,
+                       "uniform_ms_per_step": ms_step,
+                       "how": "mask + forward of the 24 layers with rho_l from schedule.layer_rhos, CUDA events "
+                              "around 5 steps"}
+    except Exception as exc:  # reported, not fatal
+        layer_aware = f"failed: {exc}"
+
+    # ---- the steps before the mask fused into the projection (ssba_qkv_rope_pool): X W^T + b, RoPE,
+    #      block means; 1024 px, Dm = 1536; X and Wqkv (27 MB) stay in L2 between launches
+    qkv = None
+    try:
+        Dm = w.heads * w.head_dim
+        X, Wq, bq = (t.to(dev) for t in synthetic.projection_inputs(w.B, w.N, Dm, seed=800 + rank))
+        pshp = (w.B, w.heads, Tb, w.head_dim)
+        outs = [torch.empty(shp, dtype=torch.bfloat16, device=dev) for _ in range(3)] + \
+               [torch.empty(pshp, dtype=torch.float32, device=dev) for _ in range(2)]
+        flops_qkv = 2.0 * w.B * w.N * Dm * 3 * Dm
+        qkv = {"flops": flops_qkv, "peak_tflops": bf16_tflops, "peak_source": peak_src}
+        for name, sh in (("unshifted", (0, 0)), ("shifted", (4, 4))):
+            dq = api.SsbaDesc(w.B, w.heads, w.H_tok, w.W_tok, w.head_dim, 8, *sh, w.rho, w.dtype)
+            fn = (lambda dq=dq: api.qkv_rope_pool(dq, X, Wq, bq, out=outs, stream=stream))
+            for _ in range(3):
+                fn()
+            tq = events_ms(fn, 20)
+            qkv[name] = {"us": tq * 1e3, "tflops": flops_qkv / (tq * 1e-3) / 1e12,
+                         "frac": flops_qkv / (tq * 1e-3) / 1e12 / bf16_tflops}
+        lin = (lambda: torch.nn.functional.linear(X, Wq))
+        for _ in range(3):
+            lin()
+        tc = events_ms(lin, 20)
+        qkv["cublas_plain_projection"] = {"us": tc * 1e3, "tflops": flops_qkv / (tc * 1e-3) / 1e12}
+        qkv["how"] = ("ssba_qkv_rope_pool (tcgen05, bias + 2-D RoPE + block means fused) against "
+                      "torch.nn.functional.linear (cuBLAS, the bare X W^T); CUDA events around 20 launches")
+    except Exception as exc:  # reported, not fatal
+        qkv = f"failed: {exc}"
+
     # ---- end to end through the public API with host buffers (pinned), copies timed
     e2e = None
     if args.e2e_steps > 0:
@@ -518,6 +586,33 @@ def run_ours(args, rank, world):
                "sample": f"{heads_sample} of {w.heads} heads of one layer (mask + forward), {dt:.2f} s, "
                          f"fp64 C with OpenMP over heads"}
 
+    # ---- the mask when the projection has pooled: selection alone (ssba_select_mask) against the
+    #      full build (ssba_build_mask re-reads Q and K); 20 launches captured in a CUDA graph,
+    #      since one launch is shorter than its host call
+    mask_split = None
+    if isinstance(qkv, dict):
+        try:
+            d1 = descs[1]
+            qb_, kb_ = outs[3], outs[4]
+            sidx = torch.empty((w.B, w.heads, Tb, keep), dtype=torch.int32, device=dev)
+            scnt = torch.empty((w.B, w.heads, Tb), dtype=torch.int32, device=dev)
+            res = {}
+            for name, fn in (("select_from_pooled", lambda: api.select_mask(d1, qb_, kb_, sidx, scnt)),
+                             ("full_mask_build",
+                              lambda: api.build_mask(d1, Qs[1], Ks[1], sidx, scnt, workspace=ws))):
+                fn()
+                torch.cuda.synchronize()
+                graph = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(graph):
+                    for _ in range(20):
+                        fn()
+                graph.replay()
+                torch.cuda.synchronize()
+                res[name + "_us"] = events_ms(graph.replay, 5) / 20 * 1e3
+            mask_split = dict(res, how="per launch, 20 launches per CUDA graph, 5 replays, 1024 px layer")
+        except Exception as exc:  # reported, not fatal
+            mask_split = f"failed: {exc}"
+
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": K,
@@ -531,6 +626,9 @@ def run_ours(args, rank, world):
             "text_joint": joint,
             "backward": bwd,
             "haar": haar,
+            "layer_aware": layer_aware,
+            "qkv_fused": qkv,
+            "mask_after_fused_pooling": mask_split,
             "speedup_vs_dense": (dense_ms / attn_ms) if isinstance(dense_ms, float) else None,
             "ideal_speedup_vs_dense": Tb / keep,
             "e2e": e2e, "cpu_baseline": cpu,
