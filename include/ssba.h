@@ -185,6 +185,28 @@ SSBA_API int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, 
 /* Bytes of the ssba_backward workspace: B * heads * N * 4 (0 for an invalid descriptor). */
 SSBA_API size_t ssba_backward_workspace_bytes(const ssba_desc* desc);
 
+/* Block compression alone (Sec. 2.2, the means q_b, k_b; Algorithm 1 MeanPool): the first
+ * half of ssba_build_mask, for ssba_forward_select.
+ *   Q, K    device, [B][heads][N][head_dim] of desc->dtype (post-RoPE), 16-byte aligned.
+ *   qb, kb  device out, fp32 [B][heads][Tb][head_dim], 16-byte aligned.
+ * Any shift; head_dim * element size a multiple of 16 bytes, head_dim <= 256. */
+SSBA_API int ssba_pool_blocks(const ssba_desc* desc, const void* Q, const void* K, float* qb, float* kb,
+                              void* stream);
+
+/* Affinity, Top-k gating and sparse attention in one launch (Sec. 2.2, Algorithm 1 from
+ * "S <- q_b k_b^T" on): each CTA computes the score rows and the kept-block lists of the query
+ * blocks it will process (the arithmetic of ssba_build_mask, so the same means give the same
+ * lists), writes them to kv_idx / kv_cnt (outputs here, same layout as ssba_build_mask), and
+ * runs the forward of ssba_forward on them.
+ *   qb, kb      device, fp32 block means from ssba_pool_blocks (or ssba_qkv_rope_pool).
+ *   scores_opt  device out or NULL, fp32 [B][heads][Tb][Tb]: the scores of the selection.
+ *   Q, K, V, O, lse, workspace as for ssba_forward.
+ * bf16 only; Tb <= 128 (else SSBA_ERR_UNSUPPORTED: use ssba_build_mask + ssba_forward). */
+SSBA_API int ssba_forward_select(const ssba_desc* desc, const void* Q, const void* K, const void* V,
+                                 const float* qb, const float* kb, int32_t* kv_idx, int32_t* kv_cnt,
+                                 float* scores_opt, void* O, float* lse, void* workspace, size_t ws_bytes,
+                                 void* stream);
+
 /* One level of the T-DVAE's 2-D Haar kernel bank F = {LL, HL, LH, HH} (Sec. 2.3
  * DWT-Enhanced Architecture), per channel, stride 2, orthonormal: for the window
  * a = x[2i][2j], b = x[2i][2j+1], c = x[2i+1][2j], d = x[2i+1][2j+1],

@@ -30,7 +30,7 @@ EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
             "ssba_test_forward_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
             "ssba_haar_iwt", "ssba_haar_dwt_pyramid", "ssba_haar_iwt_pyramid", "ssba_qkv_rope_pool",
-            "ssba_select_mask",
+            "ssba_select_mask", "ssba_pool_blocks", "ssba_forward_select",
             "ssba_get_status", "ssba_last_error")
 
 
@@ -108,6 +108,10 @@ def load_library():
         lib.ssba_qkv_rope_pool.restype = ctypes.c_int
         lib.ssba_select_mask.argtypes = [DP, P, P, P, P, P, P]
         lib.ssba_select_mask.restype = ctypes.c_int
+        lib.ssba_pool_blocks.argtypes = [DP, P, P, P, P, P]
+        lib.ssba_pool_blocks.restype = ctypes.c_int
+        lib.ssba_forward_select.argtypes = [DP, P, P, P, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
+        lib.ssba_forward_select.restype = ctypes.c_int
         lib.ssba_forward.argtypes = [DP, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_forward.restype = ctypes.c_int
         lib.ssba_forward_joint.argtypes = [DP, P, P, P, P, P, ctypes.c_int32, P, P, P, P, P, ctypes.c_size_t, P]
@@ -301,6 +305,61 @@ def select_mask(desc: SsbaDesc, qb: torch.Tensor, kb: torch.Tensor, kv_idx=None,
     _raise_on(lib.ssba_select_mask(ctypes.byref(d), qb.data_ptr(), kb.data_ptr(), kv_idx.data_ptr(),
                                    kv_cnt.data_ptr(), S.data_ptr() if S is not None else None, _stream_ptr(stream)))
     return (kv_idx, kv_cnt, S) if S is not None else (kv_idx, kv_cnt)
+
+
+def pool_blocks(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, qb=None, kb=None, stream=None):
+    """ssba_pool_blocks: (qb, kb) fp32 [B, heads, Tb, head_dim] block means of Q and K."""
+    lib = load_library()
+    d = desc.c()
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    _check(Q, "Q", shp, desc.dtype)
+    _check(K, "K", shp, desc.dtype)
+    pshp = (desc.B, desc.heads, desc.Tb, desc.head_dim)
+    qb = torch.empty(pshp, dtype=torch.float32, device=Q.device) if qb is None else qb
+    kb = torch.empty(pshp, dtype=torch.float32, device=Q.device) if kb is None else kb
+    _check(qb, "qb", pshp, torch.float32)
+    _check(kb, "kb", pshp, torch.float32)
+    _raise_on(lib.ssba_pool_blocks(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), qb.data_ptr(), kb.data_ptr(),
+                                   _stream_ptr(stream)))
+    return qb, kb
+
+
+def forward_select(desc: SsbaDesc, Q, K, V, qb, kb, kv_idx=None, kv_cnt=None, scores: bool | torch.Tensor = False,
+                   O=None, lse=None, workspace="default", stream=None):
+    """ssba_forward_select: selection inside the attention launch. Returns (O, lse, kv_idx, kv_cnt[, S])."""
+    lib = load_library()
+    d = desc.c()
+    keep = keep_count(desc)
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
+        _check(t, n, shp, desc.dtype)
+    pshp = (desc.B, desc.heads, desc.Tb, desc.head_dim)
+    _check(qb, "qb", pshp, torch.float32)
+    _check(kb, "kb", pshp, torch.float32)
+    dev = Q.device
+    kv_idx = torch.empty((desc.B, desc.heads, desc.Tb, keep), dtype=torch.int32, device=dev) if kv_idx is None \
+        else kv_idx
+    kv_cnt = torch.empty((desc.B, desc.heads, desc.Tb), dtype=torch.int32, device=dev) if kv_cnt is None else kv_cnt
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    S = None
+    if isinstance(scores, torch.Tensor):
+        S = scores
+        _check(S, "scores", (desc.B, desc.heads, desc.Tb, desc.Tb), torch.float32)
+    elif scores:
+        S = torch.empty((desc.B, desc.heads, desc.Tb, desc.Tb), dtype=torch.float32, device=dev)
+    O = torch.empty(shp, dtype=desc.dtype, device=dev) if O is None else O
+    lse = torch.empty(shp[:3], dtype=torch.float32, device=dev) if lse is None else lse
+    _check(O, "O", shp, desc.dtype)
+    _check(lse, "lse", shp[:3], torch.float32)
+    if isinstance(workspace, str):
+        workspace = default_forward_workspace(desc, dev)
+    wp, wn = _ws_args(workspace)
+    _raise_on(lib.ssba_forward_select(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), qb.data_ptr(),
+                                      kb.data_ptr(), kv_idx.data_ptr(), kv_cnt.data_ptr(),
+                                      S.data_ptr() if S is not None else None, O.data_ptr(), lse.data_ptr(), wp, wn,
+                                      _stream_ptr(stream)))
+    return (O, lse, kv_idx, kv_cnt, S) if S is not None else (O, lse, kv_idx, kv_cnt)
 
 
 def build_mask_noalloc(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=None, kv_cnt=None,
@@ -571,6 +630,47 @@ def get_status() -> int:
 def realized_sparsity(desc: SsbaDesc) -> float:
     """k_drop / Tb with k_drop = floor(Tb * rho) (host arithmetic, no device call)."""
     return math.floor(desc.Tb * desc.rho) / desc.Tb
+
+
+class BoundSelectLayer:
+    """One SSBA layer on the one-launch selection path: ``pool()`` (ssba_pool_blocks) and
+    ``attend()`` (ssba_forward_select, which also writes the kept-block lists), buffers
+    validated once and bare C calls after that."""
+
+    def __init__(self, desc: SsbaDesc, Q, K, V, qb, kb, kv_idx, kv_cnt, O, lse, stream=None,
+                 fwd_workspace="default"):
+        lib = load_library()
+        self._lib = lib
+        self._d = desc.c()
+        keep = keep_count(desc)
+        shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+        pshp = (desc.B, desc.heads, desc.Tb, desc.head_dim)
+        for t, n in ((Q, "Q"), (K, "K"), (V, "V"), (O, "O")):
+            _check(t, n, shp, desc.dtype)
+        _check(qb, "qb", pshp, torch.float32)
+        _check(kb, "kb", pshp, torch.float32)
+        _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+        _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+        _check(lse, "lse", shp[:3], torch.float32)
+        if isinstance(fwd_workspace, str):
+            fwd_workspace = default_forward_workspace(desc, Q.device)
+        fwp, fwn = _ws_args(fwd_workspace)
+        self.tensors = (Q, K, V, qb, kb, kv_idx, kv_cnt, O, lse, fwd_workspace)  # keep alive
+        st = _stream_ptr(stream)
+        self._pool_args = (ctypes.byref(self._d), Q.data_ptr(), K.data_ptr(), qb.data_ptr(), kb.data_ptr(), st)
+        self._fwd_args = (ctypes.byref(self._d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), qb.data_ptr(),
+                          kb.data_ptr(), kv_idx.data_ptr(), kv_cnt.data_ptr(), None, O.data_ptr(), lse.data_ptr(),
+                          fwp, fwn, st)
+
+    def pool(self) -> None:
+        rc = self._lib.ssba_pool_blocks(*self._pool_args)
+        if rc:
+            _raise_on(rc)
+
+    def attend(self) -> None:
+        rc = self._lib.ssba_forward_select(*self._fwd_args)
+        if rc:
+            _raise_on(rc)
 
 
 class BoundLayer:

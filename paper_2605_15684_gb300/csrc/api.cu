@@ -238,6 +238,54 @@ int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void
     return launch_attn_tc_bf16(*desc, g, keep, scale, Q, K, V, kv_idx, kv_cnt, O, lse, workspace, ws_bytes, st);
 }
 
+int ssba_pool_blocks(const ssba_desc* desc, const void* Q, const void* K, float* qb, float* kb, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_pool_blocks", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !qb || !kb) {
+        set_error("ssba_pool_blocks: Q, K, qb and kb must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    if ((desc->head_dim * elem_size(desc)) % 16 || desc->head_dim > 256) {
+        set_error("ssba_pool_blocks: head_dim*elem must be a multiple of 16 bytes and head_dim <= 256");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(qb, 16) || !aligned(kb, 16)) {
+        set_error("ssba_pool_blocks: Q, K, qb and kb must be 16-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    return launch_pool_blocks(*desc, g, Q, K, qb, kb, static_cast<cudaStream_t>(stream));
+}
+
+int ssba_forward_select(const ssba_desc* desc, const void* Q, const void* K, const void* V, const float* qb,
+                        const float* kb, int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O, float* lse,
+                        void* workspace, size_t ws_bytes, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_forward_select", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !V || !qb || !kb || !kv_idx || !kv_cnt || !O || !lse) {
+        set_error("ssba_forward_select: every pointer but scores_opt must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(qb, 16) ||
+        !aligned(kb, 16) || !aligned(lse, 4) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) ||
+        (scores_opt && !aligned(scores_opt, 4)) || (workspace && !aligned(workspace, 16))) {
+        set_error("ssba_forward_select: Q, K, V, O, qb, kb, workspace 16-byte aligned; the rest 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    if (desc->dtype != SSBA_BF16) {
+        set_error("ssba_forward_select: bf16 only (the tensor-core path)");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    return launch_attn_tc_bf16(*desc, g, keep, resolve_scale(desc), Q, K, V, kv_idx, kv_cnt, O, lse, workspace,
+                               ws_bytes, static_cast<cudaStream_t>(stream), kWaitBudgetNs, 0, nullptr, nullptr, 0, qb,
+                               kb, scores_opt);
+}
+
 int ssba_forward_joint(const ssba_desc* desc, const void* Q, const void* K, const void* V, const void* K_txt,
                        const void* V_txt, int32_t T_txt, const int32_t* kv_idx, const int32_t* kv_cnt, void* O,
                        float* lse, void* workspace, size_t ws_bytes, void* stream)

@@ -36,6 +36,10 @@
 //               thread: 768 threads on one SM). At the end of an item the row statistics
 //               (max, sum) go to shared memory.
 //   warps 8-11  epilogue: O / l in bf16 and lse, overlapping the next item's softmax.
+// In-kernel selection (ssba_forward_select): given the block means, each CTA first computes
+// the score rows and the Top-k gating of its own items (one warp per item, the arithmetic of
+// the mask kernels) and writes the lists to the caller's kv_idx / kv_cnt, which its producers
+// then read back (coherent loads); no separate selection launch and no cross-CTA dependency.
 // Tile rows follow the TMA box order of the window (tile_row_pos). All mbarrier waits are
 // bounded (globaltimer budget + CTA abort flag); a timeout is reported in the device status
 // word and the CTA drains its in-flight copies and MMAs before it exits.
@@ -45,6 +49,7 @@
 
 #include "common.cuh"
 #include "ptx.cuh"
+#include "select.cuh"
 
 namespace ssba {
 
@@ -139,6 +144,10 @@ struct TcParams {
     int* ws_cnt;       // [boundaries][4] arrival counters, zero between launches
     float2* ws_st;     // [boundaries][2][64] row (max in log2 units, sum) of each part
     float* ws_o;       // [boundaries][2][64][64] unnormalised O of each part, fp32
+    const float* sel_qb;  // in-kernel selection: block means [B*heads][Tb][64] (null: lists given)
+    const float* sel_kb;
+    int32_t* sel_cnt;     // counts written by the selection
+    float* sel_scores;    // optional S export [B*heads][Tb][Tb]
     uint64_t budget_ns;  // wall-time limit of every barrier wait
     int withhold;        // test hook: pipeline 0 announces its first K copy but never issues it,
                          // so that the waits on it run out (failure-detection test only)
@@ -162,6 +171,18 @@ struct TcParams {
 // A pipeline runs phase A first and, in it, its cut last item first, so that both parts
 // of every cut item finish early and the merges (a few global-memory round trips)
 // overlap later work instead of lengthening the end of the kernel.
+// Under in-kernel selection the items go to the pipelines in contiguous ranges (item counts
+// differing by at most one), so that the few items of a CTA share one or two heads and the
+// selection stages each head's k_b once.
+__device__ __forceinline__ int sel_item_count(const TcParams& p, int v, int V)
+{
+    return p.num_items / V + (v < p.num_items % V ? 1 : 0);
+}
+__device__ __forceinline__ int sel_first_item(const TcParams& p, int v, int V)
+{
+    return v * (p.num_items / V) + min(v, p.num_items % V);
+}
+
 __device__ __forceinline__ int split_items(const TcParams& p, int V)
 {
     return p.split ? p.num_items - (p.num_items / V - 1) * V : 0;
@@ -209,6 +230,48 @@ __device__ __forceinline__ void tmem_st_16x32bx2_x16_off32(uint32_t taddr, const
 
 __device__ __forceinline__ int clamp_label(int j, int Tb) { return j < 0 ? 0 : (j >= Tb ? Tb - 1 : j); }
 
+// A list entry: written earlier in this launch under in-kernel selection (read through L2),
+// else read-only input.
+__device__ __forceinline__ int ld_list(const TcParams& p, const int32_t* a) { return p.sel_qb ? __ldcg(a) : __ldg(a); }
+
+// Score row and Top-k gating of one item (one warp), with the arithmetic and the selection code
+// of the mask kernels (S_j = q_b . k_b[j], four interleaved partial sums over d combined in a
+// fixed order; sel::rank_select), so the same means give the same lists. kbs: the head's k_b
+// staged in shared memory, the 16-byte chunk c4 of row j at chunk c4 ^ (j & 15) (two lanes per
+// bank at most when 32 lanes read one column); qs: the item's q_b row in shared memory; S: Tb
+// words of shared scratch. Not inlined, so that its registers do not weigh on the pipeline roles.
+template <int kPer>
+__device__ __noinline__ void select_item(const TcParams& p, int item, int lane, const float* kbs, const float* qs,
+                                         uint32_t* S)
+{
+    const int Tb = p.g.Tb();
+    const float4* q4 = reinterpret_cast<const float4*>(qs);
+#pragma unroll
+    for (int m = 0; m < kPer; ++m) {
+        const int j = lane + 32 * m;
+        if (j < Tb) {
+            const float* row = kbs + j * kD;
+            const int sw = j & 15;
+            float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int c4 = 0; c4 < kD / 4; ++c4) {
+                const float4 qv = q4[c4];
+                const float4 kv = *reinterpret_cast<const float4*>(row + 4 * (c4 ^ sw));
+                a[0] = fmaf(qv.x, kv.x, a[0]);
+                a[1] = fmaf(qv.y, kv.y, a[1]);
+                a[2] = fmaf(qv.z, kv.z, a[2]);
+                a[3] = fmaf(qv.w, kv.w, a[3]);
+            }
+            const float acc = (a[0] + a[1]) + (a[2] + a[3]);
+            if (p.sel_scores) p.sel_scores[(size_t)item * Tb + j] = acc;
+            S[j] = sel::order_key(acc);
+        }
+    }
+    __syncwarp();
+    sel::rank_select<kPer>(S, Tb, p.keep, lane, const_cast<int32_t*>(p.idx) + (size_t)item * p.keep);
+    if (lane == 0) p.sel_cnt[item] = p.keep;
+    __syncwarp();
+}
 
 // Origin (row, col) of the shifted 8x8 window `label` in the unshifted grid. With block
 // 8 and a shift that is a multiple of 4, a window either fits (origin <= size - 8) or is
@@ -290,11 +353,12 @@ __device__ __forceinline__ Piece get_piece(const TcParams& p, const SlotSmem& sm
         pc.part = e.w;
     } else {
         const int r = k - sm.nA;
-        pc.item = sm.M + v + r * V;
+        pc.item = p.sel_qb ? sel_first_item(p, v, V) + r : sm.M + v + r * V;
         pc.tb = 0;
         pc.part = -1;
         pc.nb = p.units;
-        if (p.idx) pc.nb = p.ntxt + min(max(r < kCntCap ? sm.cnts[r] : __ldg(p.cnt + pc.item), 0), p.keep);
+        if (p.idx && !p.sel_qb)
+            pc.nb = p.ntxt + min(max(r < kCntCap ? sm.cnts[r] : __ldg(p.cnt + pc.item), 0), p.keep);
     }
     return pc;
 }
@@ -305,8 +369,8 @@ __device__ void build_schedule(const TcParams& p, SlotSmem& sm, int v, int V, in
 {
     const int M = split_items(p, V);
     const int rest = p.num_items - M - v;
-    const int nB = rest > 0 ? (rest + V - 1) / V : 0;
-    if (p.idx)
+    const int nB = p.sel_qb ? sel_item_count(p, v, V) : (rest > 0 ? (rest + V - 1) / V : 0);
+    if (p.idx && !p.sel_qb)
         for (int r = t; r < nB && r < kCntCap; r += nthr) sm.cnts[r] = __ldg(p.cnt + M + v + r * V);
     if (t != 0) return;
     int nA = 0;
@@ -391,6 +455,77 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     // launched just before this one (programmatic dependent launch)
     grid_dep_wait();
     grid_dep_launch();
+    if (p.sel_qb) {
+        // the lists of this CTA's items (the contiguous ranges of its two pipelines): the k_b
+        // of the heads they touch are staged by all threads in the stage buffers of both
+        // pipelines (free until the producers start), one asynchronous round per batch of
+        // heads; then one warp per item
+        const int f0 = sel_first_item(p, blockIdx.x, vgrid), n0 = sel_item_count(p, blockIdx.x, vgrid);
+        const int f1 = sel_first_item(p, blockIdx.x + gridDim.x, vgrid);
+        const int n1 = sel_item_count(p, blockIdx.x + gridDim.x, vgrid);
+        // heads of the two ranges: [h0a, h0b] and [h1a, h1b], staged in that order
+        const int h0a = f0 / Tb, h0b = n0 ? (f0 + n0 - 1) / Tb : h0a - 1;
+        const int h1a = f1 / Tb, h1b = n1 ? (f1 + n1 - 1) / Tb : h1a - 1;
+        const int nh0 = max(0, h0b - h0a + 1), nh = nh0 + max(0, h1b - h1a + 1);
+        auto head_of = [&](int hi) { return hi < nh0 ? h0a + hi : h1a + (hi - nh0); };
+        // staging: pipeline 0's k, v, q buffers end with the scratch (per warp 128 key words and
+        // a 64-float query row, then up to kSelQRows shared query rows); the rest of them and
+        // pipeline 1's hold the heads
+        constexpr uint32_t kRegion = (kKStages + kVStages + 2) * kTileBytes;  // k, v, q of one pipeline
+        constexpr int kSelQRows = 48;
+        constexpr int kWarpScratch = 128 + kD;  // words per warp: keys, then its own query row
+        constexpr uint32_t kScratch = (kThreads / 32) * kWarpScratch * 4 + kSelQRows * kD * 4;
+        const uint32_t hb = (uint32_t)Tb * kD * 4;
+        const int cap0 = (int)((kRegion - kScratch) / hb), cap = cap0 + (int)(kRegion / hb);
+        uint8_t* r0 = &cs.slot[0].k[0][0];
+        uint32_t* keys = reinterpret_cast<uint32_t*>(r0 + kRegion - kScratch) + gwarp * kWarpScratch;
+        float* qrows = reinterpret_cast<float*>(r0 + kRegion - kScratch + (kThreads / 32) * kWarpScratch * 4);
+        auto staged = [&](int hi) {
+            return reinterpret_cast<float*>(hi < cap0 ? r0 + hi * hb : &cs.slot[1].k[0][0] + (hi - cap0) * hb);
+        };
+        auto item_of = [&](int q) { return q < n0 ? f0 + q : f1 + (q - n0); };
+        for (int base = 0; base < nh; base += cap) {
+            const int m = min(cap, nh - base);
+            // asynchronous 16-byte copies, all in flight at once: the heads' k_b (chunk c4 of row
+            // j to chunk c4 ^ (j & 15)) and, in the first round, the items' q_b rows
+            for (int e = threadIdx.x; e < m * Tb * (kD / 4); e += kThreads) {
+                const int hi = e / (Tb * (kD / 4)), rem = e - hi * Tb * (kD / 4);
+                const int j = rem / (kD / 4), c4 = rem - j * (kD / 4);
+                const float* src = p.sel_kb + ((size_t)head_of(base + hi) * Tb + j) * kD + 4 * c4;
+                const uint32_t dst = smem_u32(staged(hi) + j * kD + 4 * (c4 ^ (j & 15)));
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+            }
+            if (base == 0)
+                for (int e = threadIdx.x; e < min(n0 + n1, kSelQRows) * (kD / 4); e += kThreads) {
+                    const int q = e / (kD / 4), c4 = e - q * (kD / 4);
+                    const float* src = p.sel_qb + (size_t)item_of(q) * kD + 4 * c4;
+                    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(qrows + q * kD + 4 * c4)),
+                                 "l"(src) : "memory");
+                }
+            asm volatile("cp.async.wait_all;" ::: "memory");
+            __syncthreads();
+            // the items whose head is in this batch
+            for (int q = gwarp; q < n0 + n1; q += kThreads / 32) {
+                const int item = item_of(q);
+                const int h = item / Tb;
+                const int hi = (q < n0 ? h - h0a : nh0 + h - h1a) - base;
+                if (hi < 0 || hi >= m) continue;
+                const float* qs = qrows + q * kD;
+                if (q >= kSelQRows) {  // rows past the staged ones: this warp's own copy
+                    float* own = reinterpret_cast<float*>(keys) + 128;  // after its keys
+                    if (lane < kD / 4)
+                        reinterpret_cast<float4*>(own)[lane] =
+                            __ldg(reinterpret_cast<const float4*>(p.sel_qb + (size_t)item * kD) + lane);
+                    __syncwarp();
+                    qs = own;
+                }
+                if (Tb <= 32) select_item<1>(p, item, lane, staged(hi), qs, keys);
+                else if (Tb <= 64) select_item<2>(p, item, lane, staged(hi), qs, keys);
+                else select_item<4>(p, item, lane, staged(hi), qs, keys);
+            }
+            __syncthreads();
+        }
+    }
     build_schedule(p, sm, vcta, vgrid, threadIdx.x % (kSlotWarps * 32), kSlotWarps * 32);
     if (gwarp == 0 && lane < 12) tma_prefetch_desc(lane < 4 ? &maps.q[lane] : (lane < 8 ? &maps.k[lane - 4] : &maps.v[lane - 8]));
     if (gwarp == 1) {
@@ -427,7 +562,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             // piece ahead with cp.async)
             uint32_t* lab = reinterpret_cast<uint32_t*>(sm.labels[is_k ? 0 : 1]);
             for (int t = lane; t < nimg && t < kLabelCap; t += 32) {
-                const int j = list ? clamp_label(__ldg(list + t), Tb) : ti0 - p.ntxt + t;
+                const int j = list ? clamp_label(ld_list(p, list + t), Tb) : ti0 - p.ntxt + t;
                 lab[t] = j < kWinCap ? cs.win[j] : window_entry(p.g, j);
             }
             __syncwarp();
@@ -468,7 +603,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     if (t < kLabelCap) {
                         e = lab[t];
                     } else {
-                        const int j = list ? clamp_label(__ldg(list + t), Tb) : ti0 - p.ntxt + t;
+                        const int j = list ? clamp_label(ld_list(p, list + t), Tb) : ti0 - p.ntxt + t;
                         e = j < kWinCap ? cs.win[j] : window_entry(p.g, j);
                     }
                     const uint32_t slot = g % nst;
@@ -920,8 +1055,12 @@ size_t attn_tc_workspace_bytes() { return ws_cnt_bytes() + ws_st_bytes() + ws_o_
 int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
                         const void* V, const int32_t* idx, const int32_t* cnt, void* O, float* lse, void* ws,
                         size_t ws_bytes, cudaStream_t st, uint64_t budget_ns, int withhold, const void* Kt,
-                        const void* Vt, int t_txt)
+                        const void* Vt, int t_txt, const float* sel_qb, const float* sel_kb, float* sel_scores)
 {
+    if (sel_qb && (g.Tb() > 128 || t_txt > 0 || !idx || !cnt)) {
+        set_error("ssba_forward_select: needs Tb <= 128, no text segment and list outputs");
+        return SSBA_ERR_UNSUPPORTED;
+    }
     if (d.head_dim != kD || g.blk != 8 || (g.sr % 4) || (g.sc % 4)) {
         set_error("ssba_forward (bf16): needs head_dim=64, block=8 and shifts that are multiples of 4");
         return SSBA_ERR_UNSUPPORTED;
@@ -960,6 +1099,10 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
     p.scale_log2 = scale * 1.4426950408889634f;
     p.budget_ns = budget_ns;
     p.withhold = withhold;
+    p.sel_qb = sel_qb;
+    p.sel_kb = sel_kb;
+    p.sel_cnt = const_cast<int32_t*>(cnt);
+    p.sel_scores = sel_scores;
     p.status = device_status_word();
     if (!p.status) {
         set_error("ssba_forward (bf16): could not resolve the device status word");
@@ -990,7 +1133,8 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
         // more than another, and when items are long: a merge costs a few global-memory
         // round trips (about 5 us under load, measured), which 11-block items do not
         // earn back but 64-block items (dense) do (179 vs 198 us at 1024 px, 24 heads).
-        p.split = (p.units >= kSplitMinKeep && p.num_items >= kSlots * grid && p.num_items % (kSlots * grid) != 0)
+        p.split = (!sel_qb && p.units >= kSplitMinKeep && p.num_items >= kSlots * grid &&
+                   p.num_items % (kSlots * grid) != 0)
                       ? 1 : 0;
     }
     // programmatic dependent launch: the kernel may start (barriers, tensor memory, window

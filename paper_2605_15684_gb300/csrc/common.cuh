@@ -38,6 +38,10 @@ struct Grid {
 // Host-side launchers (defined in the .cu files, called by api.cu).
 int launch_pool(const ssba_desc& d, const Grid& g, const void* Q, const void* K, float* qb, float* kb,
                 cudaStream_t st);
+// Block means with the pooling arithmetic of the fused mask kernel (head_dim 64, 8x8 blocks;
+// other shapes fall back to launch_pool), programmatic dependent launch.
+int launch_pool_blocks(const ssba_desc& d, const Grid& g, const void* Q, const void* K, float* qb, float* kb,
+                       cudaStream_t st);
 int launch_select(const ssba_desc& d, const Grid& g, int keep, const float* qb, const float* kb,
                   int32_t* idx, int32_t* cnt, float* scores, cudaStream_t st);
 // Pool + affinity + selection in one launch (head_dim 64, 8x8 blocks, Tb <= 256); returns
@@ -54,7 +58,8 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
                         const void* K, const void* V, const int32_t* idx, const int32_t* cnt, void* O,
                         float* lse, void* ws, size_t ws_bytes, cudaStream_t st,
                         uint64_t budget_ns = kWaitBudgetNs, int withhold = 0, const void* Kt = nullptr,
-                        const void* Vt = nullptr, int t_txt = 0);
+                        const void* Vt = nullptr, int t_txt = 0, const float* sel_qb = nullptr,
+                        const float* sel_kb = nullptr, float* sel_scores = nullptr);
 int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V,
                          void* O, float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
 // Bytes of the split-merge workspace of the bf16 forward on the current device.

@@ -21,6 +21,7 @@
 
 #include "common.cuh"
 #include "ptx.cuh"
+#include "select.cuh"
 
 namespace ssba {
 
@@ -154,42 +155,6 @@ constexpr int kSelKeyChunk = 256;
 constexpr int kMaxTb = 2048;
 constexpr int kRankMaxTb = 256;  // rows up to this length use rank counting, longer ones radix select
 
-__device__ __forceinline__ uint32_t order_key(float s)
-{
-    float f = s + 0.0f;  // -0.0 -> +0.0 so that equal values compare equal
-    uint32_t u = __float_as_uint(f);
-    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
-
-// Kept labels of one row by rank counting; lane l owns labels l + 32m, m < kPer.
-template <int kPer>
-__device__ __forceinline__ void rank_select(const uint32_t* S, int Tb, int keep, int lane, int32_t* dst)
-{
-    uint32_t mine[kPer];
-    int rank[kPer];
-#pragma unroll
-    for (int m = 0; m < kPer; ++m) {
-        const int j = lane + 32 * m;
-        mine[m] = j < Tb ? S[j] : 0u;
-        rank[m] = 0;
-    }
-#pragma unroll 8
-    for (int k = 0; k < Tb; ++k) {
-        const uint32_t v = S[k];  // broadcast read
-#pragma unroll
-        for (int m = 0; m < kPer; ++m) rank[m] += (v > mine[m]) || (v == mine[m] && k < lane + 32 * m);
-    }
-    int out = 0;
-#pragma unroll
-    for (int m = 0; m < kPer; ++m) {
-        const int j = lane + 32 * m;
-        const bool kept = j < Tb && rank[m] < keep;
-        const uint32_t km = __ballot_sync(0xffffffffu, kept);
-        if (kept) dst[out + __popc(km & ((1u << lane) - 1u))] = j;
-        out += __popc(km);
-    }
-}
-
 // One warp per query block (row i of S), kSelWarps rows per CTA.
 // smem: kbT [d][kSelKeyChunk + 1] (padded transpose of a key chunk) | q rows [kSelWarps][d]
 //       | S rows as order keys [kSelWarps][Tb]
@@ -247,7 +212,7 @@ __global__ void __launch_bounds__(kSelWarps * 32) ssba_select_kernel(const float
                 for (; c < d; ++c) a[0] = fmaf(qs[warp * d + c], kbT[c * kLd + j], a[0]);
                 const float acc = (a[0] + a[1]) + (a[2] + a[3]);
                 if (scores) scores[rowoff * Tb + j0 + j] = acc;
-                S[j0 + j] = order_key(acc);
+                S[j0 + j] = sel::order_key(acc);
             }
         }
     }
@@ -255,10 +220,10 @@ __global__ void __launch_bounds__(kSelWarps * 32) ssba_select_kernel(const float
     if (!active) return;
     int32_t* dst = idx + rowoff * keep;
 
-    if (Tb <= 32) rank_select<1>(S, Tb, keep, lane, dst);
-    else if (Tb <= 64) rank_select<2>(S, Tb, keep, lane, dst);
-    else if (Tb <= 128) rank_select<4>(S, Tb, keep, lane, dst);
-    else if (Tb <= kRankMaxTb) rank_select<8>(S, Tb, keep, lane, dst);
+    if (Tb <= 32) sel::rank_select<1>(S, Tb, keep, lane, dst);
+    else if (Tb <= 64) sel::rank_select<2>(S, Tb, keep, lane, dst);
+    else if (Tb <= 128) sel::rank_select<4>(S, Tb, keep, lane, dst);
+    else if (Tb <= kRankMaxTb) sel::rank_select<8>(S, Tb, keep, lane, dst);
     else {
         // keep-th largest key by MSB-first radix select
         uint32_t prefix = 0, pmask = 0;
@@ -426,20 +391,108 @@ __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const 
                 for (int u = 0; u < 4; ++u) a[u] = fmaf(q[c + u], kbT[(c + u) * ld + j], a[u]);
             const float acc = (a[0] + a[1]) + (a[2] + a[3]);
             if (scores) scores[rowoff * Tb + j] = acc;
-            S[j] = order_key(acc);
+            S[j] = sel::order_key(acc);
         }
         __syncwarp();
         int32_t* dst = idx + rowoff * keep;
-        if (Tb <= 32) rank_select<1>(S, Tb, keep, lane, dst);
-        else if (Tb <= 64) rank_select<2>(S, Tb, keep, lane, dst);
-        else if (Tb <= 128) rank_select<4>(S, Tb, keep, lane, dst);
-        else rank_select<8>(S, Tb, keep, lane, dst);
+        if (Tb <= 32) sel::rank_select<1>(S, Tb, keep, lane, dst);
+        else if (Tb <= 64) sel::rank_select<2>(S, Tb, keep, lane, dst);
+        else if (Tb <= 128) sel::rank_select<4>(S, Tb, keep, lane, dst);
+        else sel::rank_select<8>(S, Tb, keep, lane, dst);
         if (lane == 0) cnt[rowoff] = keep;
         __syncwarp();
     }
 }
 
+// Block means alone, with the pooling loop of ssba_mask_fused_kernel (so the same inputs give
+// bit-identical means): CTA = kPoolWin blocks of one (batch*head), warp w pools tensor (w & 1)
+// of block w / 2, every load of a lane in flight at once; programmatic dependent launch.
+constexpr int kPoolWin = 4;
+template <typename T>
+__global__ void __launch_bounds__(2 * kPoolWin * 32) ssba_pool_blocks_kernel(const T* __restrict__ Q,
+                                                                             const T* __restrict__ K, Grid g,
+                                                                             float* __restrict__ qb,
+                                                                             float* __restrict__ kb)
+{
+    constexpr int kD = 64;
+    constexpr int VE = Vec<T>::kElems;
+    constexpr int CPR = kD / VE;
+    constexpr int RPI = 32 / CPR;
+    constexpr int LOADS = 64 / RPI;
+    constexpr int BATCH = LOADS < 16 ? LOADS : 16;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int Tb = g.Tb();
+    const int label = blockIdx.x * kPoolWin + (warp >> 1), which = warp & 1, bh = blockIdx.y;
+    const int N = g.H * g.W;
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
+    if (label >= Tb) return;
+    const int col = lane % CPR, r0 = lane / CPR;
+    const T* X = (which ? K : Q) + (size_t)bh * N * kD + col * VE;
+    const int br = label / g.bw, bc = label - br * g.bw;
+    const int rb = br * 8 - g.sr, cb = bc * 8 - g.sc;
+    float acc[VE];
+#pragma unroll
+    for (int e = 0; e < VE; ++e) acc[e] = 0.f;
+#pragma unroll
+    for (int i0 = 0; i0 < LOADS; i0 += BATCH) {
+        uint4 v[BATCH];
+#pragma unroll
+        for (int i = 0; i < BATCH; ++i) {
+            const int pos = r0 + (i0 + i) * RPI;
+            int r = rb + (pos >> 3), c = cb + (pos & 7);
+            r += r < 0 ? g.H : 0;
+            c += c < 0 ? g.W : 0;
+            v[i] = __ldg(reinterpret_cast<const uint4*>(X + (size_t)(r * g.W + c) * kD));
+        }
+#pragma unroll
+        for (int i = 0; i < BATCH; ++i) {
+            float f[VE];
+            Vec<T>::to_f32(v[i], f);
+#pragma unroll
+            for (int e = 0; e < VE; ++e) acc[e] += f[e];
+        }
+    }
+#pragma unroll
+    for (int o = CPR; o < 32; o <<= 1)
+#pragma unroll
+        for (int e = 0; e < VE; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+    if (r0 == 0) {
+        float* dst = (which ? kb : qb) + ((size_t)bh * Tb + label) * kD + col * VE;
+#pragma unroll
+        for (int e = 0; e < VE; ++e) dst[e] = acc[e] * (1.0f / 64.0f);
+    }
+}
+
 }  // namespace
+
+int launch_pool_blocks(const ssba_desc& d, const Grid& g, const void* Q, const void* K, float* qb, float* kb,
+                       cudaStream_t st)
+{
+    if (d.head_dim != 64 || g.blk != 8) return launch_pool(d, g, Q, K, qb, kb, st);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((g.Tb() + kPoolWin - 1) / kPoolWin, d.B * d.heads, 1);
+    cfg.blockDim = dim3(2 * kPoolWin * 32, 1, 1);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e;
+    if (d.dtype == SSBA_BF16)
+        e = cudaLaunchKernelEx(&cfg, ssba_pool_blocks_kernel<__nv_bfloat16>, static_cast<const __nv_bfloat16*>(Q),
+                               static_cast<const __nv_bfloat16*>(K), g, qb, kb);
+    else
+        e = cudaLaunchKernelEx(&cfg, ssba_pool_blocks_kernel<float>, static_cast<const float*>(Q),
+                               static_cast<const float*>(K), g, qb, kb);
+    if (e == cudaSuccess) e = cudaGetLastError();
+    if (e != cudaSuccess) {
+        set_error("ssba_pool_blocks_kernel launch: %s", cudaGetErrorString(e));
+        return SSBA_ERR_CUDA;
+    }
+    return SSBA_OK;
+}
 
 int launch_pool(const ssba_desc& d, const Grid& g, const void* Q, const void* K, float* qb, float* kb,
                 cudaStream_t st)

@@ -1,0 +1,75 @@
+"""GPU parity of the one-launch selection + attention path (ssba_pool_blocks, then
+ssba_forward_select) through the C-ABI, against the oracle: the block means, the kept-block
+lists (exact on the GPU's own scores, equal to ssba_select_mask's on the same means, and
+margin-gated against the oracle's mask) and O / lse (bf16 tolerance of tests/parity.py)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2605_15684_gb300 import api, build, synthetic
+from tests.parity import check_mask, check_out
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    api.load_library()
+    yield
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
+
+
+def _case(B, h, H, W, shift, rho, std=1.0, seed=0, workspace="default"):
+    q, k, v = synthetic.qkv(B, h, H * W, 64, torch.bfloat16, seed, std)
+    qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
+    desc = api.SsbaDesc(B, h, H, W, shift_r=shift[0], shift_c=shift[1], rho=rho, dtype=torch.bfloat16)
+    qb, kb = api.pool_blocks(desc, qd, kd)
+    O, lse, idx, cnt, S = api.forward_select(desc, qd, kd, vd, qb, kb, scores=True, workspace=workspace)
+    torch.cuda.synchronize()
+    return desc, (q, k, v), (qb, kb), (O, lse, idx, cnt, S)
+
+
+@pytest.mark.parametrize("B,h,H,W,shift,rho,std", [
+    (1, 4, 16, 16, (4, 4), 0.75, 1.0),
+    (1, 24, 32, 32, (0, 0), 0.8416, 0.125),    # 512 px
+    (1, 24, 64, 64, (4, 4), 0.8416, 1.0),      # 1024 px headline, shifted layer
+    (1, 24, 64, 64, (0, 0), 0.8416, 1.0),      # 1024 px, unshifted layer
+    (2, 3, 24, 40, (4, -4), 0.6, 1.0),         # non-square, odd block count (15)
+    (1, 2, 88, 88, (4, 4), 0.9, 1.0),          # Tb = 121: four labels per lane in the selection
+])
+def test_forward_select_matches_oracle(B, h, H, W, shift, rho, std):
+    desc, (q, k, v), (qb, kb), (O, lse, idx, cnt, S) = _case(B, h, H, W, shift, rho, std)
+    # block means against the oracle's (64 fp32 additions of bf16 values)
+    ref_q = oracle.pooled_blocks(q.double().numpy(), H, W, 8, shift)
+    mag = oracle.pooled_blocks(np.abs(q.double().numpy()), H, W, 8, shift)
+    assert np.all(np.abs(qb.cpu().double().numpy() - ref_q) <= 2.0 ** -17 * mag + 1e-12)
+    # the lists: exact on the GPU's scores, margin-gated against the oracle
+    keep = oracle.keep_count(H * W // 64, rho)
+    idx_o, cnt_o, S_o = oracle.build_mask(q, k, H, W, 8, shift, rho, return_scores=True)
+    near = check_mask(idx.cpu().numpy(), cnt.cpu().numpy(), S.cpu().numpy(), S_o, idx_o, keep)
+    assert near < 0.1 * B * h * (H * W // 64)
+    # the same means through ssba_select_mask give the same lists, bit for bit
+    idx2, cnt2 = api.select_mask(desc, qb, kb)
+    torch.cuda.synchronize()
+    assert torch.equal(idx2, idx) and torch.equal(cnt2, cnt)
+    # O and lse against the oracle's forward on these lists
+    Oo, lo = oracle.forward(q, k, v, idx.cpu().numpy(), H, W, 8, shift)
+    check_out(O.float().cpu().numpy(), lse.cpu().numpy(), Oo, lo, "bf16")
+
+
+def test_forward_select_without_workspace_matches_default():
+    args = (1, 4, 32, 32, (4, 4), 0.75)
+    _, _, _, (O1, l1, i1, c1, _) = _case(*args, seed=3)
+    _, _, _, (O2, l2, i2, c2, _) = _case(*args, seed=3, workspace=None)
+    assert torch.equal(i1, i2) and torch.equal(O1, O2) and torch.equal(l1, l2)
+
+
+def test_forward_select_rejects_long_rows():
+    q, k, v = (t.cuda() for t in synthetic.qkv(1, 1, 96 * 96, 64, torch.bfloat16, 0))  # Tb = 144
+    desc = api.SsbaDesc(1, 1, 96, 96, rho=0.8, dtype=torch.bfloat16)
+    qb, kb = api.pool_blocks(desc, q, k)
+    with pytest.raises(api.SsbaError, match="Tb <= 128"):
+        api.forward_select(desc, q, k, v, qb, kb)
