@@ -201,6 +201,29 @@ def test_qkv_and_select_validation(lib):
         api.SSBA_ERR_UNSUPPORTED
 
 
+def test_pool_and_select_forward_validation(lib):
+    """ssba_pool_blocks and ssba_forward_select check pointers, alignment, dtype and the row
+    length before any launch."""
+    d = desc()
+    assert lib.ssba_pool_blocks(ctypes.byref(d), FAKE, None, FAKE, FAKE, None) == api.SSBA_ERR_INVALID
+    assert lib.ssba_pool_blocks(ctypes.byref(d), FAKE, FAKE, FAKE + 4, FAKE, None) == api.SSBA_ERR_INVALID
+    assert lib.ssba_pool_blocks(ctypes.byref(desc(head_dim=12)), FAKE, FAKE, FAKE, FAKE, None) == \
+        api.SSBA_ERR_UNSUPPORTED
+    good = [FAKE] * 11  # Q K V qb kb idx cnt scores O lse workspace
+    fs = lambda dd, v, n=0: lib.ssba_forward_select(ctypes.byref(dd), *v, n, None)
+    bad = list(good)
+    bad[3] = None  # no block means
+    assert fs(d, bad) == api.SSBA_ERR_INVALID
+    bad = list(good)
+    bad[8] = FAKE + 8  # misaligned O
+    assert fs(d, bad) == api.SSBA_ERR_INVALID
+    assert fs(desc(dtype=api.SSBA_FP32), good) == api.SSBA_ERR_UNSUPPORTED
+    assert b"bf16" in lib.ssba_last_error()
+    # rows longer than 128 blocks: the two-launch path
+    assert fs(desc(H_tok=96, W_tok=96), good) == api.SSBA_ERR_UNSUPPORTED
+    assert b"Tb <= 128" in lib.ssba_last_error()
+
+
 def ct_byref(d):
     return ctypes.byref(d)
 
