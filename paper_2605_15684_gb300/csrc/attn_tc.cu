@@ -236,7 +236,8 @@ __device__ __forceinline__ int ld_list(const TcParams& p, const int32_t* a) { re
 
 // Score row and Top-k gating of one item (one warp), with the arithmetic and the selection code
 // of the mask kernels (S_j = q_b . k_b[j], four interleaved partial sums over d combined in a
-// fixed order; sel::rank_select), so the same means give the same lists. kbs: the head's k_b
+// fixed order; the total order of sel::rank_select, walked by sel::ballot_select on keys held
+// in registers), so the same means give the same lists. kbs: the head's k_b
 // staged in shared memory, the 16-byte chunk c4 of row j at chunk c4 ^ (j & 15) (two lanes per
 // bank at most when 32 lanes read one column); qs: the item's q_b row in shared memory; S: Tb
 // words of shared scratch. Not inlined, so that its registers do not weigh on the pipeline roles.
@@ -246,9 +247,11 @@ __device__ __noinline__ void select_item(const TcParams& p, int item, int lane, 
 {
     const int Tb = p.g.Tb();
     const float4* q4 = reinterpret_cast<const float4*>(qs);
+    uint32_t key[kPer];
 #pragma unroll
     for (int m = 0; m < kPer; ++m) {
         const int j = lane + 32 * m;
+        key[m] = 0u;
         if (j < Tb) {
             const float* row = kbs + j * kD;
             const int sw = j & 15;
@@ -264,11 +267,11 @@ __device__ __noinline__ void select_item(const TcParams& p, int item, int lane, 
             }
             const float acc = (a[0] + a[1]) + (a[2] + a[3]);
             if (p.sel_scores) p.sel_scores[(size_t)item * Tb + j] = acc;
-            S[j] = sel::order_key(acc);
+            key[m] = sel::order_key(acc);
         }
     }
-    __syncwarp();
-    sel::rank_select<kPer>(S, Tb, p.keep, lane, const_cast<int32_t*>(p.idx) + (size_t)item * p.keep);
+    (void)S;
+    sel::ballot_select<kPer>(key, Tb, p.keep, lane, const_cast<int32_t*>(p.idx) + (size_t)item * p.keep);
     if (lane == 0) p.sel_cnt[item] = p.keep;
     __syncwarp();
 }

@@ -45,5 +45,44 @@ __device__ __forceinline__ void rank_select(const uint32_t* S, int Tb, int keep,
     }
 }
 
+// The same selection with the keys in registers (lane l holds the keys of labels l + 32 m,
+// 0 for labels >= Tb): the keep-th largest key T by an MSB-first radix walk over ballots, then
+// kept = key > T, or key == T among the first equal ones in label order. Same total order, so
+// the same lists as rank_select; 32 rounds of kPer ballots instead of Tb shared-memory reads.
+template <int kPer>
+__device__ __forceinline__ void ballot_select(const uint32_t (&key)[kPer], int Tb, int keep, int lane, int32_t* dst)
+{
+    bool valid[kPer];
+#pragma unroll
+    for (int m = 0; m < kPer; ++m) valid[m] = lane + 32 * m < Tb;
+    uint32_t prefix = 0u, pmask = 0u;
+    int remaining = keep;
+#pragma unroll 4
+    for (int bit = 31; bit >= 0; --bit) {
+        const uint32_t trial = prefix | (1u << bit), tmask = pmask | (1u << bit);
+        int c = 0;
+#pragma unroll
+        for (int m = 0; m < kPer; ++m) c += __popc(__ballot_sync(0xffffffffu, valid[m] && (key[m] & tmask) == trial));
+        if (c >= remaining)
+            prefix = trial;
+        else
+            remaining -= c;
+        pmask = tmask;
+    }
+    const uint32_t T = prefix;
+    int out = 0, eq_seen = 0;
+#pragma unroll
+    for (int m = 0; m < kPer; ++m) {
+        const bool gt = valid[m] && key[m] > T, eq = valid[m] && key[m] == T;
+        const uint32_t eqm = __ballot_sync(0xffffffffu, eq);
+        const int eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
+        const bool kept = gt || (eq && eq_rank < remaining);
+        const uint32_t km = __ballot_sync(0xffffffffu, kept);
+        if (kept) dst[out + __popc(km & ((1u << lane) - 1u))] = lane + 32 * m;
+        out += __popc(km);
+        eq_seen += __popc(eqm);
+    }
+}
+
 }  // namespace sel
 }  // namespace ssba
