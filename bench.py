@@ -448,8 +448,8 @@ def run_ours(args, rank, world):
         tb = e0.elapsed_time(e1) / reps
         F_b = 2.5 * F_layer
         bwd = {"ms_per_layer": tb, "effective_tflops": F_b / (tb * 1e-3) / 1e12, "flops_per_layer": F_b,
-               "how": "ssba_backward (CUDA cores, fp32) per layer on the layer's forward O and lse and a "
-                      "synthetic dO, CUDA events"}
+               "how": "ssba_backward (tcgen05 kernels: dQ and D per query block, then dK, dV per key block) "
+                      "per layer on the layer's forward O and lse and a synthetic dO, CUDA events"}
     except Exception as exc:  # reported, not fatal
         bwd = f"failed: {exc}"
 

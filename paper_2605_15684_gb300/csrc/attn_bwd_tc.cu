@@ -1,0 +1,503 @@
+// attn_bwd_tc.cu -- gradients of the block-sparse attention (the backward of Algorithm 1's
+// SparseAttention over the same kept blocks) on the sm_103a tensor cores, bf16 inputs.
+//
+// For the output gradient dO, with p_nm = exp(scale q_n.k_m - lse_n) over the kept pairs:
+//   D_n = dO_n . O_n,  ds_nm = p_nm (dO_n . v_m - D_n),
+//   dQ_n = scale sum_m ds_nm k_m,  dK_m = scale sum_n ds_nm q_n,  dV_m = sum_n p_nm dO_n.
+// Two kernels, as the CUDA-core version, deterministic (no atomics), 128 threads per CTA,
+// one (batch*head, block) per CTA, each 64 x 64 tile product a tcgen05.mma kind::f16 with
+// M=64 (four K=16 steps) issued by one thread:
+//   ssba_bwd_dq_tc_kernel    query block i: for each kept key block j (list order)
+//                              S  = Q_i K_j^T,  dP = dO_i V_j^T        (A, B from shared memory)
+//                              dS = P o (dP - D) in registers, bf16 back into TMEM over S
+//                              dQ += dS K_j                           (A from TMEM, B MN-major)
+//                            and writes D for the second kernel.
+//   ssba_bwd_dkdv_tc_kernel  key block j: for each query block i whose list holds j (ascending)
+//                              S^T = K_j Q_i^T,  dP^T = V_j dO_i^T
+//                              P^T, dS^T in registers, bf16 back into TMEM over S^T and dP^T
+//                              dV += P^T dO_i,  dK += dS^T Q_i
+// Tiles are gathered token by token (the shifted window) with 16-byte cp.async into the
+// 128-byte-swizzled layout the MMA descriptors read (K-major for A/B, MN-major as the second
+// operand of the accumulating products), the next pair's tiles in flight while the current
+// one computes. TMEM: S, dP, and one or two fp32 accumulators (256 columns, two CTAs per SM).
+// The thread that owns TMEM lane (row) r of the M=64 data path holds half a row: columns
+// [32 h, 32 h + 32), h = lane / 16. Every mbarrier wait is bounded; a timeout is written to the
+// device status word and the CTA drains its MMAs before it exits.
+#include <cstdint>
+
+#include "common.cuh"
+#include "ptx.cuh"
+
+namespace ssba {
+
+namespace {
+
+using namespace ptx;
+
+constexpr int kD = 64;
+constexpr int kT = 64;                   // tokens per block
+constexpr int kThreads = 128;
+constexpr uint32_t kTile = kT * kD * 2;  // 8 KB
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kColS = 0, kColDP = 64, kColA0 = 128, kColA1 = 192;
+constexpr uint32_t kIdescK = idesc_bf16_f32(64, 64, false, false);  // A, B K-major
+constexpr uint32_t kIdescMN = idesc_bf16_f32(64, 64, false, true);  // B MN-major
+constexpr size_t kSmemBytes = 100 * 1024;  // also keeps residency at two CTAs per SM (TMEM)
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Block `label` of a [N][64] bf16 head into a 1024-aligned 8 KB tile: row r = in-window
+// position r, 16-byte chunk c at chunk c ^ (r & 7) (the 128-byte swizzle).
+__device__ __forceinline__ void load_tile(uint32_t dst, const __nv_bfloat16* X, const Grid& g, int label)
+{
+    for (int e = threadIdx.x; e < kT * 8; e += kThreads) {
+        const int r = e >> 3, c = e & 7;
+        cp_async16(dst + r * 128 + ((c ^ (r & 7)) << 4), X + (size_t)g.token(label, r) * kD + c * 8);
+    }
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
+{
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ float fast_exp2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// C (64 x 64, fp32 TMEM at column `col`) = A B^T with A, B K-major 64 x 64 tiles in shared memory.
+__device__ __forceinline__ void mma_kk(uint32_t col, uint32_t a, uint32_t b)
+{
+    const uint64_t ad = sdesc_sw128(a, 16, 1024), bd = sdesc_sw128(b, 16, 1024);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) mma_ss(col, ad + (uint64_t)(k * 2), bd + (uint64_t)(k * 2), kIdescK, k > 0 ? 1u : 0u);
+}
+
+// C (+)= A B with A (64 x 64 bf16, packed pairs) in TMEM at column `acol` and B the shared tile
+// read MN-major (rows = the contraction index).
+__device__ __forceinline__ void mma_tb(uint32_t col, uint32_t acol, uint32_t b, bool accumulate)
+{
+    const uint64_t bd = sdesc_sw128(b, 8192, 1024);
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        mma_ts(col, acol + k * 8, bd + (uint64_t)(k * 128), kIdescMN, (accumulate || k > 0) ? 1u : 0u);
+}
+
+struct alignas(1024) BwdSmem {
+    uint8_t a[kTile];        // dq: Q_i;  dkdv: K_j
+    uint8_t b[kTile];        // dq: dO_i; dkdv: V_j
+    uint8_t x[2][kTile];     // dq: K_j;  dkdv: Q_i   (double-buffered)
+    uint8_t y[2][kTile];     // dq: V_j;  dkdv: dO_i
+    float ls[2][kT];         // dkdv: lse * log2(e) of the query block
+    float ds[2][kT];         // dkdv: D of the query block
+    int list[256];           // dkdv: the query blocks holding this key block, ascending
+    int wcount[kThreads / 32];
+    uint64_t bar_s, bar_a, drain;
+    uint32_t tmem_base;
+    int abort_flag;
+};
+static_assert(sizeof(BwdSmem) + 1024 <= kSmemBytes, "shared memory");
+
+struct BwdParams {
+    const __nv_bfloat16 *Q, *K, *V, *O, *dO;
+    const float* lse;
+    const int32_t* idx;
+    const int32_t* cnt;
+    float *dQ, *dK, *dV, *Dbuf;
+    Grid g;
+    int keep;
+    float scale;
+    int* status;
+    uint64_t budget_ns;
+};
+
+__device__ __forceinline__ BwdSmem& smem_layout()
+{
+    extern __shared__ uint8_t raw[];
+    return *reinterpret_cast<BwdSmem*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023));
+}
+
+__device__ __forceinline__ void setup(BwdSmem& sm)
+{
+    if (threadIdx.x == 0) {
+        sm.abort_flag = 0;
+        mbar_init(smem_u32(&sm.bar_s), 1);
+        mbar_init(smem_u32(&sm.bar_a), 1);
+        mbar_init(smem_u32(&sm.drain), 1);
+        fence_mbar_init();
+    }
+    if (threadIdx.x < 32) {
+        tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+}
+
+__device__ __forceinline__ void teardown(BwdSmem& sm, const BwdParams& p, bool dead, uint32_t issued)
+{
+    cp_async_wait<0>();
+    if (dead) {
+        if (threadIdx.x == 0) {
+            if (issued) {  // the MMAs still in flight
+                mma_commit(smem_u32(&sm.drain));
+                const uint64_t t0 = globaltimer_ns();
+                while (!mbar_try_wait(smem_u32(&sm.drain), 0) && globaltimer_ns() - t0 < p.budget_ns) {
+                }
+            }
+            atomicExch(p.status, SSBA_ERR_TIMEOUT);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (threadIdx.x < 32) tmem_dealloc(sm.tmem_base, kTmemCols);
+}
+
+// Writes the 64 x 64 fp32 accumulator at TMEM column `col`, times `mul`, to rows
+// g.token(label, r) of out (one [N][64] head).
+__device__ __forceinline__ void store_acc(uint32_t taddr, float* out, const Grid& g, int label, float mul)
+{
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = lane >> 4;
+    const int r = warp * 16 + (lane & 15);
+    uint32_t v[32];
+    tmem_ld_16x32bx2_x16_off32(taddr, *reinterpret_cast<uint32_t(*)[16]>(&v[0]));
+    tmem_ld_16x32bx2_x16_off32(taddr + 16, *reinterpret_cast<uint32_t(*)[16]>(&v[16]));
+    tmem_wait_ld();
+    float4* dst = reinterpret_cast<float4*>(out + (size_t)g.token(label, r) * kD + 32 * h);
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+        dst[i] = make_float4(__uint_as_float(v[4 * i]) * mul, __uint_as_float(v[4 * i + 1]) * mul,
+                             __uint_as_float(v[4 * i + 2]) * mul, __uint_as_float(v[4 * i + 3]) * mul);
+}
+
+__global__ void __launch_bounds__(kThreads) ssba_bwd_dq_tc_kernel(const BwdParams p)
+{
+    BwdSmem& sm = smem_layout();
+    const int label = blockIdx.x, bh = blockIdx.y;
+    const Grid g = p.g;
+    const int Tb = g.Tb(), N = g.H * g.W;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = lane >> 4;
+    const int r = warp * 16 + (lane & 15);
+    const size_t head = (size_t)bh * N * kD;
+    const size_t row = (size_t)bh * N + g.token(label, r);
+    volatile int* abortf = &sm.abort_flag;
+    setup(sm);
+    const uint32_t tb = sm.tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    const uint32_t tb0 = sm.tmem_base;
+
+    // D for this row (both halves of the row's threads hold it) and the log2-domain lse
+    float Dr = 0.f;
+    {
+        const uint4* go = reinterpret_cast<const uint4*>(p.dO + row * kD + 32 * h);
+        const uint4* oo = reinterpret_cast<const uint4*>(p.O + row * kD + 32 * h);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint4 a = __ldg(go + i), b = __ldg(oo + i);
+            const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 fa = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&aw[k]));
+                const float2 fb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&bw[k]));
+                Dr = fmaf(fa.x, fb.x, Dr);
+                Dr = fmaf(fa.y, fb.y, Dr);
+            }
+        }
+    }
+    Dr += __shfl_xor_sync(0xffffffffu, Dr, 16);
+    if (h == 0) p.Dbuf[row] = Dr;
+    const float c = p.scale * 1.4426950408889634f;
+    const float L2 = p.lse[row] * 1.4426950408889634f;
+
+    const int32_t* list = p.idx + ((size_t)bh * Tb + label) * p.keep;
+    const int n = min(max(p.cnt[(size_t)bh * Tb + label], 0), p.keep);
+    load_tile(smem_u32(sm.a), p.Q + head, g, label);
+    load_tile(smem_u32(sm.b), p.dO + head, g, label);
+    if (n > 0) {
+        const int j0 = min(max(list[0], 0), Tb - 1);
+        load_tile(smem_u32(sm.x[0]), p.K + head, g, j0);
+        load_tile(smem_u32(sm.y[0]), p.V + head, g, j0);
+    }
+    cp_async_commit();
+    bool dead = false;
+    uint32_t issued = 0;
+    for (int t = 0; t < n && !dead; ++t) {
+        const int buf = t & 1;
+        // pair t-1's dQ product has read dS (TMEM over S) and the other buffers: only then may
+        // S be overwritten and those buffers refilled (every wait ends in a CTA-wide vote, so
+        // that no thread leaves the loop while another waits at a barrier in it)
+        if (t >= 1) {
+            const bool ok = mbar_wait(smem_u32(&sm.bar_a), (t - 1) & 1, abortf, p.budget_ns);
+            if (__syncthreads_or(!ok)) {
+                dead = true;
+                break;
+            }
+        }
+        if (t + 1 < n) {
+            const int jn = min(max(list[t + 1], 0), Tb - 1);
+            load_tile(smem_u32(sm.x[buf ^ 1]), p.K + head, g, jn);
+            load_tile(smem_u32(sm.y[buf ^ 1]), p.V + head, g, jn);
+            cp_async_commit();
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        fence_proxy_async_smem();  // the tiles this thread copied, visible to the tensor cores
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            tc_fence_after();
+            mma_kk(tb0 + kColS, smem_u32(sm.a), smem_u32(sm.x[buf]));   // S = Q K^T
+            mma_kk(tb0 + kColDP, smem_u32(sm.b), smem_u32(sm.y[buf]));  // dP = dO V^T
+            mma_commit(smem_u32(&sm.bar_s));
+        }
+        issued = 1;
+        {
+            const bool ok = mbar_wait(smem_u32(&sm.bar_s), t & 1, abortf, p.budget_ns);
+            if (__syncthreads_or(!ok)) {
+                dead = true;
+                break;
+            }
+        }
+        tc_fence_after();
+        uint32_t s[32], dp[32];
+        tmem_ld_16x32bx2_x16_off32(tb + kColS, *reinterpret_cast<uint32_t(*)[16]>(&s[0]));
+        tmem_ld_16x32bx2_x16_off32(tb + kColS + 16, *reinterpret_cast<uint32_t(*)[16]>(&s[16]));
+        tmem_ld_16x32bx2_x16_off32(tb + kColDP, *reinterpret_cast<uint32_t(*)[16]>(&dp[0]));
+        tmem_ld_16x32bx2_x16_off32(tb + kColDP + 16, *reinterpret_cast<uint32_t(*)[16]>(&dp[16]));
+        tmem_wait_ld();
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const float p0 = fast_exp2(fmaf(__uint_as_float(s[2 * i]), c, -L2));
+            const float p1 = fast_exp2(fmaf(__uint_as_float(s[2 * i + 1]), c, -L2));
+            pk[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - Dr), p1 * (__uint_as_float(dp[2 * i + 1]) - Dr));
+        }
+        tmem_st_16x32bx2_x16_off16(tb + kColS, pk);  // dS (bf16 pairs) over S
+        tmem_wait_st();
+        tc_fence_before();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            tc_fence_after();
+            mma_tb(tb0 + kColA0, tb0 + kColS, smem_u32(sm.x[buf]), t > 0);  // dQ += dS K
+            mma_commit(smem_u32(&sm.bar_a));
+        }
+    }
+    if (!dead && n > 0) {
+        const bool ok = mbar_wait(smem_u32(&sm.bar_a), (n - 1) & 1, abortf, p.budget_ns);
+        dead = __syncthreads_or(!ok);
+    }
+    if (!dead) {
+        tc_fence_after();
+        if (n > 0) {
+            store_acc(tb + kColA0, p.dQ + head, g, label, p.scale);
+        } else {
+            float4* dst = reinterpret_cast<float4*>(p.dQ + row * kD + 32 * h);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) dst[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    }
+    teardown(sm, p, dead, issued);
+}
+
+__global__ void __launch_bounds__(kThreads) ssba_bwd_dkdv_tc_kernel(const BwdParams p)
+{
+    BwdSmem& sm = smem_layout();
+    const int label = blockIdx.x, bh = blockIdx.y;
+    const Grid g = p.g;
+    const int Tb = g.Tb(), N = g.H * g.W;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = lane >> 4;
+    const size_t head = (size_t)bh * N * kD;
+    volatile int* abortf = &sm.abort_flag;
+    setup(sm);
+    const uint32_t tb = sm.tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    const uint32_t tb0 = sm.tmem_base;
+    const float c = p.scale * 1.4426950408889634f;
+
+    load_tile(smem_u32(sm.a), p.K + head, g, label);
+    load_tile(smem_u32(sm.b), p.V + head, g, label);
+    cp_async_commit();
+
+    // the query blocks whose lists hold this key block, ascending
+    int total = 0;
+    for (int i0 = 0; i0 < Tb; i0 += kThreads) {
+        const int i = i0 + threadIdx.x;
+        bool has = false;
+        if (i < Tb) {
+            const int32_t* l = p.idx + ((size_t)bh * Tb + i) * p.keep;
+            const int nn = min(max(p.cnt[(size_t)bh * Tb + i], 0), p.keep);
+            for (int t = 0; t < nn; ++t) has |= __ldg(l + t) == label;
+        }
+        const unsigned b = __ballot_sync(0xffffffffu, has);
+        __syncthreads();
+        if (lane == 0) sm.wcount[warp] = __popc(b);
+        __syncthreads();
+        int off = total;
+        for (int w = 0; w < warp; ++w) off += sm.wcount[w];
+        if (has) sm.list[off + __popc(b & ((1u << lane) - 1u))] = i;
+        for (int w = 0; w < kThreads / 32; ++w) total += sm.wcount[w];
+    }
+    __syncthreads();
+    const int n = total;
+
+    auto prefetch = [&](int t, int buf) {
+        const int qi = sm.list[t];
+        load_tile(smem_u32(sm.x[buf]), p.Q + head, g, qi);
+        load_tile(smem_u32(sm.y[buf]), p.dO + head, g, qi);
+        if (threadIdx.x < kT) {
+            const size_t qrow = (size_t)bh * N + g.token(qi, threadIdx.x);
+            sm.ls[buf][threadIdx.x] = __ldg(p.lse + qrow) * 1.4426950408889634f;
+            sm.ds[buf][threadIdx.x] = p.Dbuf[qrow];
+        }
+        cp_async_commit();
+    };
+    if (n > 0) prefetch(0, 0);
+    bool dead = false;
+    uint32_t issued = 0;
+    for (int t = 0; t < n && !dead; ++t) {
+        const int buf = t & 1;
+        // pair t-1's products have read P^T, dS^T (TMEM over S^T, dP^T) and the other buffers
+        if (t >= 1) {
+            const bool ok = mbar_wait(smem_u32(&sm.bar_a), (t - 1) & 1, abortf, p.budget_ns);
+            if (__syncthreads_or(!ok)) {
+                dead = true;
+                break;
+            }
+        }
+        if (t + 1 < n) {
+            prefetch(t + 1, buf ^ 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            tc_fence_after();
+            mma_kk(tb0 + kColS, smem_u32(sm.a), smem_u32(sm.x[buf]));   // S^T = K Q^T
+            mma_kk(tb0 + kColDP, smem_u32(sm.b), smem_u32(sm.y[buf]));  // dP^T = V dO^T
+            mma_commit(smem_u32(&sm.bar_s));
+        }
+        issued = 1;
+        {
+            const bool ok = mbar_wait(smem_u32(&sm.bar_s), t & 1, abortf, p.budget_ns);
+            if (__syncthreads_or(!ok)) {
+                dead = true;
+                break;
+            }
+        }
+        tc_fence_after();
+        uint32_t s[32], dp[32];
+        tmem_ld_16x32bx2_x16_off32(tb + kColS, *reinterpret_cast<uint32_t(*)[16]>(&s[0]));
+        tmem_ld_16x32bx2_x16_off32(tb + kColS + 16, *reinterpret_cast<uint32_t(*)[16]>(&s[16]));
+        tmem_ld_16x32bx2_x16_off32(tb + kColDP, *reinterpret_cast<uint32_t(*)[16]>(&dp[0]));
+        tmem_ld_16x32bx2_x16_off32(tb + kColDP + 16, *reinterpret_cast<uint32_t(*)[16]>(&dp[16]));
+        tmem_wait_ld();
+        // columns are the query rows 32 h + i of the block
+        const float* Lq = sm.ls[buf] + 32 * h;
+        const float* Dq = sm.ds[buf] + 32 * h;
+        uint32_t pp[16], dd[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const float p0 = fast_exp2(fmaf(__uint_as_float(s[2 * i]), c, -Lq[2 * i]));
+            const float p1 = fast_exp2(fmaf(__uint_as_float(s[2 * i + 1]), c, -Lq[2 * i + 1]));
+            pp[i] = pack_bf16(p0, p1);
+            dd[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - Dq[2 * i]),
+                              p1 * (__uint_as_float(dp[2 * i + 1]) - Dq[2 * i + 1]));
+        }
+        tmem_st_16x32bx2_x16_off16(tb + kColS, pp);   // P^T over S^T
+        tmem_st_16x32bx2_x16_off16(tb + kColDP, dd);  // dS^T over dP^T
+        tmem_wait_st();
+        tc_fence_before();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            tc_fence_after();
+            mma_tb(tb0 + kColA0, tb0 + kColS, smem_u32(sm.y[buf]), t > 0);   // dV += P^T dO
+            mma_tb(tb0 + kColA1, tb0 + kColDP, smem_u32(sm.x[buf]), t > 0);  // dK += dS^T Q
+            mma_commit(smem_u32(&sm.bar_a));
+        }
+    }
+    if (!dead && n > 0) {
+        const bool ok = mbar_wait(smem_u32(&sm.bar_a), (n - 1) & 1, abortf, p.budget_ns);
+        dead = __syncthreads_or(!ok);
+    }
+    if (!dead) {
+        tc_fence_after();
+        if (n > 0) {
+            store_acc(tb + kColA0, p.dV + head, g, label, 1.0f);
+            store_acc(tb + kColA1, p.dK + head, g, label, p.scale);
+        } else {
+            const int r = warp * 16 + (lane & 15);
+            const size_t krow = (size_t)bh * N + g.token(label, r);
+            float4* a = reinterpret_cast<float4*>(p.dV + krow * kD + 32 * h);
+            float4* b = reinterpret_cast<float4*>(p.dK + krow * kD + 32 * h);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                a[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+                b[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+        }
+    }
+    teardown(sm, p, dead, issued);
+}
+
+}  // namespace
+
+int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
+                       const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
+                       const int32_t* cnt, float* dQ, float* dK, float* dV, float* Dbuf, cudaStream_t st)
+{
+    if (d.head_dim != kD || g.blk != 8 || d.dtype != SSBA_BF16 || g.Tb() > 256) return SSBA_ERR_UNSUPPORTED;
+    BwdParams p;
+    p.Q = static_cast<const __nv_bfloat16*>(Q);
+    p.K = static_cast<const __nv_bfloat16*>(K);
+    p.V = static_cast<const __nv_bfloat16*>(V);
+    p.O = static_cast<const __nv_bfloat16*>(O);
+    p.dO = static_cast<const __nv_bfloat16*>(dO);
+    p.lse = lse;
+    p.idx = idx;
+    p.cnt = cnt;
+    p.dQ = dQ;
+    p.dK = dK;
+    p.dV = dV;
+    p.Dbuf = Dbuf;
+    p.g = g;
+    p.keep = keep;
+    p.scale = scale;
+    p.budget_ns = kWaitBudgetNs;
+    p.status = device_status_word();
+    if (!p.status) {
+        set_error("ssba_backward: could not resolve the device status word");
+        return SSBA_ERR_CUDA;
+    }
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaFuncSetAttribute(ssba_bwd_dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        cudaFuncSetAttribute(ssba_bwd_dkdv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        attr_set = true;
+    }
+    dim3 grid(g.Tb(), d.B * d.heads);
+    ssba_bwd_dq_tc_kernel<<<grid, kThreads, kSmemBytes, st>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess) {
+        ssba_bwd_dkdv_tc_kernel<<<grid, kThreads, kSmemBytes, st>>>(p);
+        e = cudaGetLastError();
+    }
+    if (e != cudaSuccess) {
+        set_error("ssba_backward (tensor cores) launch: %s", cudaGetErrorString(e));
+        return SSBA_ERR_CUDA;
+    }
+    return SSBA_OK;
+}
+
+}  // namespace ssba

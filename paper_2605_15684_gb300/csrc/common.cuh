@@ -69,6 +69,12 @@ int launch_backward(const ssba_desc& d, const Grid& g, int keep, float scale, co
                     const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
                     const int32_t* cnt, float* dQ, float* dK, float* dV, float* Dbuf, cudaStream_t st);
 
+// The same gradients on the tensor cores (bf16, head_dim 64, 8x8 blocks, Tb <= 256); returns
+// SSBA_ERR_UNSUPPORTED without launching for other shapes.
+int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
+                       const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
+                       const int32_t* cnt, float* dQ, float* dK, float* dV, float* Dbuf, cudaStream_t st);
+
 int launch_haar(bool inverse, const void* in, void* out, int N, int C, int H, int W, int nb, int dtype,
                 cudaStream_t st);
 int launch_qkv_rope_pool(const ssba_desc& d, const Grid& g, const void* X, const void* Wqkv, const float* bias,
