@@ -52,13 +52,36 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
+// Token of in-window position pos of the window whose unshifted origin is (r0, c0) (the map of
+// Grid::token with blk = 8, the window origin computed once per tile).
+struct WinOrigin {
+    int r0, c0;
+};
+__device__ __forceinline__ WinOrigin win_origin(const Grid& g, int label)
+{
+    const int br = label / g.bw, bc = label - br * g.bw;
+    int r0 = br * 8 - g.sr, c0 = bc * 8 - g.sc;
+    r0 += r0 < 0 ? g.H : 0;
+    c0 += c0 < 0 ? g.W : 0;
+    return {r0, c0};
+}
+__device__ __forceinline__ int win_token(const Grid& g, WinOrigin o, int pos)
+{
+    int r = o.r0 + (pos >> 3), c = o.c0 + (pos & 7);
+    r -= r >= g.H ? g.H : 0;
+    c -= c >= g.W ? g.W : 0;
+    return r * g.W + c;
+}
+
 // Block `label` of a [N][64] bf16 head into a 1024-aligned 8 KB tile: row r = in-window
 // position r, 16-byte chunk c at chunk c ^ (r & 7) (the 128-byte swizzle).
 __device__ __forceinline__ void load_tile(uint32_t dst, const __nv_bfloat16* X, const Grid& g, int label)
 {
-    for (int e = threadIdx.x; e < kT * 8; e += kThreads) {
-        const int r = e >> 3, c = e & 7;
-        cp_async16(dst + r * 128 + ((c ^ (r & 7)) << 4), X + (size_t)g.token(label, r) * kD + c * 8);
+    const WinOrigin o = win_origin(g, label);
+#pragma unroll
+    for (int i = 0; i < kT * 8 / kThreads; ++i) {
+        const int e = threadIdx.x + i * kThreads, r = e >> 3, c = e & 7;
+        cp_async16(dst + r * 128 + ((c ^ (r & 7)) << 4), X + (size_t)win_token(g, o, r) * kD + c * 8);
     }
 }
 
@@ -336,7 +359,14 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dkdv_tc_kernel(const BwdPar
         if (i < Tb) {
             const int32_t* l = p.idx + ((size_t)bh * Tb + i) * p.keep;
             const int nn = min(max(p.cnt[(size_t)bh * Tb + i], 0), p.keep);
-            for (int t = 0; t < nn; ++t) has |= __ldg(l + t) == label;
+            // four list entries in flight at a time
+            for (int t = 0; t < nn; t += 4) {
+                int v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) v[u] = t + u < nn ? __ldg(l + t + u) : -1;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) has |= v[u] == label;
+            }
         }
         const unsigned b = __ballot_sync(0xffffffffu, has);
         __syncthreads();
@@ -355,7 +385,7 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dkdv_tc_kernel(const BwdPar
         load_tile(smem_u32(sm.x[buf]), p.Q + head, g, qi);
         load_tile(smem_u32(sm.y[buf]), p.dO + head, g, qi);
         if (threadIdx.x < kT) {
-            const size_t qrow = (size_t)bh * N + g.token(qi, threadIdx.x);
+            const size_t qrow = (size_t)bh * N + win_token(g, win_origin(g, qi), threadIdx.x);
             sm.ls[buf][threadIdx.x] = __ldg(p.lse + qrow) * 1.4426950408889634f;
             sm.ds[buf][threadIdx.x] = p.Dbuf[qrow];
         }
