@@ -207,6 +207,22 @@ SSBA_API int ssba_forward_select(const ssba_desc* desc, const void* Q, const voi
                                  float* scores_opt, void* O, float* lse, void* workspace, size_t ws_bytes,
                                  void* stream);
 
+/* The whole of Algorithm 1 after RoPE in one launch (Sec. 2.2): block compression (the means
+ * q_b, k_b, with the pooling arithmetic of ssba_pool_blocks, so the same Q, K give the same
+ * means and lists), affinity, Top-k gating and the sparse attention. The persistent grid (one
+ * CTA per SM) first pools every block of the layer into qb / kb, meets at a grid-wide barrier
+ * (bounded wait; a timeout returns through ssba_get_status as SSBA_ERR_TIMEOUT, with O and
+ * the lists not written), then runs ssba_forward_select on those means.
+ *   qb, kb      device out, fp32 [B][heads][Tb][head_dim], 16-byte aligned: the block means.
+ *   workspace   REQUIRED here, at least ssba_forward_workspace_bytes(desc) bytes: it holds the
+ *               barrier's counters. The rules of ssba_forward's workspace hold (zero-filled before
+ *               first use, left zero-filled, zeroed again after SSBA_ERR_TIMEOUT, one per stream).
+ *   the rest    as ssba_forward_select.
+ * bf16 only; Tb <= 128 (else SSBA_ERR_UNSUPPORTED); SSBA_ERR_WORKSPACE without a workspace. */
+SSBA_API int ssba_forward_fused(const ssba_desc* desc, const void* Q, const void* K, const void* V, float* qb,
+                                float* kb, int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O,
+                                float* lse, void* workspace, size_t ws_bytes, void* stream);
+
 /* One level of the T-DVAE's 2-D Haar kernel bank F = {LL, HL, LH, HH} (Sec. 2.3
  * DWT-Enhanced Architecture), per channel, stride 2, orthonormal: for the window
  * a = x[2i][2j], b = x[2i][2j+1], c = x[2i+1][2j], d = x[2i+1][2j+1],

@@ -30,7 +30,7 @@ EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
             "ssba_test_forward_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
             "ssba_haar_iwt", "ssba_haar_dwt_pyramid", "ssba_haar_iwt_pyramid", "ssba_qkv_rope_pool",
-            "ssba_select_mask", "ssba_pool_blocks", "ssba_forward_select",
+            "ssba_select_mask", "ssba_pool_blocks", "ssba_forward_select", "ssba_forward_fused",
             "ssba_get_status", "ssba_last_error")
 
 
@@ -112,6 +112,8 @@ def load_library():
         lib.ssba_pool_blocks.restype = ctypes.c_int
         lib.ssba_forward_select.argtypes = [DP, P, P, P, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_forward_select.restype = ctypes.c_int
+        lib.ssba_forward_fused.argtypes = [DP, P, P, P, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
+        lib.ssba_forward_fused.restype = ctypes.c_int
         lib.ssba_forward.argtypes = [DP, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_forward.restype = ctypes.c_int
         lib.ssba_forward_joint.argtypes = [DP, P, P, P, P, P, ctypes.c_int32, P, P, P, P, P, ctypes.c_size_t, P]
@@ -324,19 +326,19 @@ def pool_blocks(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, qb=None, kb=No
     return qb, kb
 
 
-def forward_select(desc: SsbaDesc, Q, K, V, qb, kb, kv_idx=None, kv_cnt=None, scores: bool | torch.Tensor = False,
-                   O=None, lse=None, workspace="default", stream=None):
-    """ssba_forward_select: selection inside the attention launch. Returns (O, lse, kv_idx, kv_cnt[, S])."""
+def _forward_select_call(fn_name, desc, Q, K, V, qb, kb, kv_idx, kv_cnt, scores, O, lse, workspace, stream):
     lib = load_library()
     d = desc.c()
     keep = keep_count(desc)
     shp = (desc.B, desc.heads, desc.N, desc.head_dim)
     for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
         _check(t, n, shp, desc.dtype)
+    dev = Q.device
     pshp = (desc.B, desc.heads, desc.Tb, desc.head_dim)
+    qb = torch.empty(pshp, dtype=torch.float32, device=dev) if qb is None else qb
+    kb = torch.empty(pshp, dtype=torch.float32, device=dev) if kb is None else kb
     _check(qb, "qb", pshp, torch.float32)
     _check(kb, "kb", pshp, torch.float32)
-    dev = Q.device
     kv_idx = torch.empty((desc.B, desc.heads, desc.Tb, keep), dtype=torch.int32, device=dev) if kv_idx is None \
         else kv_idx
     kv_cnt = torch.empty((desc.B, desc.heads, desc.Tb), dtype=torch.int32, device=dev) if kv_cnt is None else kv_cnt
@@ -355,11 +357,32 @@ def forward_select(desc: SsbaDesc, Q, K, V, qb, kb, kv_idx=None, kv_cnt=None, sc
     if isinstance(workspace, str):
         workspace = default_forward_workspace(desc, dev)
     wp, wn = _ws_args(workspace)
-    _raise_on(lib.ssba_forward_select(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), qb.data_ptr(),
-                                      kb.data_ptr(), kv_idx.data_ptr(), kv_cnt.data_ptr(),
-                                      S.data_ptr() if S is not None else None, O.data_ptr(), lse.data_ptr(), wp, wn,
-                                      _stream_ptr(stream)))
+    _raise_on(getattr(lib, fn_name)(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), qb.data_ptr(),
+                                    kb.data_ptr(), kv_idx.data_ptr(), kv_cnt.data_ptr(),
+                                    S.data_ptr() if S is not None else None, O.data_ptr(), lse.data_ptr(), wp, wn,
+                                    _stream_ptr(stream)))
+    return qb, kb, kv_idx, kv_cnt, S, O, lse
+
+
+def forward_select(desc: SsbaDesc, Q, K, V, qb, kb, kv_idx=None, kv_cnt=None, scores: bool | torch.Tensor = False,
+                   O=None, lse=None, workspace="default", stream=None):
+    """ssba_forward_select: selection inside the attention launch. Returns (O, lse, kv_idx, kv_cnt[, S])."""
+    if qb is None or kb is None:
+        raise SsbaError(SSBA_ERR_INVALID, "forward_select needs the block means qb, kb")
+    _, _, kv_idx, kv_cnt, S, O, lse = _forward_select_call("ssba_forward_select", desc, Q, K, V, qb, kb, kv_idx,
+                                                           kv_cnt, scores, O, lse, workspace, stream)
     return (O, lse, kv_idx, kv_cnt, S) if S is not None else (O, lse, kv_idx, kv_cnt)
+
+
+def forward_fused(desc: SsbaDesc, Q, K, V, qb=None, kb=None, kv_idx=None, kv_cnt=None,
+                  scores: bool | torch.Tensor = False, O=None, lse=None, workspace="default", stream=None):
+    """ssba_forward_fused: pooling, selection and attention in one launch.
+    Returns (O, lse, kv_idx, kv_cnt, qb, kb[, S])."""
+    if workspace is None:
+        raise SsbaError(SSBA_ERR_WORKSPACE, "forward_fused needs a forward workspace")
+    qb, kb, kv_idx, kv_cnt, S, O, lse = _forward_select_call("ssba_forward_fused", desc, Q, K, V, qb, kb, kv_idx,
+                                                             kv_cnt, scores, O, lse, workspace, stream)
+    return (O, lse, kv_idx, kv_cnt, qb, kb, S) if S is not None else (O, lse, kv_idx, kv_cnt, qb, kb)
 
 
 def build_mask_noalloc(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=None, kv_cnt=None,
@@ -634,8 +657,9 @@ def realized_sparsity(desc: SsbaDesc) -> float:
 
 class BoundSelectLayer:
     """One SSBA layer on the one-launch selection path: ``pool()`` (ssba_pool_blocks) and
-    ``attend()`` (ssba_forward_select, which also writes the kept-block lists), buffers
-    validated once and bare C calls after that."""
+    ``attend()`` (ssba_forward_select, which also writes the kept-block lists), or ``fused()``
+    (ssba_forward_fused: both in one launch), buffers validated once and bare C calls after
+    that."""
 
     def __init__(self, desc: SsbaDesc, Q, K, V, qb, kb, kv_idx, kv_cnt, O, lse, stream=None,
                  fwd_workspace="default"):
@@ -655,6 +679,8 @@ class BoundSelectLayer:
         if isinstance(fwd_workspace, str):
             fwd_workspace = default_forward_workspace(desc, Q.device)
         fwp, fwn = _ws_args(fwd_workspace)
+        if fwp is not None and fwn < forward_workspace_bytes(desc):
+            raise SsbaError(SSBA_ERR_WORKSPACE, f"forward workspace needs {forward_workspace_bytes(desc)} bytes")
         self.tensors = (Q, K, V, qb, kb, kv_idx, kv_cnt, O, lse, fwd_workspace)  # keep alive
         st = _stream_ptr(stream)
         self._pool_args = (ctypes.byref(self._d), Q.data_ptr(), K.data_ptr(), qb.data_ptr(), kb.data_ptr(), st)
@@ -669,6 +695,11 @@ class BoundSelectLayer:
 
     def attend(self) -> None:
         rc = self._lib.ssba_forward_select(*self._fwd_args)
+        if rc:
+            _raise_on(rc)
+
+    def fused(self) -> None:
+        rc = self._lib.ssba_forward_fused(*self._fwd_args)
         if rc:
             _raise_on(rc)
 

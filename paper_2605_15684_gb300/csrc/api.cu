@@ -259,31 +259,53 @@ int ssba_pool_blocks(const ssba_desc* desc, const void* Q, const void* K, float*
     return launch_pool_blocks(*desc, g, Q, K, qb, kb, static_cast<cudaStream_t>(stream));
 }
 
-int ssba_forward_select(const ssba_desc* desc, const void* Q, const void* K, const void* V, const float* qb,
-                        const float* kb, int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O, float* lse,
-                        void* workspace, size_t ws_bytes, void* stream)
+namespace {
+int forward_select_impl(const char* name, bool pool, const ssba_desc* desc, const void* Q, const void* K,
+                        const void* V, const float* qb, const float* kb, int32_t* kv_idx, int32_t* kv_cnt,
+                        float* scores_opt, void* O, float* lse, void* workspace, size_t ws_bytes, void* stream)
 {
     Grid g;
     int keep;
-    int rc = check_desc(desc, "ssba_forward_select", &g, &keep);
+    int rc = check_desc(desc, name, &g, &keep);
     if (rc != SSBA_OK) return rc;
     if (!Q || !K || !V || !qb || !kb || !kv_idx || !kv_cnt || !O || !lse) {
-        set_error("ssba_forward_select: every pointer but scores_opt must be non-null");
+        set_error("%s: every pointer but scores_opt must be non-null", name);
         return SSBA_ERR_INVALID;
     }
     if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(qb, 16) ||
         !aligned(kb, 16) || !aligned(lse, 4) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) ||
         (scores_opt && !aligned(scores_opt, 4)) || (workspace && !aligned(workspace, 16))) {
-        set_error("ssba_forward_select: Q, K, V, O, qb, kb, workspace 16-byte aligned; the rest 4-byte aligned");
+        set_error("%s: Q, K, V, O, qb, kb, workspace 16-byte aligned; the rest 4-byte aligned", name);
         return SSBA_ERR_INVALID;
     }
     if (desc->dtype != SSBA_BF16) {
-        set_error("ssba_forward_select: bf16 only (the tensor-core path)");
+        set_error("%s: bf16 only (the tensor-core path)", name);
         return SSBA_ERR_UNSUPPORTED;
+    }
+    if (pool && !workspace) {
+        set_error("%s: needs a workspace of ssba_forward_workspace_bytes(desc) bytes", name);
+        return SSBA_ERR_WORKSPACE;
     }
     return launch_attn_tc_bf16(*desc, g, keep, resolve_scale(desc), Q, K, V, kv_idx, kv_cnt, O, lse, workspace,
                                ws_bytes, static_cast<cudaStream_t>(stream), kWaitBudgetNs, 0, nullptr, nullptr, 0, qb,
-                               kb, scores_opt);
+                               kb, scores_opt, pool);
+}
+}  // namespace
+
+int ssba_forward_select(const ssba_desc* desc, const void* Q, const void* K, const void* V, const float* qb,
+                        const float* kb, int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O, float* lse,
+                        void* workspace, size_t ws_bytes, void* stream)
+{
+    return forward_select_impl("ssba_forward_select", false, desc, Q, K, V, qb, kb, kv_idx, kv_cnt, scores_opt, O,
+                               lse, workspace, ws_bytes, stream);
+}
+
+int ssba_forward_fused(const ssba_desc* desc, const void* Q, const void* K, const void* V, float* qb, float* kb,
+                       int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O, float* lse, void* workspace,
+                       size_t ws_bytes, void* stream)
+{
+    return forward_select_impl("ssba_forward_fused", true, desc, Q, K, V, qb, kb, kv_idx, kv_cnt, scores_opt, O, lse,
+                               workspace, ws_bytes, stream);
 }
 
 int ssba_forward_joint(const ssba_desc* desc, const void* Q, const void* K, const void* V, const void* K_txt,

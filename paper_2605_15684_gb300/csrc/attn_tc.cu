@@ -115,6 +115,7 @@ constexpr int kWinCap = 256;  // labels whose window (origin, box shape) is tabu
 struct __align__(1024) SmemLayout {
     SlotSmem slot[kSlots];
     uint32_t win[kWinCap];  // label -> r0 | c0 << 15 | box shape << 30 (see window_entry)
+    uint64_t pool_bar[kThreads / 32];  // one per warp: its block's rows landed (in-kernel pooling)
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -148,6 +149,11 @@ struct TcParams {
     const float* sel_kb;
     int32_t* sel_cnt;     // counts written by the selection
     float* sel_scores;    // optional S export [B*heads][Tb][Tb]
+    // in-kernel pooling (ssba_forward_fused): every warp of the grid pools one (block, tensor)
+    // unit into sel_qb / sel_kb, then the CTAs meet at a grid barrier (null: means given)
+    const __nv_bfloat16* pool_q;
+    const __nv_bfloat16* pool_k;
+    unsigned* gsync;  // grid barrier words in the workspace (arrivals, departures)
     uint64_t budget_ns;  // wall-time limit of every barrier wait
     int withhold;        // test hook: pipeline 0 announces its first K copy but never issues it,
                          // so that the waits on it run out (failure-detection test only)
@@ -229,6 +235,106 @@ __device__ __forceinline__ void tmem_st_16x32bx2_x16_off32(uint32_t taddr, const
 }
 
 __device__ __forceinline__ int clamp_label(int j, int Tb) { return j < 0 ? 0 : (j >= Tb ? Tb - 1 : j); }
+
+// Block means of the whole layer inside the launch: unit u is (tensor u & 1, item u >> 1), one
+// unit per warp and round, assigned warp-major over the grid so that the CTAs get equal
+// shares. Lanes 0..7 bulk-copy the unit's eight token rows (one copy per row, two where the
+// shifted window wraps the right edge) into this warp's 8 KB of the idle stage buffers, and
+// after the copies land every lane sums its (row group, column chunk) with the loop order of
+// ssba_pool_blocks_kernel, so the means are those of ssba_pool_blocks bit for bit. Returns
+// false if a copy did not land in time (after a second bounded wait for it).
+__device__ __noinline__ bool pool_phase(const TcParams& p, SmemLayout& cs, int gwarp, int lane, volatile int* abortf)
+{
+    constexpr int VE = 8, CPR = kD / VE, RPI = 32 / CPR, LOADS = 64 / RPI;
+    constexpr int kWarps = kThreads / 32, kPerSlot = kWarps / kSlots;
+    static_assert(kPerSlot * kTileBytes <= (kKStages + kVStages + 2) * kTileBytes, "pool buffers");
+    const Grid& g = p.g;
+    const int Tb = g.Tb(), N = g.H * g.W;
+    const int col = lane % CPR, r0 = lane / CPR;
+    const uint8_t* buf = &cs.slot[gwarp / kPerSlot].k[0][0] + (gwarp % kPerSlot) * kTileBytes;
+    const uint32_t bar = smem_u32(&cs.pool_bar[gwarp]);
+    const int nw = gridDim.x * kWarps;
+    int round = 0;
+    for (int u = gwarp * gridDim.x + blockIdx.x; u < 2 * p.num_items; u += nw, ++round) {
+        const int which = u & 1, item = u >> 1;
+        const int bh = item / Tb, label = item - bh * Tb;
+        const int br = label / g.bw, bc = label - br * g.bw;
+        const int rb = br * 8 - g.sr, cb = bc * 8 - g.sc;
+        if (round > 0) {
+            __syncwarp();
+            fence_proxy_async_smem();  // the last round's reads before the copies overwrite them
+        }
+        if (lane == 0) mbar_arrive_expect_tx(bar, kTileBytes);
+        __syncwarp();
+        if (lane < 8) {
+            const __nv_bfloat16* X = (which ? p.pool_k : p.pool_q) + (size_t)bh * N * kD;
+            int r = rb + lane;
+            r += r < 0 ? g.H : 0;
+            const uint32_t dst = smem_u32(buf) + lane * 8 * kD * 2;
+            // columns cb .. cb + 7 with -W < cb <= W - 8, each negative one taken + W
+            if (cb >= 0 || cb <= -8) {  // one run of 8 columns
+                bulk_load(dst, X + (size_t)(r * g.W + (cb < 0 ? cb + g.W : cb)) * kD, 8 * kD * 2, bar);
+            } else {  // columns W + cb .. W - 1, then 0 .. 7 + cb
+                const int n1 = -cb;  // 1 .. 7
+                bulk_load(dst, X + (size_t)(r * g.W + g.W + cb) * kD, n1 * kD * 2, bar);
+                bulk_load(dst + n1 * kD * 2, X + (size_t)r * g.W * kD, (8 - n1) * kD * 2, bar);
+            }
+        }
+        if (!mbar_wait(bar, round & 1, abortf, p.budget_ns)) {
+            volatile int never = 0;  // wait once more, for the copies only, before giving up
+            mbar_wait(bar, round & 1, &never, p.budget_ns);
+            return false;
+        }
+        float acc[VE];
+#pragma unroll
+        for (int e = 0; e < VE; ++e) acc[e] = 0.f;
+#pragma unroll
+        for (int i = 0; i < LOADS; ++i) {
+            const int pos = r0 + i * RPI;
+            const uint4 v = *reinterpret_cast<const uint4*>(buf + (pos * kD + col * VE) * 2);
+            const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float2 f = __bfloat1622float2(h2[e]);
+                acc[2 * e] += f.x;
+                acc[2 * e + 1] += f.y;
+            }
+        }
+#pragma unroll
+        for (int o = CPR; o < 32; o <<= 1)
+#pragma unroll
+            for (int e = 0; e < VE; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+        if (r0 == 0) {
+            float* dst = const_cast<float*>(which ? p.sel_kb : p.sel_qb) + ((size_t)bh * Tb + label) * kD + col * VE;
+            constexpr float kInv = 1.0f / 64.0f;
+            reinterpret_cast<float4*>(dst)[0] = make_float4(acc[0] * kInv, acc[1] * kInv, acc[2] * kInv, acc[3] * kInv);
+            reinterpret_cast<float4*>(dst)[1] = make_float4(acc[4] * kInv, acc[5] * kInv, acc[6] * kInv, acc[7] * kInv);
+        }
+    }
+    return true;
+}
+
+// Grid-wide barrier for a persistent launch whose CTAs are all resident (one per SM, grid at
+// most the SM count; the next grid is released only after it). w[0] counts arrivals, w[1]
+// departures; the last CTA to depart sets both back to zero, so a call that completes leaves
+// the workspace zero-filled. Waits are bounded; returns false on timeout or abort (the words
+// are then left as they are, like the rest of the workspace after a timeout).
+__device__ bool grid_barrier(unsigned* w, unsigned n, volatile int* abortf, uint64_t budget_ns)
+{
+    __threadfence();
+    atomicAdd(&w[0], 1u);
+    const uint64_t t0 = globaltimer_ns();
+    while (*reinterpret_cast<volatile unsigned*>(&w[0]) != n) {
+        if (*abortf || globaltimer_ns() - t0 > budget_ns) return false;
+        __nanosleep(64);
+    }
+    __threadfence();
+    if (atomicAdd(&w[1], 1u) == n - 1) {  // every CTA has seen w[0] == n
+        atomicExch(&w[0], 0u);
+        atomicExch(&w[1], 0u);
+    }
+    return true;
+}
 
 // A list entry: written earlier in this launch under in-kernel selection (read through L2),
 // else read-only input.
@@ -451,12 +557,31 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         mbar_init(smem_u32(&sm.o_free), 4);
         mbar_init(smem_u32(&sm.drain[0]), 1);
         mbar_init(smem_u32(&sm.drain[1]), 1);
+        if (p.pool_q)
+            for (int w = slot * kSlotWarps; w < (slot + 1) * kSlotWarps; ++w) mbar_init(smem_u32(&cs.pool_bar[w]), 1);
         fence_mbar_init();
     }
     for (int l = threadIdx.x; l < Tb && l < kWinCap; l += kThreads) cs.win[l] = window_entry(g, l);
     // everything above reads no input; the lists, counts and tensors may come from the grid
     // launched just before this one (programmatic dependent launch)
     grid_dep_wait();
+    if (p.pool_q) {
+        bool pool_fail = false;
+        // the block means of the whole layer: every warp of the grid one (block, tensor) unit,
+        // then a grid barrier; the next grid is released only after it, so that it cannot take
+        // an SM that one of these CTAs still waits for
+        __syncthreads();  // the pooling barriers are initialised
+        pool_fail = !pool_phase(p, cs, gwarp, lane, abortf);
+        __threadfence();  // this CTA's means, visible to the whole GPU before it arrives
+        pool_fail = __syncthreads_or(pool_fail);
+        if (threadIdx.x == 0 && !pool_fail) pool_fail = !grid_barrier(p.gsync, gridDim.x, abortf, p.budget_ns);
+        if (__syncthreads_or(pool_fail)) {
+            // nothing allocated or in flight yet: report and leave (the means of the other CTAs
+            // may be missing, so no list of this CTA can be trusted)
+            if (threadIdx.x == 0) atomicExch(p.status, SSBA_ERR_TIMEOUT);
+            return;
+        }
+    }
     grid_dep_launch();
     if (p.sel_qb) {
         // the lists of this CTA's items (the contiguous ranges of its two pipelines): the k_b
@@ -518,7 +643,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     float* own = reinterpret_cast<float*>(keys) + 128;  // after its keys
                     if (lane < kD / 4)
                         reinterpret_cast<float4*>(own)[lane] =
-                            __ldg(reinterpret_cast<const float4*>(p.sel_qb + (size_t)item * kD) + lane);
+                            __ldcg(reinterpret_cast<const float4*>(p.sel_qb + (size_t)item * kD) + lane);
                     __syncwarp();
                     qs = own;
                 }
@@ -535,6 +660,9 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         tmem_alloc(smem_u32(&cs.tmem_base), kTmemCols);
         tmem_relinquish();
     }
+    // the stage buffers held the pooled rows and the staged means (generic accesses); the
+    // producers' tensor copies (async proxy) overwrite them next
+    if (p.sel_qb) fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -1053,13 +1181,19 @@ size_t ws_st_bytes() { return align256(ws_boundaries() * 2 * kRows * sizeof(floa
 size_t ws_o_bytes() { return ws_boundaries() * 2 * kRows * kD * sizeof(float); }
 }  // namespace
 
-size_t attn_tc_workspace_bytes() { return ws_cnt_bytes() + ws_st_bytes() + ws_o_bytes(); }
+// ... then 256 bytes for the grid barrier words of the launch that pools.
+size_t attn_tc_workspace_bytes() { return ws_cnt_bytes() + ws_st_bytes() + align256(ws_o_bytes()) + 256; }
 
 int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
                         const void* V, const int32_t* idx, const int32_t* cnt, void* O, float* lse, void* ws,
                         size_t ws_bytes, cudaStream_t st, uint64_t budget_ns, int withhold, const void* Kt,
-                        const void* Vt, int t_txt, const float* sel_qb, const float* sel_kb, float* sel_scores)
+                        const void* Vt, int t_txt, const float* sel_qb, const float* sel_kb, float* sel_scores,
+                        bool pool)
 {
+    if (pool && (!ws || !sel_qb || !sel_kb)) {
+        set_error("ssba_forward_fused: needs a forward workspace and the block-mean buffers");
+        return SSBA_ERR_WORKSPACE;
+    }
     if (sel_qb && (g.Tb() > 128 || t_txt > 0 || !idx || !cnt)) {
         set_error("ssba_forward_select: needs Tb <= 128, no text segment and list outputs");
         return SSBA_ERR_UNSUPPORTED;
@@ -1106,6 +1240,11 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
     p.sel_kb = sel_kb;
     p.sel_cnt = const_cast<int32_t*>(cnt);
     p.sel_scores = sel_scores;
+    p.pool_q = pool ? static_cast<const __nv_bfloat16*>(Q) : nullptr;
+    p.pool_k = pool ? static_cast<const __nv_bfloat16*>(K) : nullptr;
+    p.gsync = pool ? reinterpret_cast<unsigned*>(static_cast<char*>(ws) + ws_cnt_bytes() + ws_st_bytes() +
+                                                 align256(ws_o_bytes()))
+                   : nullptr;
     p.status = device_status_word();
     if (!p.status) {
         set_error("ssba_forward (bf16): could not resolve the device status word");

@@ -59,7 +59,7 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
                         float* lse, void* ws, size_t ws_bytes, cudaStream_t st,
                         uint64_t budget_ns = kWaitBudgetNs, int withhold = 0, const void* Kt = nullptr,
                         const void* Vt = nullptr, int t_txt = 0, const float* sel_qb = nullptr,
-                        const float* sel_kb = nullptr, float* sel_scores = nullptr);
+                        const float* sel_kb = nullptr, float* sel_scores = nullptr, bool pool = false);
 int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V,
                          void* O, float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
 // Bytes of the split-merge workspace of the bf16 forward on the current device.

@@ -181,14 +181,6 @@ __device__ __forceinline__ void tile_rc(const TileGeo& o, int rho, int& a, int& 
     }
 }
 
-// One bulk copy global -> shared (16-byte aligned, size a multiple of 16), counted on bar.
-__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar)
-{
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-                 "l"(src), "r"(bytes), "r"(bar)
-                 : "memory");
-}
-
 __device__ __forceinline__ uint32_t pack2(float lo, float hi)
 {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);

@@ -222,6 +222,18 @@ def test_pool_and_select_forward_validation(lib):
     # rows longer than 128 blocks: the two-launch path
     assert fs(desc(H_tok=96, W_tok=96), good) == api.SSBA_ERR_UNSUPPORTED
     assert b"Tb <= 128" in lib.ssba_last_error()
+    # the fused launch: the same checks, and a workspace is required (it holds the barrier)
+    ff = lambda dd, v, n=0: lib.ssba_forward_fused(ctypes.byref(dd), *v, n, None)
+    bad = list(good)
+    bad[10] = None
+    assert ff(d, bad) == api.SSBA_ERR_WORKSPACE
+    assert b"workspace" in lib.ssba_last_error()
+    bad = list(good)
+    bad[4] = FAKE + 4  # misaligned kb
+    assert ff(d, bad) == api.SSBA_ERR_INVALID
+    assert ff(desc(dtype=api.SSBA_FP32), good) == api.SSBA_ERR_UNSUPPORTED
+    assert ff(desc(H_tok=96, W_tok=96), good) == api.SSBA_ERR_UNSUPPORTED
+    assert b"Tb <= 128" in lib.ssba_last_error()
 
 
 def ct_byref(d):

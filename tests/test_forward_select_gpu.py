@@ -60,6 +60,60 @@ def test_forward_select_matches_oracle(B, h, H, W, shift, rho, std):
     check_out(O.float().cpu().numpy(), lse.cpu().numpy(), Oo, lo, "bf16")
 
 
+@pytest.mark.parametrize("B,h,H,W,shift,rho", [
+    (1, 4, 16, 16, (4, 4), 0.75),       # 8 CTAs
+    (1, 24, 64, 64, (4, 4), 0.8416),    # 1024 px headline, shifted layer: the full grid
+    (1, 24, 64, 64, (0, 0), 0.8416),
+    (2, 3, 24, 40, (4, -4), 0.6),       # odd block count; column shift 36: whole windows wrap
+    (1, 8, 64, 64, (12, 52), 0.8416),   # shifts past one block on both axes
+    (1, 2, 88, 88, (4, 4), 0.9),        # Tb = 121
+    (1, 48, 64, 64, (4, 4), 0.8416),    # more units than warps in the grid: several per warp
+])
+def test_forward_fused_equals_two_launches(B, h, H, W, shift, rho):
+    """ssba_forward_fused pools inside the launch with the arithmetic of ssba_pool_blocks:
+    means, lists, scores, O and lse identical to pool_blocks + forward_select, which the test
+    above pins to the oracle; and the grid barrier's counters are back at zero afterwards."""
+    desc, _, (qb, kb), (O, lse, idx, cnt, S) = _case(B, h, H, W, shift, rho, seed=11)
+    q, k, v = (t.cuda() for t in synthetic.qkv(B, h, H * W, 64, torch.bfloat16, 11, 1.0))
+    ws = torch.zeros(api.forward_workspace_bytes(desc), dtype=torch.uint8, device="cuda")
+    for _ in range(3):  # repeated launches on one workspace
+        O2, l2, i2, c2, qb2, kb2, S2 = api.forward_fused(desc, q, k, v, scores=True, workspace=ws)
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
+    assert torch.equal(qb2, qb) and torch.equal(kb2, kb)
+    assert torch.equal(i2, idx) and torch.equal(c2, cnt) and torch.equal(S2, S)
+    assert torch.equal(O2, O) and torch.equal(l2, lse)
+    assert int(ws[-256:].count_nonzero()) == 0
+
+
+def test_forward_fused_graph_replay():
+    """The fused launch captured in a CUDA graph and replayed: same results each replay."""
+    B, h, H, W = 1, 24, 64, 64
+    desc = api.SsbaDesc(B, h, H, W, shift_r=4, shift_c=4, rho=0.8416, dtype=torch.bfloat16)
+    q, k, v = (t.cuda() for t in synthetic.qkv(B, h, H * W, 64, torch.bfloat16, 5, 1.0))
+    ref = api.forward_fused(desc, q, k, v)
+    torch.cuda.synchronize()
+    outs = [torch.empty_like(t) for t in ref]
+    ws = api.default_forward_workspace(desc, q.device)
+    st = torch.cuda.Stream()
+    st.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(st):
+        layer = api.BoundSelectLayer(desc, q, k, v, outs[4], outs[5], outs[2], outs[3], outs[0], outs[1],
+                                     stream=st, fwd_workspace=ws)
+        layer.fused()  # warm-up outside the capture
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=st):
+            layer.fused()
+    for _ in range(3):
+        for t in outs:
+            t.zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        assert api.get_status() == api.SSBA_OK
+        for a, b in zip(outs, ref):
+            assert torch.equal(a, b)
+
+
 def test_forward_select_without_workspace_matches_default():
     args = (1, 4, 32, 32, (4, 4), 0.75)
     _, _, _, (O1, l1, i1, c1, _) = _case(*args, seed=3)
