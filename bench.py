@@ -4,10 +4,10 @@
 A step is one pass of the whole hot path over one batch: the 24 SSBA layers of the
 1024 px DiT (64 x 64 image tokens, B=1, 24 heads x 64, rho = 0.8416 -> keep 11 of 64
 blocks per query block), layer l with window shift (0,0) if l is even else (4,4); each
-layer pools its block means from its own Q/K (ssba_pool_blocks) and then runs one launch
-that computes the affinities, selects the kept blocks and runs the block-sparse forward
-(ssba_forward_select). The two-launch path (ssba_build_mask + ssba_forward) is measured
-beside it, outside the timed region. Each
+layer is one launch (ssba_forward_fused) that pools the block means from its own Q/K,
+computes the affinities, selects the kept blocks and runs the block-sparse forward. The
+pooling as a launch of its own (ssba_pool_blocks + ssba_forward_select) and the two-launch
+path (ssba_build_mask + ssba_forward) are measured beside it, outside the timed region. Each
 layer has its own seeded synthetic Q/K/V (906 MB in all), so every layer's inputs are
 cold in L2 when it runs.
 
@@ -91,7 +91,7 @@ def config_dict(w, keep, layers):
     Tb = w.N // 64
     return {
         "workload": f"{w.name} x{layers} layers, shifts (0,0)/(4,4) alternating, mask rebuilt per layer "
-                    f"(block means, then selection inside the attention launch)",
+                    f"(pooling, selection and attention in one launch per layer)",
         "B": w.B, "heads": w.heads, "grid": [w.H_tok, w.W_tok], "N": w.N, "head_dim": w.head_dim,
         "block": 8, "rho": w.rho, "Tb": Tb, "keep": keep,
         "realized_sparsity": round((Tb - keep) / Tb, 6), "layers": layers,
@@ -268,7 +268,7 @@ def run_ours(args, rank, world):
     pshp = (w.B, w.heads, Tb, w.head_dim)
     qbs = [torch.empty(pshp, dtype=torch.float32, device=dev) for _ in range(L)]
     kbs = [torch.empty(pshp, dtype=torch.float32, device=dev) for _ in range(L)]
-    # the timed path: block means, then selection + attention in one launch
+    # the timed path: pooling, selection and attention in one launch per layer (ssba_forward_fused)
     layers = [api.BoundSelectLayer(descs[l], Qs[l], Ks[l], Vs[l], qbs[l], kbs[l], idx[l], cnt[l], Os[l], lses[l],
                                    stream) for l in range(L)]
     # the two-launch path (mask kernel, then the forward on its lists), measured beside it
@@ -279,12 +279,9 @@ def run_ours(args, rank, world):
         for l, ly in enumerate(layers):
             if ev is not None:
                 ev[0][l].record(stream)
-            ly.pool()
+            ly.fused()
             if ev is not None:
                 ev[1][l].record(stream)
-            ly.attend()
-            if ev is not None:
-                ev[2][l].record(stream)
 
     for _ in range(max(3, args.warmup)):
         step()
@@ -296,7 +293,7 @@ def run_ours(args, rank, world):
 
     # ---- timed region: K steps, per-kernel events on the launching stream
     K = args.steps
-    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(L)] for _ in range(3)] for _ in range(K)]
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(L)] for _ in range(2)] for _ in range(K)]
     gpu_id = None
     try:
         gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
@@ -330,8 +327,7 @@ def run_ours(args, rank, world):
     for s in range(K):
         step(evs[s])
     torch.cuda.synchronize()
-    mask_ms = statistics.mean(evs[s][0][l].elapsed_time(evs[s][1][l]) for s in range(K) for l in range(L))
-    attn_ms = statistics.mean(evs[s][1][l].elapsed_time(evs[s][2][l]) for s in range(K) for l in range(L))
+    attn_ms = statistics.mean(evs[s][0][l].elapsed_time(evs[s][1][l]) for s in range(K) for l in range(L))
     st[0] = api.get_status()
     if int(st[0]) != api.SSBA_OK:
         raise RuntimeError(f"device status {int(st[0])} after the timed region")
@@ -339,22 +335,62 @@ def run_ours(args, rank, world):
     F_layer = kept_flops(w.B, w.heads, Tb, keep, w.head_dim)
     value = whole_job_tflops(world, L * F_layer, ms_step * 1e-3)
 
-    # ---- roofline of the dominant kernel (the attention kernel)
+    # ---- roofline of the dominant kernel (the only one: the fused launch)
     hbm_gbs, bf16_tflops, peak_src = measured_peaks()
     attn_tflops = F_layer / (attn_ms * 1e-3) / 1e12
-    attn_bytes = 4 * w.B * w.heads * w.N * w.head_dim * 2 + w.B * w.heads * w.N * 4
+    # Q, K, V read and O written once, lse written, the block means written
+    attn_bytes = (4 * w.B * w.heads * w.N * w.head_dim * 2 + w.B * w.heads * w.N * 4
+                  + 2 * w.B * w.heads * Tb * w.head_dim * 4)
     traffic = profiled_traffic()
-    roofline = {"kernel": "ssba_attn_tc_kernel", "bound": "tensor", "achieved": attn_tflops,
+    roofline = {"kernel": "ssba_attn_tc_kernel (ssba_forward_fused)", "bound": "tensor", "achieved": attn_tflops,
                 "peak": bf16_tflops, "unit": "TFLOP/s", "frac": attn_tflops / bf16_tflops,
                 "traffic": traffic, "algorithmic_bytes": attn_bytes,
                 "algorithmic_flops": F_layer, "avg_launch_ms": attn_ms,
                 "peak_source": f"{peak_src} dense bf16 (burst)",
                 "hbm_frac": attn_bytes / (attn_ms * 1e-3) / 1e9 / hbm_gbs}
+
+    # ---- the same layers with the pooling as a launch of its own (ssba_pool_blocks, then
+    #      ssba_forward_select), outside the timed region: its step time, and the pooling kernel's
+    #      duration (CUDA events around each launch) for its own roofline
     pool_bytes = 2 * w.B * w.heads * w.N * w.head_dim * 2 + 2 * w.B * w.heads * Tb * w.head_dim * 4
-    mask_roof = {"kernels": "ssba_pool_blocks_kernel (1 launch per layer)", "bound": "hbm",
-                 "achieved": pool_bytes / (mask_ms * 1e-3) / 1e9, "peak": hbm_gbs, "unit": "GB/s",
-                 "frac": pool_bytes / (mask_ms * 1e-3) / 1e9 / hbm_gbs, "algorithmic_bytes": pool_bytes,
-                 "avg_call_ms": mask_ms}
+    pool_select = None
+    mask_roof = None
+    mask_ms = None
+    try:
+        def step_ps():
+            for ly in layers:
+                ly.pool()
+                ly.attend()
+
+        for _ in range(3):
+            step_ps()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(5):
+            step_ps()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        tps = e0.elapsed_time(e1) / 5
+        evp = [[torch.cuda.Event(enable_timing=True) for _ in range(L)] for _ in range(3)]
+        for l, ly in enumerate(layers):
+            evp[0][l].record(stream)
+            ly.pool()
+            evp[1][l].record(stream)
+            ly.attend()
+            evp[2][l].record(stream)
+        torch.cuda.synchronize()
+        mask_ms = statistics.mean(evp[0][l].elapsed_time(evp[1][l]) for l in range(L))
+        sel_ms = statistics.mean(evp[1][l].elapsed_time(evp[2][l]) for l in range(L))
+        pool_select = {"ms_per_step": tps, "value": whole_job_tflops(1, L * F_layer, tps * 1e-3),
+                       "pool_ms_per_layer": mask_ms, "select_attention_ms_per_layer": sel_ms,
+                       "how": "ssba_pool_blocks + ssba_forward_select per layer, CUDA events around 5 steps; "
+                              "per-kernel durations from events around each launch of one step"}
+        mask_roof = {"kernels": "ssba_pool_blocks_kernel (pool + select path, 1 launch per layer)", "bound": "hbm",
+                     "achieved": pool_bytes / (mask_ms * 1e-3) / 1e9, "peak": hbm_gbs, "unit": "GB/s",
+                     "frac": pool_bytes / (mask_ms * 1e-3) / 1e9 / hbm_gbs, "algorithmic_bytes": pool_bytes,
+                     "avg_call_ms": mask_ms}
+    except Exception as exc:  # reported, not fatal
+        pool_select = f"failed: {exc}"
 
     # ---- the two-launch path on the same layers (mask kernel with its selection, then the forward
     #      on the lists), outside the timed region
@@ -521,8 +557,7 @@ def run_ours(args, rank, world):
 
         def lstep():
             for ly in llayers:
-                ly.pool()
-                ly.attend()
+                ly.fused()
 
         for _ in range(3):
             lstep()
@@ -531,8 +566,8 @@ def run_ours(args, rank, world):
         layer_aware = {"ms_per_step": tl, "effective_tflops": F_l / (tl * 1e-3) / 1e12,
                        "mean_sparsity": 1.0 - sum(lkeep) / (L * Tb), "keep_per_layer": lkeep,
                        "uniform_ms_per_step": ms_step,
-                       "how": "pool + selecting forward of the 24 layers with rho_l from schedule.layer_rhos, CUDA events "
-                              "around 5 steps"}
+                       "how": "the fused launch (ssba_forward_fused) of the 24 layers with rho_l from "
+                              "schedule.layer_rhos, CUDA events around 5 steps"}
     except Exception as exc:  # reported, not fatal
         layer_aware = f"failed: {exc}"
 
@@ -588,8 +623,7 @@ def run_ours(args, rank, world):
             for l, ly in enumerate(layers):
                 stream.wait_event(h2d_done[l])
                 stream.wait_event(d2h_done[l])  # previous step's read-back of O[l] finished
-                ly.pool()
-                ly.attend()
+                ly.fused()
                 comp_done[l].record(stream)
                 d2h_s.wait_event(comp_done[l])
                 with torch.cuda.stream(d2h_s):
@@ -612,8 +646,8 @@ def run_ours(args, rank, world):
         d2h = L * (w.B * w.heads * w.N * w.head_dim * 2 + w.B * w.heads * w.N * 4)
         e2e = {"value": whole_job_tflops(world, L * F_layer, e2e_s), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "steps": args.e2e_steps,
-               "how": "pinned host Q/K/V -> device on a copy stream, block means + selecting forward, O and lse -> "
-                      "pinned host on a second copy stream; host wall clock around the steps"}
+               "how": "pinned host Q/K/V -> device on a copy stream, the fused launch (ssba_forward_fused), O and "
+                      "lse -> pinned host on a second copy stream; host wall clock around the steps"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -659,8 +693,9 @@ def run_ours(args, rank, world):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": dict(config_dict(w, keep, L), parallelism="replicas" if world > 1 else "single GPU"),
             "latency_ms_per_layer": ms_step / L,
-            "attention_ms_per_layer": attn_ms, "pool_ms_per_layer": mask_ms,
+            "attention_ms_per_layer": attn_ms,
             "roofline": roofline, "roofline_pool": mask_roof,
+            "pool_select_path": pool_select,
             "two_launch_path": two_launch,
             "dense_attention_ms_per_layer": dense_ms,
             "text_joint": joint,
@@ -672,7 +707,7 @@ def run_ours(args, rank, world):
             "speedup_vs_dense": (dense_ms / attn_ms) if isinstance(dense_ms, float) else None,
             "ideal_speedup_vs_dense": Tb / keep,
             "e2e": e2e, "cpu_baseline": cpu,
-            "gpu_launches": K * L * 2,
+            "gpu_launches": K * L,
             "clocks": clocks.summary(wall0, wall1),
         }
         print(json.dumps(line), flush=True)

@@ -122,6 +122,8 @@ struct __align__(1024) SmemLayout {
 
 // Four maps per tensor, one per box shape, over the [B*heads][H][W][d] bf16 view, and
 // the text keys and values as [B*heads][T_txt][d] (64-row boxes, zero fill past T_txt).
+static_assert(sizeof(SmemLayout) + 1024 <= 232448, "shared memory of one CTA (227 KB opt-in limit)");
+
 struct TileMaps {
     CUtensorMap q[4], k[4], v[4];
     CUtensorMap kt, vt;
@@ -315,25 +317,33 @@ __device__ __noinline__ bool pool_phase(const TcParams& p, SmemLayout& cs, int g
 }
 
 // Grid-wide barrier for a persistent launch whose CTAs are all resident (one per SM, grid at
-// most the SM count; the next grid is released only after it). w[0] counts arrivals, w[1]
-// departures; the last CTA to depart sets both back to zero, so a call that completes leaves
-// the workspace zero-filled. Waits are bounded; returns false on timeout or abort (the words
-// are then left as they are, like the rest of the workspace after a timeout).
-__device__ bool grid_barrier(unsigned* w, unsigned n, volatile int* abortf, uint64_t budget_ns)
+// most the SM count; the next grid is released only after it). Called by one thread of each
+// CTA after a CTA barrier: a release add makes the CTA's writes (ordered before it by that
+// barrier) visible with its arrival, and an acquire load sees every other CTA's. w[0] counts
+// arrivals; the reset is left to grid_barrier_depart at the end of the kernel, off the
+// critical path. Bounded; returns false on timeout or abort.
+__device__ bool grid_barrier_arrive_wait(unsigned* w, unsigned n, volatile int* abortf, uint64_t budget_ns)
 {
-    __threadfence();
-    atomicAdd(&w[0], 1u);
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(w) : "memory");
     const uint64_t t0 = globaltimer_ns();
-    while (*reinterpret_cast<volatile unsigned*>(&w[0]) != n) {
+    for (;;) {
+        unsigned v;
+        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(w) : "memory");
+        if (v == n) return true;
         if (*abortf || globaltimer_ns() - t0 > budget_ns) return false;
-        __nanosleep(64);
     }
-    __threadfence();
-    if (atomicAdd(&w[1], 1u) == n - 1) {  // every CTA has seen w[0] == n
+}
+
+// After the whole CTA is done (every CTA of the grid has passed the barrier by then): w[1]
+// counts departures, and the last CTA to leave sets both words back to zero, so a call that
+// completes leaves the workspace zero-filled. (A CTA that gave up at the barrier does not
+// depart; the workspace is then zeroed again by the caller, as after any timeout.)
+__device__ void grid_barrier_depart(unsigned* w, unsigned n)
+{
+    if (atomicAdd(&w[1], 1u) == n - 1) {
         atomicExch(&w[0], 0u);
         atomicExch(&w[1], 0u);
     }
-    return true;
 }
 
 // A list entry: written earlier in this launch under in-kernel selection (read through L2),
@@ -345,8 +355,8 @@ __device__ __forceinline__ int ld_list(const TcParams& p, const int32_t* a) { re
 // fixed order; the total order of sel::rank_select, walked by sel::ballot_select on keys held
 // in registers), so the same means give the same lists. kbs: the head's k_b
 // staged in shared memory, the 16-byte chunk c4 of row j at chunk c4 ^ (j & 15) (two lanes per
-// bank at most when 32 lanes read one column); qs: the item's q_b row in shared memory; S: Tb
-// words of shared scratch. Not inlined, so that its registers do not weigh on the pipeline roles.
+// bank at most when 32 lanes read one column); qs: the item's q_b row in shared memory. Not
+// inlined, so that its registers do not weigh on the pipeline roles.
 template <int kPer>
 __device__ __noinline__ void select_item(const TcParams& p, int item, int lane, const float* kbs, const float* qs,
                                          uint32_t* S)
@@ -516,19 +526,11 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     SmemLayout& cs = *reinterpret_cast<SmemLayout*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                     ~static_cast<uintptr_t>(1023));
     const int gwarp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int slot = gwarp / kSlotWarps;   // which pipeline of this CTA
-    const int warp = gwarp % kSlotWarps;   // role within the pipeline
+    // the pipelines' variables are defined after the pooling below, so that they are not live
+    // across its call (at 80 registers a thread, values live across a call are spilled)
+    {
+    const int slot = gwarp / kSlotWarps;
     SlotSmem& sm = cs.slot[slot];
-    volatile int* abortf = &cs.abort_flag;
-    // pipeline `slot` of CTA b is pipeline b + slot * gridDim.x of 2 * gridDim.x: the items
-    // left over after whole rounds go to the first pipelines, one per CTA, and the other
-    // pipeline of such a CTA finishes first and leaves it the SM
-    const int vcta = slot * gridDim.x + blockIdx.x;
-    const int vgrid = gridDim.x * kSlots;
-    const Grid g = p.g;
-    const int Tb = g.Tb();
-    const int N = g.H * g.W;
-
     if (threadIdx.x % (kSlotWarps * 32) == 0) {
         if (slot == 0) cs.abort_flag = 0;
         for (int s = 0; s < kKStages; ++s) {
@@ -561,28 +563,45 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             for (int w = slot * kSlotWarps; w < (slot + 1) * kSlotWarps; ++w) mbar_init(smem_u32(&cs.pool_bar[w]), 1);
         fence_mbar_init();
     }
-    for (int l = threadIdx.x; l < Tb && l < kWinCap; l += kThreads) cs.win[l] = window_entry(g, l);
+    const Grid g = p.g;
+    for (int l = threadIdx.x; l < g.Tb() && l < kWinCap; l += kThreads) cs.win[l] = window_entry(g, l);
+    }
     // everything above reads no input; the lists, counts and tensors may come from the grid
     // launched just before this one (programmatic dependent launch)
     grid_dep_wait();
+    bool pool_fail = false;
     if (p.pool_q) {
-        bool pool_fail = false;
         // the block means of the whole layer: every warp of the grid one (block, tensor) unit,
         // then a grid barrier; the next grid is released only after it, so that it cannot take
         // an SM that one of these CTAs still waits for
         __syncthreads();  // the pooling barriers are initialised
-        pool_fail = !pool_phase(p, cs, gwarp, lane, abortf);
-        __threadfence();  // this CTA's means, visible to the whole GPU before it arrives
+        pool_fail = !pool_phase(p, cs, gwarp, lane, &cs.abort_flag);
+        pool_fail = __syncthreads_or(pool_fail);  // also orders this CTA's means before the arrival
+        if (threadIdx.x == 0 && !pool_fail)
+            pool_fail = !grid_barrier_arrive_wait(p.gsync, gridDim.x, &cs.abort_flag, p.budget_ns);
+        // on a timeout the means of other CTAs may be missing: the status is set, and the raised
+        // abort flag makes every role leave at its first wait that does not complete at once
+        // (lists selected from stale means still hold labels in [0, Tb)). No early return and
+        // no condition on the selection: either costs the pipeline roles registers (spills).
         pool_fail = __syncthreads_or(pool_fail);
-        if (threadIdx.x == 0 && !pool_fail) pool_fail = !grid_barrier(p.gsync, gridDim.x, abortf, p.budget_ns);
-        if (__syncthreads_or(pool_fail)) {
-            // nothing allocated or in flight yet: report and leave (the means of the other CTAs
-            // may be missing, so no list of this CTA can be trusted)
-            if (threadIdx.x == 0) atomicExch(p.status, SSBA_ERR_TIMEOUT);
-            return;
+        if (pool_fail && threadIdx.x == 0) {
+            atomicExch(p.status, SSBA_ERR_TIMEOUT);
+            cs.abort_flag = 1;
         }
     }
     grid_dep_launch();
+    const int slot = gwarp / kSlotWarps;   // which pipeline of this CTA
+    const int warp = gwarp % kSlotWarps;   // role within the pipeline
+    SlotSmem& sm = cs.slot[slot];
+    volatile int* abortf = &cs.abort_flag;
+    // pipeline `slot` of CTA b is pipeline b + slot * gridDim.x of 2 * gridDim.x: the items
+    // left over after whole rounds go to the first pipelines, one per CTA, and the other
+    // pipeline of such a CTA finishes first and leaves it the SM
+    const int vcta = slot * gridDim.x + blockIdx.x;
+    const int vgrid = gridDim.x * kSlots;
+    const Grid g = p.g;
+    const int Tb = g.Tb();
+    const int N = g.H * g.W;
     if (p.sel_qb) {
         // the lists of this CTA's items (the contiguous ranges of its two pipelines): the k_b
         // of the heads they touch are staged by all threads in the stage buffers of both
@@ -1098,6 +1117,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     __syncthreads();
     tc_fence_after();
     if (gwarp == 1) tmem_dealloc(cs.tmem_base, kTmemCols);
+    if (p.pool_q && threadIdx.x == 0 && !cs.abort_flag) grid_barrier_depart(p.gsync, gridDim.x);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
