@@ -571,6 +571,88 @@ def run_ours(args, rank, world):
     except Exception as exc:  # reported, not fatal
         layer_aware = f"failed: {exc}"
 
+    # ---- the other workloads of the paper's range, outside the timed region: the 512 px model
+    #      (24 layers), the elastic sweep at 1024 px (32x32 and 64x64 grids x sparsity x batch)
+    #      and the 2048 px stress (24 layers, 84 % and 90 %). Per config: the time per layer on
+    #      its path (the fused launch for Tb <= 128, else ssba_build_mask + ssba_forward), the
+    #      effective TFLOP/s over kept blocks and its fraction of the measured peak, and the
+    #      same-build dense kernel. Inputs: N(0,1) (512 px: x 1/8) drawn on the device from a
+    #      seeded generator, alternating shifts, and enough distinct layers that one pass over
+    #      them is larger than L2 (cold inputs per layer, as in the timed step)
+    sweep = None
+    try:
+        def run_config(Bc, Hc, Wc, rho, std, layers):
+            Tbc = Hc * Wc // 64
+            dsc = [api.SsbaDesc(Bc, w.heads, Hc, Wc, w.head_dim, 8, *layer_shift(l), rho, w.dtype)
+                   for l in range(layers)]
+            kc = api.keep_count(dsc[0])
+            shp_c = (Bc, w.heads, Hc * Wc, w.head_dim)
+            gen = torch.Generator(device=dev)
+            gen.manual_seed(4000 + 1000 * rank)
+            ins = [[(torch.randn(shp_c, generator=gen, device=dev) * std).to(w.dtype) for _ in range(3)]
+                   for _ in range(layers)]
+            Oc = torch.empty(shp_c, dtype=w.dtype, device=dev)
+            lc = torch.empty(shp_c[:3], dtype=torch.float32, device=dev)
+            ic = torch.empty((Bc, w.heads, Tbc, kc), dtype=torch.int32, device=dev)
+            cc = torch.empty((Bc, w.heads, Tbc), dtype=torch.int32, device=dev)
+            if Tbc <= 128:
+                pq = torch.empty((Bc, w.heads, Tbc, w.head_dim), dtype=torch.float32, device=dev)
+                pk = torch.empty_like(pq)
+                lys = [api.BoundSelectLayer(dsc[l], *ins[l], pq, pk, ic, cc, Oc, lc, stream) for l in range(layers)]
+
+                def fn():
+                    for ly in lys:
+                        ly.fused()
+                path = "ssba_forward_fused"
+            else:
+                wsc = torch.empty(api.mask_workspace_bytes(dsc[0]), dtype=torch.uint8, device=dev)
+                lys = [api.BoundLayer(dsc[l], *ins[l], ic, cc, Oc, lc, wsc, stream) for l in range(layers)]
+
+                def fn():
+                    for ly in lys:
+                        ly.mask()
+                        ly.attend()
+                path = "ssba_build_mask + ssba_forward"
+            for _ in range(3):
+                fn()
+            t_layer = events_ms(fn, 5) / layers
+            nd = min(layers, 8)
+
+            def fd():
+                for l in range(nd):
+                    api.forward_dense(dsc[l], *ins[l], Oc, lc)
+            fd()
+            t_dense = events_ms(fd, 3) / nd
+            Fc = kept_flops(Bc, w.heads, Tbc, kc, w.head_dim)
+            tf = Fc / (t_layer * 1e-3) / 1e12
+            del ins, lys
+            return {"grid": [Hc, Wc], "B": Bc, "rho": rho, "keep": kc, "Tb": Tbc,
+                    "realized_sparsity": round((Tbc - kc) / Tbc, 6), "layers": layers, "path": path,
+                    "ms_per_layer": t_layer, "effective_tflops": tf, "frac": tf / bf16_tflops,
+                    "dense_ms_per_layer": t_dense, "speedup_vs_dense": t_dense / t_layer,
+                    "ideal_speedup_vs_dense": Tbc / kc}
+
+        def n_layers(Bc, Hc, Wc):
+            per = 3 * Bc * w.heads * Hc * Wc * w.head_dim * 2
+            return min(24, max(1, math.ceil(2 * 129e6 / per)))
+
+        cases = {"512px_24_layers": run_config(1, 32, 32, 0.8416, 0.125, 24)}
+        for (Hc, Wc) in ((32, 32), (64, 64)):
+            for Bc in (1, 4):
+                for rho in (0.0, 0.5, 0.75, 0.8416, 0.9):
+                    cases[f"sweep_{Hc}x{Wc}_B{Bc}_rho{rho}"] = run_config(Bc, Hc, Wc, rho, 1.0, n_layers(Bc, Hc, Wc))
+        for rho in (0.84, 0.9):
+            cases[f"2048px_24_layers_rho{rho}"] = run_config(1, 128, 128, rho, 1.0, 24)
+        # the headline layer back to back on resident inputs (warm L2) against the timed step (cold)
+        warm = events_ms(lambda: layers[1].fused(), 20)
+        cases["1024px_warm_l2"] = {"ms_per_layer": warm, "effective_tflops": F_layer / (warm * 1e-3) / 1e12,
+                                   "how": "one shifted 1024 px layer's fused launch 20 times back to back"}
+        sweep = dict(cases, peak_tflops=bf16_tflops, peak_source=peak_src,
+                     how="CUDA events around 5 passes over the config's layers after 3 warm-up passes; "
+                         "dense: ssba_forward_dense on up to 8 of the layers")
+    except Exception as exc:  # reported, not fatal
+        sweep = f"failed: {exc}"
+
     # ---- the steps before the mask fused into the projection (ssba_qkv_rope_pool): X W^T + b, RoPE,
     #      block means; 1024 px, Dm = 1536; X and Wqkv (27 MB) stay in L2 between launches
     qkv = None
@@ -658,6 +740,16 @@ def run_ours(args, rank, world):
         cpu = {"value": rate, "unit": "TFLOP/s", "cores": min(threads, heads_sample), "kind": "oracle",
                "sample": f"{heads_sample} of {w.heads} heads of one layer (mask + forward), {dt:.2f} s, "
                          f"fp64 C with OpenMP over heads"}
+        try:  # one thread at the 512 px config
+            from paper_2605_15684_gb300 import synthetic as _syn
+            oracle.set_threads(1)
+            rate1, dt1 = oracle_sample(_syn.PX512, 8)
+            cpu["single_thread_512px"] = {"value": rate1, "unit": "TFLOP/s", "cores": 1, "seconds": dt1,
+                                          "sample": "8 of 24 heads of one 512 px layer (mask + forward)"}
+        except Exception as exc:  # reported, not fatal
+            cpu["single_thread_512px"] = f"failed: {exc}"
+        finally:
+            oracle.set_threads(threads)
 
     # ---- the mask when the projection has pooled: selection alone (ssba_select_mask) against the
     #      full build (ssba_build_mask re-reads Q and K); 20 launches captured in a CUDA graph,
@@ -702,6 +794,7 @@ def run_ours(args, rank, world):
             "backward": bwd,
             "haar": haar,
             "layer_aware": layer_aware,
+            "configs_sweep": sweep,
             "qkv_fused": qkv,
             "mask_after_fused_pooling": mask_split,
             "speedup_vs_dense": (dense_ms / attn_ms) if isinstance(dense_ms, float) else None,
