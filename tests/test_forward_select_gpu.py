@@ -127,3 +127,5 @@ def test_forward_select_rejects_long_rows():
     qb, kb = api.pool_blocks(desc, q, k)
     with pytest.raises(api.SsbaError, match="Tb <= 128"):
         api.forward_select(desc, q, k, v, qb, kb)
+    with pytest.raises(api.SsbaError, match="Tb <= 128"):
+        api.forward_fused(desc, q, k, v)
