@@ -253,4 +253,8 @@ def test_python_binding_validates_before_calling(lib):
     q = torch.zeros(1, 2, 256, 64, dtype=torch.bfloat16)
     with pytest.raises(api.SsbaError, match="CUDA tensor"):
         api.build_mask(dsc, q, q)
+    with pytest.raises(api.SsbaError, match="CUDA tensor"):
+        api.forward_fused(dsc, q, q, q)
+    with pytest.raises(api.SsbaError, match="workspace"):
+        api.forward_fused(dsc, q, q, q, workspace=None)
     assert api.realized_sparsity(api.SsbaDesc(1, 24, 64, 64, rho=0.8416)) == 53 / 64
