@@ -151,8 +151,9 @@ SSBA_API int ssba_forward_joint(const ssba_desc* desc, const void* Q, const void
                                 const int32_t* kv_idx, const int32_t* kv_cnt, void* O, float* lse,
                                 void* workspace, size_t ws_bytes, void* stream);
 
-/* Bytes of the optional ssba_forward / ssba_forward_dense workspace for desc on the
- * current device (it scales with the device's SM count: about 10 MB on 152 SMs);
+/* Bytes of the optional ssba_forward / ssba_forward_dense / ssba_forward_select workspace, and
+ * of the required one of ssba_forward_fused, for desc on the current device (it scales with the
+ * device's SM count: about 10 MB on 152 SMs);
  * 0 for an fp32 or an invalid descriptor. Host only, no device work. */
 SSBA_API size_t ssba_forward_workspace_bytes(const ssba_desc* desc);
 
