@@ -324,6 +324,18 @@ SSBA_API int ssba_test_forward_timeout(const ssba_desc* desc, const void* Q, con
                                        const int32_t* kv_idx, const int32_t* kv_cnt, void* O, float* lse,
                                        uint64_t budget_ns, void* stream);
 
+/* Test hook for failure detection in the fused launch (no counterpart in the paper): runs
+ * ssba_forward_fused with every wait limited to budget_ns of wall time (clamped to [1 ms, 2 s])
+ * and CTA 0 withholding its arrival at the grid barrier, so that every CTA's barrier wait runs
+ * out. Each CTA then reports SSBA_ERR_TIMEOUT in the device status word, raises its abort flag
+ * and leaves at its first wait that does not complete at once (the means are complete, so its
+ * lists are valid); O, lse and the lists are undefined, the workspace's barrier words are left
+ * set (zero it again, as after any timeout), and the context stays usable. No fault, trap or
+ * endless wait is involved. Arguments as ssba_forward_fused (workspace required); bf16 only. */
+SSBA_API int ssba_test_fused_timeout(const ssba_desc* desc, const void* Q, const void* K, const void* V, float* qb,
+                                     float* kb, int32_t* kv_idx, int32_t* kv_cnt, void* O, float* lse,
+                                     void* workspace, size_t ws_bytes, uint64_t budget_ns, void* stream);
+
 /* Reads and clears the device status word of the current device (SSBA_OK or
  * SSBA_ERR_TIMEOUT). Synchronous: call after the caller's stream sync. Returns
  * SSBA_OK, or SSBA_ERR_CUDA if the read failed. */

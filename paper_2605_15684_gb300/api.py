@@ -28,7 +28,7 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
 
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
-            "ssba_test_forward_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
+            "ssba_test_forward_timeout", "ssba_test_fused_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
             "ssba_haar_iwt", "ssba_haar_dwt_pyramid", "ssba_haar_iwt_pyramid", "ssba_qkv_rope_pool",
             "ssba_select_mask", "ssba_pool_blocks", "ssba_forward_select", "ssba_forward_fused",
             "ssba_get_status", "ssba_last_error")
@@ -124,6 +124,8 @@ def load_library():
         lib.ssba_forward_dense.restype = ctypes.c_int
         lib.ssba_test_forward_timeout.argtypes = [DP, P, P, P, P, P, P, P, ctypes.c_uint64, P]
         lib.ssba_test_forward_timeout.restype = ctypes.c_int
+        lib.ssba_test_fused_timeout.argtypes = [DP, P, P, P, P, P, P, P, P, P, P, ctypes.c_size_t, ctypes.c_uint64, P]
+        lib.ssba_test_fused_timeout.restype = ctypes.c_int
         lib.ssba_backward.argtypes = [DP, P, P, P, P, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_backward.restype = ctypes.c_int
         lib.ssba_backward_workspace_bytes.argtypes = [DP]
@@ -521,6 +523,29 @@ def test_forward_timeout(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O, lse, budget
     _raise_on(lib.ssba_test_forward_timeout(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(),
                                             kv_idx.data_ptr(), kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(),
                                             int(budget_ns), _stream_ptr(stream)))
+
+
+def test_fused_timeout(desc: SsbaDesc, Q, K, V, qb, kb, kv_idx, kv_cnt, O, lse, workspace,
+                       budget_ns: int = 2_000_000, stream=None) -> None:
+    """ssba_test_fused_timeout: the fused launch's failure-detection test hook (include/ssba.h)."""
+    lib = load_library()
+    d = desc.c()
+    keep = keep_count(desc)
+    shp = (desc.B, desc.heads, desc.N, desc.head_dim)
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V"), (O, "O")):
+        _check(t, n, shp, desc.dtype)
+    pshp = (desc.B, desc.heads, desc.Tb, desc.head_dim)
+    _check(qb, "qb", pshp, torch.float32)
+    _check(kb, "kb", pshp, torch.float32)
+    _check(kv_idx, "kv_idx", (desc.B, desc.heads, desc.Tb, keep), torch.int32)
+    _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
+    _check(lse, "lse", shp[:3], torch.float32)
+    wp, wn = _ws_args(workspace)
+    if wp is None:
+        raise SsbaError(SSBA_ERR_WORKSPACE, "test_fused_timeout needs a forward workspace")
+    _raise_on(lib.ssba_test_fused_timeout(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), qb.data_ptr(),
+                                          kb.data_ptr(), kv_idx.data_ptr(), kv_cnt.data_ptr(), O.data_ptr(),
+                                          lse.data_ptr(), wp, wn, int(budget_ns), _stream_ptr(stream)))
 
 
 def backward_workspace_bytes(desc: SsbaDesc) -> int:

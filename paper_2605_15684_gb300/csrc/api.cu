@@ -388,6 +388,33 @@ int ssba_test_forward_timeout(const ssba_desc* desc, const void* Q, const void* 
                                static_cast<cudaStream_t>(stream), b, 1);
 }
 
+int ssba_test_fused_timeout(const ssba_desc* desc, const void* Q, const void* K, const void* V, float* qb, float* kb,
+                            int32_t* kv_idx, int32_t* kv_cnt, void* O, float* lse, void* workspace, size_t ws_bytes,
+                            uint64_t budget_ns, void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_test_fused_timeout", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !V || !qb || !kb || !kv_idx || !kv_cnt || !O || !lse || !workspace) {
+        set_error("ssba_test_fused_timeout: every pointer must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(qb, 16) ||
+        !aligned(kb, 16) || !aligned(lse, 4) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) || !aligned(workspace, 16)) {
+        set_error("ssba_test_fused_timeout: Q, K, V, O, qb, kb, workspace 16-byte aligned; the rest 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    if (desc->dtype != SSBA_BF16) {
+        set_error("ssba_test_fused_timeout: bf16 only");
+        return SSBA_ERR_UNSUPPORTED;
+    }
+    const uint64_t b = budget_ns < 1000000ull ? 1000000ull : (budget_ns > kWaitBudgetNs ? kWaitBudgetNs : budget_ns);
+    return launch_attn_tc_bf16(*desc, g, keep, resolve_scale(desc), Q, K, V, kv_idx, kv_cnt, O, lse, workspace,
+                               ws_bytes, static_cast<cudaStream_t>(stream), b, 2, nullptr, nullptr, 0, qb, kb, nullptr,
+                               true);
+}
+
 size_t ssba_backward_workspace_bytes(const ssba_desc* desc)
 {
     Grid g;

@@ -157,8 +157,9 @@ struct TcParams {
     const __nv_bfloat16* pool_k;
     unsigned* gsync;  // grid barrier words in the workspace (arrivals, departures)
     uint64_t budget_ns;  // wall-time limit of every barrier wait
-    int withhold;        // test hook: pipeline 0 announces its first K copy but never issues it,
-                         // so that the waits on it run out (failure-detection test only)
+    int withhold;        // failure-detection test hooks: 1, pipeline 0 announces its first K copy
+                         // but never issues it, so that the waits on it run out; 2, CTA 0 does not
+                         // arrive at the grid barrier of the fused launch (0 otherwise)
 };
 
 // Work schedule, for V pipelines (two per CTA).
@@ -322,9 +323,10 @@ __device__ __noinline__ bool pool_phase(const TcParams& p, SmemLayout& cs, int g
 // barrier) visible with its arrival, and an acquire load sees every other CTA's. w[0] counts
 // arrivals; the reset is left to grid_barrier_depart at the end of the kernel, off the
 // critical path. Bounded; returns false on timeout or abort.
-__device__ bool grid_barrier_arrive_wait(unsigned* w, unsigned n, volatile int* abortf, uint64_t budget_ns)
+__device__ bool grid_barrier_arrive_wait(unsigned* w, unsigned n, volatile int* abortf, uint64_t budget_ns,
+                                         bool arrive)
 {
-    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(w) : "memory");
+    if (arrive) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(w) : "memory");
     const uint64_t t0 = globaltimer_ns();
     for (;;) {
         unsigned v;
@@ -578,7 +580,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         pool_fail = !pool_phase(p, cs, gwarp, lane, &cs.abort_flag);
         pool_fail = __syncthreads_or(pool_fail);  // also orders this CTA's means before the arrival
         if (threadIdx.x == 0 && !pool_fail)
-            pool_fail = !grid_barrier_arrive_wait(p.gsync, gridDim.x, &cs.abort_flag, p.budget_ns);
+            pool_fail = !grid_barrier_arrive_wait(p.gsync, gridDim.x, &cs.abort_flag, p.budget_ns,
+                                                  p.withhold != 2 || blockIdx.x != 0);
         // on a timeout the means of other CTAs may be missing: the status is set, and the raised
         // abort flag makes every role leave at its first wait that does not complete at once
         // (lists selected from stale means still hold labels in [0, Tb)). No early return and
@@ -743,7 +746,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                                 smem_u32(full), 0, tt * 64, bh);
                 }
                 // image blocks of the piece: list entries [ti0 - ntxt, ti0 - ntxt + nimg)
-                const bool hold = p.withhold && is_k && vcta == 0;  // test hook: never lands
+                const bool hold = p.withhold == 1 && is_k && vcta == 0;  // test hook: never lands
                 const uint32_t empty0 = smem_u32(is_k ? &sm.k_empty[0] : &sm.v_empty[0]);
                 const uint32_t full0 = smem_u32(is_k ? &sm.k_full[0] : &sm.v_full[0]);
                 const uint32_t tile0 = smem_u32(is_k ? &sm.k[0][0] : &sm.v[0][0]);

@@ -2,7 +2,9 @@
 forward is bounded in wall time. A test hook announces one K tile copy that it never
 issues, so the waits on that tile run out; the kernel must stop, drain what it issued,
 free its tensor memory and report SSBA_ERR_TIMEOUT in the device status word, and the
-CUDA context must stay usable (a normal forward right after matches the oracle)."""
+CUDA context must stay usable (a normal forward right after matches the oracle). A second
+hook makes one CTA of the fused launch withhold its arrival at the grid barrier, so that
+every CTA's barrier wait runs out, with the same requirements."""
 import pytest
 import torch
 
@@ -37,3 +39,37 @@ def test_timed_out_wait_reports_status_and_context_survives():
     O_o, lse_o = oracle.forward(q, k, v, idx_o, H, W, 8, (4, 4))
     check_out(O2.float().cpu().numpy(), lse2.cpu().numpy(), O_o, lse_o, "bf16")
     assert api.get_status() == api.SSBA_OK
+
+
+def test_grid_barrier_timeout_reports_status_and_context_survives():
+    build.build()
+    api.load_library()
+    H = W = 64
+    q, k, v = synthetic.qkv(1, 24, H * W, 64, torch.bfloat16, 12)
+    qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
+    desc = api.SsbaDesc(1, 24, H, W, shift_r=4, shift_c=4, rho=0.8416)
+    keep = api.keep_count(desc)
+    Tb = H * W // 64
+    qb = torch.empty(1, 24, Tb, 64, device="cuda")
+    kb = torch.empty_like(qb)
+    idx = torch.empty(1, 24, Tb, keep, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(1, 24, Tb, dtype=torch.int32, device="cuda")
+    O = torch.empty_like(qd)
+    lse = torch.empty(1, 24, H * W, device="cuda")
+    ws = torch.zeros(api.forward_workspace_bytes(desc), dtype=torch.uint8, device="cuda")
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK  # read-and-clear: start clean
+
+    api.test_fused_timeout(desc, qd, kd, vd, qb, kb, idx, cnt, O, lse, ws, budget_ns=2_000_000)
+    torch.cuda.synchronize()  # every CTA gives up at the barrier and returns: no hang, no CUDA error
+    assert api.get_status() == api.SSBA_ERR_TIMEOUT
+    assert api.get_status() == api.SSBA_OK
+
+    ws.zero_()  # the barrier words are left set after a timeout
+    O2, l2, i2, c2, qb2, kb2 = api.forward_fused(desc, qd, kd, vd, workspace=ws)
+    qb3, kb3 = api.pool_blocks(desc, qd, kd)
+    O3, l3, i3, c3 = api.forward_select(desc, qd, kd, vd, qb3, kb3)
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
+    assert torch.equal(i2, i3) and torch.equal(O2, O3) and torch.equal(l2, l3)
+    assert int(ws[-256:].count_nonzero()) == 0
