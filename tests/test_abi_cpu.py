@@ -234,6 +234,11 @@ def test_pool_and_select_forward_validation(lib):
     assert ff(desc(dtype=api.SSBA_FP32), good) == api.SSBA_ERR_UNSUPPORTED
     assert ff(desc(H_tok=96, W_tok=96), good) == api.SSBA_ERR_UNSUPPORTED
     assert b"Tb <= 128" in lib.ssba_last_error()
+    # its failure-detection hook: the same checks before any launch (workspace required)
+    ft = lambda dd, v: lib.ssba_test_fused_timeout(ctypes.byref(dd), *v[:3], *v[3:5], *v[5:7], *v[8:11], 0,
+                                                   2_000_000, None)
+    assert ft(d, [FAKE] * 7 + [None] + [FAKE] * 2 + [None]) == api.SSBA_ERR_INVALID  # no workspace
+    assert ft(desc(dtype=api.SSBA_FP32), good) == api.SSBA_ERR_UNSUPPORTED
 
 
 def ct_byref(d):
