@@ -46,3 +46,34 @@ def test_noalloc_matches_workspace_entry_point_on_consecutive_calls():
         assert torch.equal(cnt, ref_cnt)
         assert torch.equal(S, ref_S)
     assert api.get_status() == api.SSBA_OK
+
+
+@pytest.mark.gpu
+def test_noalloc_scratch_area_on_consecutive_calls():
+    """Layers that the one-launch mask kernel does not take (head_dim other than 64, or more
+    than 256 blocks per row) pool into the scratch area and select from it, so these calls
+    read and write the built-in area. They run back to back on different shapes, the first
+    one filling almost all of the 4 MiB, so every later call finds the previous call's
+    means there; each must still equal ssba_build_mask with a workspace of its own."""
+    build.build()
+    lib = api.load_library()
+    cases = [
+        # 136 x 136 grid: Tb = 289 > 256; 28 heads fill 4.14 of the 4.19 MB
+        (api.SsbaDesc(1, 28, 136, 136, shift_r=4, shift_c=4, rho=0.84), 21),
+        (api.SsbaDesc(1, 8, 64, 64, head_dim=128, shift_r=4, shift_c=4, rho=0.8416), 22),
+        (api.SsbaDesc(1, 3, 136, 136, rho=0.9), 23),
+        (api.SsbaDesc(2, 5, 24, 40, head_dim=32, shift_r=3, shift_c=-5, rho=0.6, dtype=torch.float32), 24),
+        (api.SsbaDesc(1, 8, 64, 64, head_dim=128, shift_r=4, shift_c=4, rho=0.8416), 25),
+    ]
+    need0 = lib.ssba_mask_workspace_bytes(ctypes.byref(cases[0][0].c()))
+    assert (4 << 20) - (64 << 10) < need0 <= (4 << 20)
+    for desc, seed in cases:
+        q, k, _ = synthetic.qkv(desc.B, desc.heads, desc.N, desc.head_dim, desc.dtype, seed=seed)
+        q, k = q.cuda(), k.cuda()
+        idx, cnt, S = api.build_mask_noalloc(desc, q, k, scores=True)
+        ref_idx, ref_cnt, ref_S = api.build_mask(desc, q, k, scores=True)
+        torch.cuda.synchronize()
+        assert torch.equal(idx, ref_idx)
+        assert torch.equal(cnt, ref_cnt)
+        assert torch.equal(S, ref_S)
+    assert api.get_status() == api.SSBA_OK
