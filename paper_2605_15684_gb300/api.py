@@ -9,7 +9,6 @@ library must exist (``paper_2605_15684_gb300.build.build()`` makes it).
 from __future__ import annotations
 
 import ctypes
-import math
 import os
 import threading
 from dataclasses import dataclass
@@ -21,17 +20,18 @@ _LIB_PATH = os.path.join(_HERE, "libssba.so")
 _lock = threading.Lock()
 _lib = None
 
-SSBA_OK, SSBA_ERR_INVALID, SSBA_ERR_UNSUPPORTED, SSBA_ERR_CUDA, SSBA_ERR_TIMEOUT, SSBA_ERR_WORKSPACE = range(6)
+(SSBA_OK, SSBA_ERR_INVALID, SSBA_ERR_UNSUPPORTED, SSBA_ERR_CUDA, SSBA_ERR_TIMEOUT, SSBA_ERR_WORKSPACE,
+ SSBA_ERR_CHECK) = range(7)
 SSBA_BF16, SSBA_FP32 = 0, 1
 _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED", 3: "SSBA_ERR_CUDA",
-                 4: "SSBA_ERR_TIMEOUT", 5: "SSBA_ERR_WORKSPACE"}
+                 4: "SSBA_ERR_TIMEOUT", 5: "SSBA_ERR_WORKSPACE", 6: "SSBA_ERR_CHECK"}
 
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
             "ssba_test_forward_timeout", "ssba_test_fused_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
             "ssba_haar_iwt", "ssba_haar_dwt_pyramid", "ssba_haar_iwt_pyramid", "ssba_qkv_rope_pool",
             "ssba_select_mask", "ssba_pool_blocks", "ssba_forward_select", "ssba_forward_fused",
-            "ssba_get_status", "ssba_last_error")
+            "ssba_get_status", "ssba_last_error", "ssba_timeline_read")
 
 
 class SsbaError(RuntimeError):
@@ -85,12 +85,18 @@ def library_path() -> str:
     return _LIB_PATH
 
 
-def load_library():
-    """Load libssba.so (raises if it has not been built)."""
-    global _lib
+def load_library(path: str | None = None):
+    """Load libssba.so (raises if it has not been built). ``path`` selects another build of
+    the same library (the timeline or checked variant of build.py) on the first call; every
+    later call returns the library loaded first."""
+    global _lib, _LIB_PATH
     with _lock:
         if _lib is not None:
+            if path is not None and os.path.abspath(path) != _LIB_PATH:
+                raise SsbaError(SSBA_ERR_INVALID, f"{_LIB_PATH} is already loaded in this process")
             return _lib
+        if path is not None:
+            _LIB_PATH = os.path.abspath(path)
         if not os.path.exists(_LIB_PATH):
             raise SsbaError(SSBA_ERR_CUDA, f"{_LIB_PATH} is missing: run paper_2605_15684_gb300.build.build()")
         lib = ctypes.CDLL(_LIB_PATH)
@@ -143,6 +149,8 @@ def load_library():
         lib.ssba_get_status.restype = ctypes.c_int
         lib.ssba_last_error.argtypes = []
         lib.ssba_last_error.restype = ctypes.c_char_p
+        lib.ssba_timeline_read.argtypes = [P, P, P]
+        lib.ssba_timeline_read.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -676,8 +684,9 @@ def get_status() -> int:
 
 
 def realized_sparsity(desc: SsbaDesc) -> float:
-    """k_drop / Tb with k_drop = floor(Tb * rho) (host arithmetic, no device call)."""
-    return math.floor(desc.Tb * desc.rho) / desc.Tb
+    """Dropped share of the key blocks, (Tb - keep) / Tb, with keep from ssba_keep_count
+    (the library's sparsity rule; no device call)."""
+    return (desc.Tb - keep_count(desc)) / desc.Tb
 
 
 class BoundSelectLayer:
