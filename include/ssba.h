@@ -48,7 +48,10 @@ typedef enum {
     SSBA_ERR_UNSUPPORTED = 2, /* valid for the method but outside the kernels' fast path   */
     SSBA_ERR_CUDA = 3,        /* a CUDA runtime/driver call or launch failed               */
     SSBA_ERR_TIMEOUT = 4,     /* (device status) a bounded wait inside a kernel ran out    */
-    SSBA_ERR_WORKSPACE = 5    /* workspace missing or smaller than ssba_mask_workspace_bytes */
+    SSBA_ERR_WORKSPACE = 5,   /* workspace missing or smaller than ssba_mask_workspace_bytes */
+    SSBA_ERR_CHECK = 6        /* (device status, checked build only) an index list broke its
+                                 invariants: a label outside [0, Tb), not ascending, or a
+                                 count other than keep                                      */
 } ssba_status;
 
 typedef enum { SSBA_BF16 = 0, SSBA_FP32 = 1 } ssba_dtype;
@@ -343,6 +346,25 @@ SSBA_API int ssba_get_status(int32_t* device_status_out);
 
 /* Message of the calling thread's last failed call ("" if none). */
 SSBA_API const char* ssba_last_error(void);
+
+/* Diagnostics (the paper has no counterpart): the time stamps that the attention kernel
+ * (ssba_forward, ssba_forward_select, ssba_forward_fused, ...) recorded in its last launch on
+ * the current device, in a library built with -DSSBA_TIMELINE (build.py variant "timeline").
+ *   cta   host array of 256 x 16 uint64: per CTA, globaltimer nanoseconds of the launch's
+ *         phases in this order: entry, dependency wait over, first pooled rows landed, means
+ *         stored, grid barrier passed, head means staged, lists selected, pipelines start,
+ *         pipeline 0 done, pipeline 1 done, exit (0 where a phase did not run);
+ *   tile  host array of 8 x 128 x 12 uint32: for pipelines 0 and 1 of CTAs 0, 1, grid/2 and
+ *         grid-1, per tile (the pipeline's running key-block count), SM clock stamps of: K copy
+ *         issued, QK issued, softmax saw S, softmax exps done, P stored, PV issued, V copy
+ *         issued, QK's wait for a free S buffer over, S in the softmax's registers, row maxima
+ *         known, P buffer free, PV's waits over;
+ *   item  host array of 8 x 32 x 4 uint32: per item of those pipelines, SM clock stamps of: the
+ *         epilogue starts waiting for O, O ready, the epilogue done, and (item 0 only) the
+ *         pipeline's start.
+ * Synchronous (call after the caller's stream sync). The default build records nothing and
+ * returns SSBA_ERR_UNSUPPORTED; SSBA_ERR_CUDA if a copy fails. */
+SSBA_API int ssba_timeline_read(uint64_t* cta, uint32_t* tile, uint32_t* item);
 
 #ifdef __cplusplus
 }

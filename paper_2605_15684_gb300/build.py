@@ -3,6 +3,14 @@
 Each .cu file under csrc/ is compiled by nvcc in parallel and linked into one shared
 object with the CUDA runtime linked statically, so the library loads on a machine
 without a GPU driver (the driver is only needed once a call reaches the device).
+
+Variants (built only on request, each in a folder and a library of its own, so that the
+default libssba.so is never affected):
+  timeline  -DSSBA_TIMELINE: the attention kernel records time stamps of its phases and of
+            every tile of a few sampled pipelines (read by ssba_timeline_read; see timeline.py);
+  checked   -DSSBA_CHECKED: the kernels check the invariants of the index lists they read or
+            write (labels in [0, Tb), ascending, count == keep) and report a violation in the
+            device status word (SSBA_ERR_CHECK) instead of using the bad value.
 """
 from __future__ import annotations
 
@@ -19,6 +27,11 @@ INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libssba.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+VARIANTS = {"": [], "timeline": ["-DSSBA_TIMELINE"], "checked": ["-DSSBA_CHECKED"]}
+
+
+def library_file(variant: str = "") -> str:
+    return LIB if not variant else os.path.join(HERE, f"libssba_{variant}.so")
 
 
 def _nvcc() -> str:
@@ -45,16 +58,21 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    """Compile every csrc/*.cu for sm_103a and link libssba.so; returns its path."""
-    os.makedirs(OBJDIR, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, extra_flags=(), variant: str = "") -> str:
+    """Compile every csrc/*.cu for sm_103a and link libssba.so (or the variant's library);
+    returns its path."""
+    if variant not in VARIANTS:
+        raise ValueError(f"unknown build variant {variant!r}")
+    objdir = OBJDIR if not variant else OBJDIR + "_" + variant
+    lib = library_file(variant)
+    os.makedirs(objdir, exist_ok=True)
     nvcc = _nvcc()
     hdrs = _headers()
     flags = ARCH + ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
-                    "-I", INCLUDE, "-I", CSRC, "--expt-relaxed-constexpr"] + list(extra_flags)
+                    "-I", INCLUDE, "-I", CSRC, "--expt-relaxed-constexpr"] + VARIANTS[variant] + list(extra_flags)
     jobs = []
     for src in sources():
-        obj = os.path.join(OBJDIR, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(objdir, os.path.basename(src)[:-3] + ".o")
         if force or _stale(obj, [src] + hdrs):
             jobs.append((src, obj))
 
@@ -71,16 +89,17 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
         for out in ex.map(compile_one, jobs):
             if verbose and out:
                 print(out, file=sys.stderr)
-    objs = [os.path.join(OBJDIR, os.path.basename(s)[:-3] + ".o") for s in sources()]
-    if force or jobs or _stale(LIB, objs):
-        tmp = LIB + f".tmp{os.getpid()}"
+    objs = [os.path.join(objdir, os.path.basename(s)[:-3] + ".o") for s in sources()]
+    if force or jobs or _stale(lib, objs):
+        tmp = lib + f".tmp{os.getpid()}"
         cmd = [nvcc, "-shared", "-o", tmp] + objs + ARCH + ["-cudart", "static", "-Xcompiler", "-fPIC"]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose=True))
+    var = next((a.split("=", 1)[1] for a in sys.argv[1:] if a.startswith("--variant=")), "")
+    print(build(force="--force" in sys.argv, verbose=True, variant=var))

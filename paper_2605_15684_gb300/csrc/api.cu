@@ -542,4 +542,13 @@ int ssba_get_status(int32_t* device_status_out)
 
 const char* ssba_last_error(void) { return t_err; }
 
+int ssba_timeline_read(uint64_t* cta, uint32_t* tile, uint32_t* item)
+{
+    if (!cta || !tile || !item) {
+        set_error("ssba_timeline_read: null output");
+        return SSBA_ERR_INVALID;
+    }
+    return timeline_read(reinterpret_cast<unsigned long long*>(cta), tile, item);
+}
+
 }  // extern "C"

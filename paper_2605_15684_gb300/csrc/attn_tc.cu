@@ -112,6 +112,53 @@ struct __align__(1024) SlotSmem {
 
 constexpr int kWinCap = 256;  // labels whose window (origin, box shape) is tabulated per CTA (2048 px: 256)
 
+// Timeline instrumentation, compiled only into the timeline build of the library (-DSSBA_TIMELINE;
+// the default build has none of it). Per CTA, globaltimer stamps (ns) of the launch's phases; per
+// tile of eight sampled pipelines (pipeline 0 and 1 of CTAs 0, 1, gridDim/2 and gridDim-1), SM
+// clock stamps of each role's step, and per item the epilogue's. ssba_timeline_read copies them out.
+namespace tl {
+constexpr int kCtas = 256, kCtaEv = 16, kPipes = 8, kTiles = 128, kTileEv = 12, kItems = 32, kItemEv = 4;
+enum CtaEv { kEntry = 0, kDepWait, kPoolLanded, kPooled, kBarrier, kStaged, kSelected, kPipesStart, kSlot0End,
+             kSlot1End, kEnd, kFirstK, kFirstQ };
+// tile events: K copy issued, QK issued, softmax saw S, softmax done with the exps, P stored,
+// PV issued, V copy issued, QK's wait for a free S buffer over, S in the softmax's registers,
+// row maxima known, P buffer free (softmax), PV's waits over
+enum TileEv { kKIssue = 0, kQKIssue, kSmxStart, kSmxExp, kPStored, kPVIssue, kVIssue, kSFree, kSLoaded, kMaxDone,
+              kPFree, kPVReady };
+enum ItemEv { kEpiStart = 0, kEpiO, kEpiDone, kPipeClock0 };
+#ifdef SSBA_TIMELINE
+__device__ unsigned long long cta_ev[kCtas][kCtaEv];
+__device__ unsigned int tile_ev[kPipes][kTiles][kTileEv];
+__device__ unsigned int item_ev[kPipes][kItems][kItemEv];
+__device__ __forceinline__ int pipe_of(int slot)
+{
+    const int b = blockIdx.x, G = gridDim.x;
+    const int s = b == 0 ? 0 : (b == 1 ? 1 : (b == G / 2 ? 2 : (b == G - 1 ? 3 : -1)));
+    return s < 0 ? -1 : s * 2 + slot;
+}
+#endif
+}  // namespace tl
+#ifdef SSBA_TIMELINE
+#define TL_CTA(ev)                                                                              \
+    do {                                                                                        \
+        if (blockIdx.x < tl::kCtas) tl::cta_ev[blockIdx.x][ev] = ptx::globaltimer_ns();        \
+    } while (0)
+#define TL_TILE(slot, gb, ev)                                                                   \
+    do {                                                                                        \
+        const int tl_p_ = tl::pipe_of(slot);                                                    \
+        if (tl_p_ >= 0 && (gb) < (uint32_t)tl::kTiles) tl::tile_ev[tl_p_][gb][ev] = (unsigned)clock(); \
+    } while (0)
+#define TL_ITEM(slot, n, ev)                                                                    \
+    do {                                                                                        \
+        const int tl_p_ = tl::pipe_of(slot);                                                    \
+        if (tl_p_ >= 0 && (n) < (uint32_t)tl::kItems) tl::item_ev[tl_p_][n][ev] = (unsigned)clock(); \
+    } while (0)
+#else
+#define TL_CTA(ev) do { } while (0)
+#define TL_TILE(slot, gb, ev) do { } while (0)
+#define TL_ITEM(slot, n, ev) do { } while (0)
+#endif
+
 struct __align__(1024) SmemLayout {
     SlotSmem slot[kSlots];
     uint32_t win[kWinCap];  // label -> r0 | c0 << 15 | box shape << 30 (see window_entry)
@@ -288,6 +335,7 @@ __device__ __noinline__ bool pool_phase(const TcParams& p, SmemLayout& cs, int g
             mbar_wait(bar, round & 1, &never, p.budget_ns);
             return false;
         }
+        if (gwarp == 0 && lane == 0 && round == 0) TL_CTA(tl::kPoolLanded);
         float acc[VE];
 #pragma unroll
         for (int e = 0; e < VE; ++e) acc[e] = 0.f;
@@ -528,6 +576,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     SmemLayout& cs = *reinterpret_cast<SmemLayout*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                     ~static_cast<uintptr_t>(1023));
     const int gwarp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) TL_CTA(tl::kEntry);
     // the pipelines' variables are defined after the pooling below, so that they are not live
     // across its call (at 80 registers a thread, values live across a call are spilled)
     {
@@ -571,6 +620,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     // everything above reads no input; the lists, counts and tensors may come from the grid
     // launched just before this one (programmatic dependent launch)
     grid_dep_wait();
+    if (threadIdx.x == 0) TL_CTA(tl::kDepWait);
     bool pool_fail = false;
     if (p.pool_q) {
         // the block means of the whole layer: every warp of the grid one (block, tensor) unit,
@@ -579,6 +629,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         __syncthreads();  // the pooling barriers are initialised
         pool_fail = !pool_phase(p, cs, gwarp, lane, &cs.abort_flag);
         pool_fail = __syncthreads_or(pool_fail);  // also orders this CTA's means before the arrival
+        if (threadIdx.x == 0) TL_CTA(tl::kPooled);
         if (threadIdx.x == 0 && !pool_fail)
             pool_fail = !grid_barrier_arrive_wait(p.gsync, gridDim.x, &cs.abort_flag, p.budget_ns,
                                                   p.withhold != 2 || blockIdx.x != 0);
@@ -587,6 +638,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         // (lists selected from stale means still hold labels in [0, Tb)). No early return and
         // no condition on the selection: either costs the pipeline roles registers (spills).
         pool_fail = __syncthreads_or(pool_fail);
+        if (threadIdx.x == 0) TL_CTA(tl::kBarrier);
         if (pool_fail && threadIdx.x == 0) {
             atomicExch(p.status, SSBA_ERR_TIMEOUT);
             cs.abort_flag = 1;
@@ -654,6 +706,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 }
             asm volatile("cp.async.wait_all;" ::: "memory");
             __syncthreads();
+            if (threadIdx.x == 0 && base == 0) TL_CTA(tl::kStaged);
             // the items whose head is in this batch
             for (int q = gwarp; q < n0 + n1; q += kThreads / 32) {
                 const int item = item_of(q);
@@ -675,6 +728,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             }
             __syncthreads();
         }
+        if (threadIdx.x == 0) TL_CTA(tl::kSelected);
     }
     build_schedule(p, sm, vcta, vgrid, threadIdx.x % (kSlotWarps * 32), kSlotWarps * 32);
     if (gwarp == 0 && lane < 12) tma_prefetch_desc(lane < 4 ? &maps.q[lane] : (lane < 8 ? &maps.k[lane - 4] : &maps.v[lane - 8]));
@@ -690,6 +744,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     tc_fence_after();
     const uint32_t tbase = cs.tmem_base + slot * kSlotCols;
     bool dead = false;
+    if (threadIdx.x == 0) TL_CTA(tl::kPipesStart);
+    if (threadIdx.x % (kSlotWarps * 32) == 0) TL_ITEM(slot, 0u, tl::kPipeClock0);
 
     if (warp == 0 || warp == 2) {
         // ------------------------------------------------------------ TMA producers
@@ -767,6 +823,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     mbar_arrive_expect_tx(full0 + 8 * slot, kTileBytes);
                     if (hold && g == 0) continue;
                     window_boxes_e(m4, tile0 + slot * kTileBytes, full0 + 8 * slot, e, bh);
+                    TL_TILE(gwarp / kSlotWarps, g, is_k ? tl::kKIssue : tl::kVIssue);
                 }
             }
             dead = __shfl_sync(0xffffffffu, dead, 0);
@@ -811,6 +868,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     dead = true;
                     break;
                 }
+                if (lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kSFree);
                 if (!mbar_wait(smem_u32(&sm.k_full[slot]), (gb / kKStages) & 1, abortf, p.budget_ns)) {
                     dead = true;
                     break;
@@ -826,6 +884,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     mma_commit(smem_u32(&sm.s_full[sb]));
                     mma_commit(smem_u32(&sm.k_empty[slot]));
                     if (t == nblk - 1) mma_commit(smem_u32(&sm.q_empty[qb]));  // last read of this Q tile
+                    TL_TILE(gwarp / kSlotWarps, gb, tl::kQKIssue);
                 }
                 __syncwarp();
             }
@@ -861,6 +920,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     dead = true;
                     break;
                 }
+                if (lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kPVReady);
                 tc_fence_after();
                 if (elect_one_sync()) {
                     const uint64_t vdesc = sdesc_sw128(vbase + slot * kTileBytes, 8192, 1024);
@@ -871,6 +931,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                                (t > 0 || k > 0) ? 1u : 0u);
                     mma_commit(smem_u32(&sm.v_empty[slot]));
                     mma_commit(smem_u32(&sm.p_empty[pb]));
+                    TL_TILE(gwarp / kSlotWarps, gb, tl::kPVIssue);
                 }
                 __syncwarp();
             }
@@ -908,12 +969,14 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     dead = true;
                     break;
                 }
+                if (quad == 0 && lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kSmxStart);
                 tc_fence_after();
                 const uint32_t scol = tbase + lane_off + kColS + sb * 64;
                 uint32_t sr[32];
                 tmem_ld_16x32bx2_x16_off32(scol, *reinterpret_cast<uint32_t(*)[16]>(&sr[0]));
                 tmem_ld_16x32bx2_x16_off32(scol + 16, *reinterpret_cast<uint32_t(*)[16]>(&sr[16]));
                 tmem_wait_ld();
+                if (quad == 0 && lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kSLoaded);
                 {
                     // the last text block: its columns past T_txt are zero-filled keys, not keys
                     const int tt = pc.tb + t, valid = p.t_txt - tt * 64;
@@ -954,6 +1017,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                         m_used = mx2;
                     }
                 }
+                if (quad == 0 && lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kMaxDone);
                 // x = s * c - m and the row sums in packed fp32x2 arithmetic (two lanes per op)
                 uint32_t pk[16];
                 const float2 c2 = make_float2(c, c), nm2 = make_float2(-m_used, -m_used);
@@ -968,6 +1032,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 }
                 const float2 lsum = __fadd2_rn(ls2[0], ls2[1]);
                 l = fmaf(l, alpha, lsum.x + lsum.y);
+                if (quad == 0 && lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kSmxExp);
                 // P_t (bf16 pairs) into its TMEM buffer once PV_{t-2} has finished reading it
                 const uint32_t pb = gb % kPBuf;
                 if (gb >= (uint32_t)kPBuf &&
@@ -975,6 +1040,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                     dead = true;
                     break;
                 }
+                if (quad == 0 && lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kPFree);
                 tmem_st_16x32bx2_x16_off16(tbase + lane_off + kColP + pb * 32, pk);
                 if (rescale) {
                     // O must hold every earlier PV before it is rescaled; PV_t waits for p_full
@@ -999,6 +1065,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&sm.p_full[pb]));
+                if (quad == 0 && lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kPStored);
             }
             if (dead) break;
             // hand the row statistics to the epilogue warps
@@ -1025,10 +1092,12 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             const Piece pc = get_piece(p, sm, pi, vcta, vgrid);
             const int bh = pc.item / Tb, label = pc.item - bh * Tb;
             const uint32_t eb = nloc & 1;
+            if (quad == 0 && lane == 0) TL_ITEM(gwarp / kSlotWarps, nloc, tl::kEpiStart);
             if (!mbar_wait(smem_u32(&sm.o_full), nloc & 1, abortf, p.budget_ns)) {
                 dead = true;
                 break;
             }
+            if (quad == 0 && lane == 0) TL_ITEM(gwarp / kSlotWarps, nloc, tl::kEpiO);
             tc_fence_after();
             uint32_t o[32];
             tmem_ld_16x32bx2_x16_off32(tbase + lane_off + kColO, *reinterpret_cast<uint32_t(*)[16]>(&o[0]));
@@ -1112,15 +1181,18 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             rowp[6 + half] = half ? v[3] : r1v;
             if (half == 0)
                 p.lse[(size_t)bh * N + tok] = ok ? (st.x * 0.69314718055994531f + logf(st.y)) : -INFINITY;
+            if (quad == 0 && lane == 0) TL_ITEM(gwarp / kSlotWarps, nloc, tl::kEpiDone);
         }
     }
 
     if (dead) atomicExch(p.status, SSBA_ERR_TIMEOUT);
+    if (threadIdx.x % (kSlotWarps * 32) == 0) TL_CTA(slot == 0 ? tl::kSlot0End : tl::kSlot1End);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     if (gwarp == 1) tmem_dealloc(cs.tmem_base, kTmemCols);
     if (p.pool_q && threadIdx.x == 0 && !cs.abort_flag) grid_barrier_depart(p.gsync, gridDim.x);
+    if (threadIdx.x == 0) TL_CTA(tl::kEnd);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -1322,6 +1394,26 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
         return SSBA_ERR_CUDA;
     }
     return SSBA_OK;
+}
+
+// Timeline of the last launch of the attention kernel on the current device (timeline build only).
+int timeline_read(unsigned long long* cta, unsigned* tile, unsigned* item)
+{
+#ifdef SSBA_TIMELINE
+    if (cudaMemcpyFromSymbol(cta, tl::cta_ev, sizeof(tl::cta_ev)) != cudaSuccess ||
+        cudaMemcpyFromSymbol(tile, tl::tile_ev, sizeof(tl::tile_ev)) != cudaSuccess ||
+        cudaMemcpyFromSymbol(item, tl::item_ev, sizeof(tl::item_ev)) != cudaSuccess) {
+        set_error("ssba_timeline_read: copy from the device failed");
+        return SSBA_ERR_CUDA;
+    }
+    return SSBA_OK;
+#else
+    (void)cta;
+    (void)tile;
+    (void)item;
+    set_error("ssba_timeline_read: this library was built without -DSSBA_TIMELINE");
+    return SSBA_ERR_UNSUPPORTED;
+#endif
 }
 
 // Dense attention from the same kernel: no list, every key block visited in label

@@ -64,6 +64,8 @@ int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const v
                          void* O, float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
 // Bytes of the split-merge workspace of the bf16 forward on the current device.
 size_t attn_tc_workspace_bytes();
+// Copies out the attention kernel's time stamps (timeline build; else SSBA_ERR_UNSUPPORTED).
+int timeline_read(unsigned long long* cta, unsigned* tile, unsigned* item);
 
 int launch_backward(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
                     const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
