@@ -353,7 +353,8 @@ SSBA_API const char* ssba_last_error(void);
  *   cta   host array of 256 x 16 uint64: per CTA, globaltimer nanoseconds of the launch's
  *         phases in this order: entry, dependency wait over, first pooled rows landed, means
  *         stored, grid barrier passed, head means staged, lists selected, pipelines start,
- *         pipeline 0 done, pipeline 1 done, exit (0 where a phase did not run);
+ *         pipeline 0 done, pipeline 1 done, exit, and for warp 0's first item the start of
+ *         its selection, its score row done, its list done (0 where a phase did not run);
  *   tile  host array of 8 x 128 x 12 uint32: for pipelines 0 and 1 of CTAs 0, 1, grid/2 and
  *         grid-1, per tile (the pipeline's running key-block count), SM clock stamps of: K copy
  *         issued, QK issued, softmax saw S, softmax exps done, P stored, PV issued, V copy

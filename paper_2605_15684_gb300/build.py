@@ -6,8 +6,9 @@ without a GPU driver (the driver is only needed once a call reaches the device).
 
 Variants (built only on request, each in a folder and a library of its own, so that the
 default libssba.so is never affected):
-  timeline  -DSSBA_TIMELINE: the attention kernel records time stamps of its phases and of
+  timeline  -DSSBA_TIMELINE=2: the attention kernel records time stamps of its phases and of
             every tile of a few sampled pipelines (read by ssba_timeline_read; see timeline.py);
+  phases    -DSSBA_TIMELINE=1: the phase stamps only, which barely perturb the launch;
   checked   -DSSBA_CHECKED: the kernels check the invariants of the index lists they read or
             write (labels in [0, Tb), ascending, count == keep) and report a violation in the
             device status word (SSBA_ERR_CHECK) instead of using the bad value.
@@ -27,7 +28,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libssba.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-VARIANTS = {"": [], "timeline": ["-DSSBA_TIMELINE"], "checked": ["-DSSBA_CHECKED"]}
+VARIANTS = {"": [], "timeline": ["-DSSBA_TIMELINE=2"], "phases": ["-DSSBA_TIMELINE=1"], "checked": ["-DSSBA_CHECKED"]}
 
 
 def library_file(variant: str = "") -> str:

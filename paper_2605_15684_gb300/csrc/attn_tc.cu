@@ -117,9 +117,9 @@ constexpr int kWinCap = 256;  // labels whose window (origin, box shape) is tabu
 // tile of eight sampled pipelines (pipeline 0 and 1 of CTAs 0, 1, gridDim/2 and gridDim-1), SM
 // clock stamps of each role's step, and per item the epilogue's. ssba_timeline_read copies them out.
 namespace tl {
-constexpr int kCtas = 256, kCtaEv = 16, kPipes = 8, kTiles = 128, kTileEv = 12, kItems = 32, kItemEv = 4;
+constexpr int kCtas = 256, kCtaEv = 16, kPipes = 4 * kSlots, kTiles = 128, kTileEv = 12, kItems = 32, kItemEv = 4;
 enum CtaEv { kEntry = 0, kDepWait, kPoolLanded, kPooled, kBarrier, kStaged, kSelected, kPipesStart, kSlot0End,
-             kSlot1End, kEnd, kFirstK, kFirstQ };
+             kSlot1End, kEnd, kSelStart, kScoresDone, kWalkDone };
 // tile events: K copy issued, QK issued, softmax saw S, softmax done with the exps, P stored,
 // PV issued, V copy issued, QK's wait for a free S buffer over, S in the softmax's registers,
 // row maxima known, P buffer free (softmax), PV's waits over
@@ -134,15 +134,18 @@ __device__ __forceinline__ int pipe_of(int slot)
 {
     const int b = blockIdx.x, G = gridDim.x;
     const int s = b == 0 ? 0 : (b == 1 ? 1 : (b == G / 2 ? 2 : (b == G - 1 ? 3 : -1)));
-    return s < 0 ? -1 : s * 2 + slot;
+    return s < 0 ? -1 : s * kSlots + slot;
 }
 #endif
 }  // namespace tl
+// -DSSBA_TIMELINE=1 records the per-CTA phase stamps only (they barely perturb the launch);
+// -DSSBA_TIMELINE=2 also the per-tile and per-item stamps of the sampled pipelines.
 #ifdef SSBA_TIMELINE
 #define TL_CTA(ev)                                                                              \
     do {                                                                                        \
         if (blockIdx.x < tl::kCtas) tl::cta_ev[blockIdx.x][ev] = ptx::globaltimer_ns();        \
     } while (0)
+#if SSBA_TIMELINE >= 2
 #define TL_TILE(slot, gb, ev)                                                                   \
     do {                                                                                        \
         const int tl_p_ = tl::pipe_of(slot);                                                    \
@@ -153,6 +156,10 @@ __device__ __forceinline__ int pipe_of(int slot)
         const int tl_p_ = tl::pipe_of(slot);                                                    \
         if (tl_p_ >= 0 && (n) < (uint32_t)tl::kItems) tl::item_ev[tl_p_][n][ev] = (unsigned)clock(); \
     } while (0)
+#else
+#define TL_TILE(slot, gb, ev) do { } while (0)
+#define TL_ITEM(slot, n, ev) do { } while (0)
+#endif
 #else
 #define TL_CTA(ev) do { } while (0)
 #define TL_TILE(slot, gb, ev) do { } while (0)
@@ -412,6 +419,8 @@ __device__ __noinline__ void select_item(const TcParams& p, int item, int lane, 
                                          uint32_t* S)
 {
     const int Tb = p.g.Tb();
+    const bool stamp = threadIdx.x == 0 && item == sel_first_item(p, blockIdx.x, gridDim.x * kSlots);
+    if (stamp) TL_CTA(tl::kSelStart);
     const float4* q4 = reinterpret_cast<const float4*>(qs);
     uint32_t key[kPer];
 #pragma unroll
@@ -437,7 +446,9 @@ __device__ __noinline__ void select_item(const TcParams& p, int item, int lane, 
         }
     }
     (void)S;
+    if (stamp) TL_CTA(tl::kScoresDone);
     sel::ballot_select<kPer>(key, Tb, p.keep, lane, const_cast<int32_t*>(p.idx) + (size_t)item * p.keep);
+    if (stamp) TL_CTA(tl::kWalkDone);
     if (lane == 0) p.sel_cnt[item] = p.keep;
     __syncwarp();
 }

@@ -46,9 +46,12 @@ __device__ __forceinline__ void rank_select(const uint32_t* S, int Tb, int keep,
 }
 
 // The same selection with the keys in registers (lane l holds the keys of labels l + 32 m,
-// 0 for labels >= Tb): the keep-th largest key T by an MSB-first radix walk over ballots, then
-// kept = key > T, or key == T among the first equal ones in label order. Same total order, so
-// the same lists as rank_select; 32 rounds of kPer ballots instead of Tb shared-memory reads.
+// 0 for labels >= Tb): an MSB-first radix walk over ballots narrows the keys whose high bits
+// equal a prefix to the group that holds the keep-th largest key; keys above the group are
+// kept, and within it the largest ones, the first equal ones in label order. The walk stops as
+// soon as the group holds exactly the keys still to keep (all of it is then kept; for random
+// scores after about a dozen of the 32 bits). Same total order, so the same lists as
+// rank_select; kPer ballots a round instead of Tb shared-memory reads.
 template <int kPer>
 __device__ __forceinline__ void ballot_select(const uint32_t (&key)[kPer], int Tb, int keep, int lane, int32_t* dst)
 {
@@ -56,24 +59,26 @@ __device__ __forceinline__ void ballot_select(const uint32_t (&key)[kPer], int T
 #pragma unroll
     for (int m = 0; m < kPer; ++m) valid[m] = lane + 32 * m < Tb;
     uint32_t prefix = 0u, pmask = 0u;
-    int remaining = keep;
-#pragma unroll 4
-    for (int bit = 31; bit >= 0; --bit) {
+    int remaining = keep, group = Tb;  // keys still to keep; keys whose bits under pmask equal prefix
+    for (int bit = 31; bit >= 0 && group != remaining; --bit) {
         const uint32_t trial = prefix | (1u << bit), tmask = pmask | (1u << bit);
         int c = 0;
 #pragma unroll
         for (int m = 0; m < kPer; ++m) c += __popc(__ballot_sync(0xffffffffu, valid[m] && (key[m] & tmask) == trial));
-        if (c >= remaining)
+        if (c >= remaining) {
             prefix = trial;
-        else
+            group = c;
+        } else {
             remaining -= c;
+            group -= c;
+        }
         pmask = tmask;
     }
-    const uint32_t T = prefix;
     int out = 0, eq_seen = 0;
 #pragma unroll
     for (int m = 0; m < kPer; ++m) {
-        const bool gt = valid[m] && key[m] > T, eq = valid[m] && key[m] == T;
+        const uint32_t hi = key[m] & pmask;
+        const bool gt = valid[m] && hi > prefix, eq = valid[m] && hi == prefix;
         const uint32_t eqm = __ballot_sync(0xffffffffu, eq);
         const int eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
         const bool kept = gt || (eq && eq_rank < remaining);

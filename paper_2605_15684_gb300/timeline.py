@@ -2,7 +2,7 @@
 its pipelines, from the time stamps of the timeline build (build.py variant "timeline",
 -DSSBA_TIMELINE; the default library records nothing).
 
-    python -m paper_2605_15684_gb300.timeline [--layers 24] [--isolated]
+    python -m paper_2605_15684_gb300.timeline [--layers 24] [--isolated] [--phases-only]
 
 Runs the benchmark's 1024 px step (64 x 64 grid, B = 1, 24 heads x 64, rho = 0.8416, layer l
 with seed l and shift (0,0) / (4,4) alternating, one ssba_forward_fused launch per layer) a few
@@ -28,7 +28,7 @@ from . import api, build, synthetic
 
 CTA_EVENTS = ["entry", "dep wait over", "pool rows landed", "means stored", "grid barrier passed",
               "head means staged", "lists selected", "pipelines start", "pipeline 0 done", "pipeline 1 done",
-              "exit"]
+              "exit", "warp 0 selects", "its score row done", "its list done"]
 TILE_EVENTS = ["K issued", "QK issued", "softmax saw S", "exps done", "P stored", "PV issued", "V issued",
                "S buffer free", "S loaded", "row max known", "P buffer free", "PV waits over"]
 N_CTA, CTA_EV, N_PIPE, N_TILE, TILE_EV, N_ITEM, ITEM_EV = 256, 16, 8, 128, 12, 32, 4
@@ -56,7 +56,7 @@ def report(lib, grid: int, tag: str) -> None:
             ("max known -> exps done", 9, 3), ("exps done -> P buffer free", 3, 10), ("P buffer free -> P stored", 10, 4),
             ("P stored -> next saw S", 4, -1),
             ("P stored -> PV waits over", 4, 11), ("PV waits over -> PV issued", 11, 5),
-            ("K issued -> QK issued", 0, 1), ("V issued -> PV issued", 6, 5),
+            ("K issued -> QK issued", 0, 1),
             ("S buffer free -> QK issued", 7, 1)]
     for pi in range(N_PIPE):
         def ev(t, e):
@@ -92,8 +92,10 @@ def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--layers", type=int, default=24)
     ap.add_argument("--isolated", action="store_true")
+    ap.add_argument("--phases-only", action="store_true",
+                    help="the build that records the phase stamps only (per-tile stamps cost time)")
     args = ap.parse_args()
-    lib = api.load_library(build.build(variant="timeline"))
+    lib = api.load_library(build.build(variant="phases" if args.phases_only else "timeline"))
     dev = torch.device("cuda", 0)
     w = synthetic.PX1024
     L = args.layers
