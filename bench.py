@@ -157,7 +157,36 @@ class ClockSampler:
                                    default=None)}
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the platform string)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.strip().startswith("Model name:"):
+                return ln.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for ln in f:
+                if ln.lower().startswith("model name"):
+                    return ln.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.machine() + " " + platform.processor()
+
+
 # ----------------------------------------------------------------------------- roofline helpers
+def measured_peaks_sustained() -> float:
+    """The measured sustained dense bf16 rate (for a kernel timed inside a long step)."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops_sustained"])
+    except Exception:
+        return 1700.0
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -227,7 +256,7 @@ def run_reference(args, rank):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": config_dict(w, keep, args.layers),
         "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": min(threads, heads_sample),
-                         "kind": "oracle", "sample": sample},
+                         "nproc": os.cpu_count(), "cpu_model": cpu_model(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -335,9 +364,15 @@ def run_ours(args, rank, world):
     F_layer = kept_flops(w.B, w.heads, Tb, keep, w.head_dim)
     value = whole_job_tflops(world, L * F_layer, ms_step * 1e-3)
 
-    # ---- roofline of the dominant kernel (the only one: the fused launch)
+    # ---- roofline of the dominant kernel (the only one: the fused launch). Its average launch
+    #      duration over the timed region is the region's event time over its L * K launches (the
+    #      launches run back to back on one stream, overlapping only through programmatic
+    #      dependent launch); the duration with an event around each launch, which ends that
+    #      overlap, is reported beside it.
     hbm_gbs, bf16_tflops, peak_src = measured_peaks()
-    attn_tflops = F_layer / (attn_ms * 1e-3) / 1e12
+    layer_ms = ms_step / L
+    attn_tflops = F_layer / (layer_ms * 1e-3) / 1e12
+    attn_tflops_ev = F_layer / (attn_ms * 1e-3) / 1e12
     # Q, K, V read and O written once, lse written, the block means written
     attn_bytes = (4 * w.B * w.heads * w.N * w.head_dim * 2 + w.B * w.heads * w.N * 4
                   + 2 * w.B * w.heads * Tb * w.head_dim * 4)
@@ -345,9 +380,15 @@ def run_ours(args, rank, world):
     roofline = {"kernel": "ssba_attn_tc_kernel (ssba_forward_fused)", "bound": "tensor", "achieved": attn_tflops,
                 "peak": bf16_tflops, "unit": "TFLOP/s", "frac": attn_tflops / bf16_tflops,
                 "traffic": traffic, "algorithmic_bytes": attn_bytes,
-                "algorithmic_flops": F_layer, "avg_launch_ms": attn_ms,
+                "algorithmic_flops": F_layer, "avg_launch_ms": layer_ms,
+                "how": "algorithmic flops per launch / (timed-region event time / launches in it)",
+                "per_launch_events": {"avg_launch_ms": attn_ms, "achieved": attn_tflops_ev,
+                                      "frac": attn_tflops_ev / bf16_tflops,
+                                      "how": "an event pair around each launch of K more steps (ends the overlap "
+                                             "of consecutive launches)"},
                 "peak_source": f"{peak_src} dense bf16 (burst)",
-                "hbm_frac": attn_bytes / (attn_ms * 1e-3) / 1e9 / hbm_gbs}
+                "frac_of_sustained": attn_tflops / measured_peaks_sustained(),
+                "hbm_frac": attn_bytes / (layer_ms * 1e-3) / 1e9 / hbm_gbs}
 
     # ---- the same layers with the pooling as a launch of its own (ssba_pool_blocks, then
     #      ssba_forward_select), outside the timed region: its step time, and the pooling kernel's
@@ -423,7 +464,7 @@ def run_ours(args, rank, world):
         for _ in range(3):
             api.forward_dense(descs[0], Qs[0], Ks[0], Vs[0], Od, ld)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        reps = 20
+        reps = L  # the step's layers, back to back like the sparse step
         e0.record(stream)
         for r in range(reps):
             api.forward_dense(descs[r % 2], Qs[r % L], Ks[r % L], Vs[r % L], Od, ld)
@@ -738,6 +779,7 @@ def run_ours(args, rank, world):
         heads_sample = max(1, min(w.heads, threads))
         rate, dt = oracle_sample(w, heads_sample)
         cpu = {"value": rate, "unit": "TFLOP/s", "cores": min(threads, heads_sample), "kind": "oracle",
+               "nproc": os.cpu_count(), "cpu_model": cpu_model(),
                "sample": f"{heads_sample} of {w.heads} heads of one layer (mask + forward), {dt:.2f} s, "
                          f"fp64 C with OpenMP over heads"}
         try:  # one thread at the 512 px config
@@ -797,7 +839,9 @@ def run_ours(args, rank, world):
             "configs_sweep": sweep,
             "qkv_fused": qkv,
             "mask_after_fused_pooling": mask_split,
-            "speedup_vs_dense": (dense_ms / attn_ms) if isinstance(dense_ms, float) else None,
+            "speedup_vs_dense": (dense_ms / layer_ms) if isinstance(dense_ms, float) else None,
+            "speedup_vs_dense_how": "per layer, both back to back over the step's layers: "
+                                    "ssba_forward_dense against the fused sparse launch",
             "ideal_speedup_vs_dense": Tb / keep,
             "e2e": e2e, "cpu_baseline": cpu,
             "gpu_launches": K * L,
