@@ -180,8 +180,11 @@ SSBA_API int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void
  *   dQ, dK, dV      device out, fp32 [B][heads][N][head_dim], every element written.
  *   workspace       device scratch of at least ssba_backward_workspace_bytes(desc) bytes
  *                   (the D_n values), 16-byte aligned.
- * CUDA cores in fp32 (any dtype), head_dim = 64 and block = 8; deterministic (no atomics:
- * the key gradients are gathered per key block over the query blocks that keep it). */
+ * bf16 inputs with head_dim = 64, 8x8 blocks and Tb <= 256 run on the tensor cores (tcgen05
+ * products of 64-row tiles with fp32 accumulation in tensor memory; P and dS rounded to bf16
+ * before their products, as the forward rounds P); fp32 inputs, and other shapes, on CUDA cores
+ * in fp32. head_dim = 64 and block = 8 in both. Deterministic (no atomics: the key gradients are
+ * gathered per key block over the query blocks that keep it). */
 SSBA_API int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, const void* V, const void* O,
                            const float* lse, const void* dO, const int32_t* kv_idx, const int32_t* kv_cnt,
                            float* dQ, float* dK, float* dV, void* workspace, size_t ws_bytes, void* stream);
@@ -307,6 +310,8 @@ SSBA_API int ssba_select_mask(const ssba_desc* desc, const float* qb, const floa
  *   GPU that loads the library holds the scratch area until the process exits.
  *   Set-up: the first call on each device looks up the area's device address with that
  *   device current (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   The address is kept per device and context: after a cudaDeviceReset the next call looks
+ *   it up again (the area then starts afresh, which the build never relies on).
  *   Sharing: every call uses the same area, which keeps the last call's contents. Nothing in
  *   it needs to start at zero (the pooling kernel writes every value the selection kernel
  *   reads). Calls that overlap on the GPU -- on two streams, or from two host threads --

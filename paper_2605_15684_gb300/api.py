@@ -202,13 +202,16 @@ def forward_workspace_bytes(desc: SsbaDesc) -> int:
 _fwd_ws: dict = {}
 
 
-def default_forward_workspace(desc: SsbaDesc, device) -> torch.Tensor:
-    """A zero-filled forward workspace kept per device and reused by every call that
-    passes none. The kernels leave it zero-filled, so calls ordered on one stream can
-    share it; calls that may overlap on the GPU must pass workspaces of their own."""
+def default_forward_workspace(desc: SsbaDesc, device, stream=None) -> torch.Tensor:
+    """A zero-filled forward workspace kept per (device, stream) and reused by every call on
+    that stream that passes none (``stream`` None: the current stream). The kernels leave it
+    zero-filled, so the calls of one stream, which run in order, can share it; calls on two
+    streams get two workspaces, so they never share its counters or barrier words."""
     need = forward_workspace_bytes(desc)
     dev = torch.device(device)
-    key = dev.index if dev.index is not None else torch.cuda.current_device()
+    idx = dev.index if dev.index is not None else torch.cuda.current_device()
+    with torch.cuda.device(idx):
+        key = (idx, _stream_ptr(stream))
     with _lock:
         ws = _fwd_ws.get(key)
         if ws is None or ws.numel() < need:
@@ -365,7 +368,7 @@ def _forward_select_call(fn_name, desc, Q, K, V, qb, kb, kv_idx, kv_cnt, scores,
     _check(O, "O", shp, desc.dtype)
     _check(lse, "lse", shp[:3], torch.float32)
     if isinstance(workspace, str):
-        workspace = default_forward_workspace(desc, dev)
+        workspace = default_forward_workspace(desc, dev, stream)
     wp, wn = _ws_args(workspace)
     _raise_on(getattr(lib, fn_name)(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), qb.data_ptr(),
                                     kb.data_ptr(), kv_idx.data_ptr(), kv_cnt.data_ptr(),
@@ -429,7 +432,7 @@ def build_mask_noalloc(desc: SsbaDesc, Q: torch.Tensor, K: torch.Tensor, kv_idx=
 
 def forward(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O=None, lse=None, workspace="default", stream=None):
     """ssba_forward: returns (O [B,h,N,d] in desc.dtype, lse [B,h,N] fp32).
-    ``workspace``: "default" (the per-device one of default_forward_workspace), None (no
+    ``workspace``: "default" (the per-stream one of default_forward_workspace), None (no
     workspace: whole-query-block shares) or a zero-filled uint8 CUDA tensor."""
     lib = load_library()
     d = desc.c()
@@ -448,7 +451,7 @@ def forward(desc: SsbaDesc, Q, K, V, kv_idx, kv_cnt, O=None, lse=None, workspace
     _check(O, "O", shp, desc.dtype)
     _check(lse, "lse", shp[:3], torch.float32)
     if isinstance(workspace, str):
-        workspace = default_forward_workspace(desc, Q.device) if desc.dtype == torch.bfloat16 else None
+        workspace = default_forward_workspace(desc, Q.device, stream) if desc.dtype == torch.bfloat16 else None
     wp, wn = _ws_args(workspace)
     rc = lib.ssba_forward(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), kv_idx.data_ptr(),
                           kv_cnt.data_ptr(), O.data_ptr(), lse.data_ptr(), wp, wn, _stream_ptr(stream))
@@ -482,7 +485,7 @@ def forward_joint(desc: SsbaDesc, Q, K, V, K_txt, V_txt, kv_idx, kv_cnt, O=None,
     _check(O, "O", shp, desc.dtype)
     _check(lse, "lse", shp[:3], torch.float32)
     if isinstance(workspace, str):
-        workspace = default_forward_workspace(desc, Q.device) if desc.dtype == torch.bfloat16 else None
+        workspace = default_forward_workspace(desc, Q.device, stream) if desc.dtype == torch.bfloat16 else None
     wp, wn = _ws_args(workspace)
     rc = lib.ssba_forward_joint(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(),
                                 K_txt.data_ptr() if T_txt > 0 else None, V_txt.data_ptr() if T_txt > 0 else None,
@@ -506,7 +509,7 @@ def forward_dense(desc: SsbaDesc, Q, K, V, O=None, lse=None, workspace="default"
     _check(O, "O", shp, desc.dtype)
     _check(lse, "lse", shp[:3], torch.float32)
     if isinstance(workspace, str):
-        workspace = default_forward_workspace(desc, Q.device) if desc.dtype == torch.bfloat16 else None
+        workspace = default_forward_workspace(desc, Q.device, stream) if desc.dtype == torch.bfloat16 else None
     wp, wn = _ws_args(workspace)
     rc = lib.ssba_forward_dense(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), O.data_ptr(),
                                 lse.data_ptr(), wp, wn, _stream_ptr(stream))
@@ -711,7 +714,7 @@ class BoundSelectLayer:
         _check(kv_cnt, "kv_cnt", (desc.B, desc.heads, desc.Tb), torch.int32)
         _check(lse, "lse", shp[:3], torch.float32)
         if isinstance(fwd_workspace, str):
-            fwd_workspace = default_forward_workspace(desc, Q.device)
+            fwd_workspace = default_forward_workspace(desc, Q.device, stream)
         fwp, fwn = _ws_args(fwd_workspace)
         if fwp is not None and fwn < forward_workspace_bytes(desc):
             raise SsbaError(SSBA_ERR_WORKSPACE, f"forward workspace needs {forward_workspace_bytes(desc)} bytes")
@@ -759,7 +762,7 @@ class BoundLayer:
         if workspace.numel() * workspace.element_size() < need:
             raise SsbaError(SSBA_ERR_WORKSPACE, f"workspace needs {need} bytes")
         if isinstance(fwd_workspace, str):
-            fwd_workspace = default_forward_workspace(desc, Q.device) if desc.dtype == torch.bfloat16 else None
+            fwd_workspace = default_forward_workspace(desc, Q.device, stream) if desc.dtype == torch.bfloat16 else None
         fwp, fwn = _ws_args(fwd_workspace)
         if fwp is not None and fwn < forward_workspace_bytes(desc):
             raise SsbaError(SSBA_ERR_WORKSPACE, f"forward workspace needs {forward_workspace_bytes(desc)} bytes")

@@ -93,7 +93,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=(), variant: s
     objs = [os.path.join(objdir, os.path.basename(s)[:-3] + ".o") for s in sources()]
     if force or jobs or _stale(lib, objs):
         tmp = lib + f".tmp{os.getpid()}"
-        cmd = [nvcc, "-shared", "-o", tmp] + objs + ARCH + ["-cudart", "static", "-Xcompiler", "-fPIC"]
+        cmd = [nvcc, "-shared", "-o", tmp] + objs + ARCH + ["-cudart", "static", "-Xcompiler", "-fPIC", "-ldl"]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -12,18 +12,75 @@ namespace ssba {
 
 __device__ int g_status = 0;
 
+int current_device()
+{
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return -1;
+    }
+    return dev;
+}
+
+int device_sm_count()
+{
+    static int cache[kMaxDevices] = {};
+    static std::mutex m;
+    const int dev = current_device();
+    if (dev < 0 || dev >= kMaxDevices) return 1;
+    std::lock_guard<std::mutex> lock(m);
+    if (cache[dev] > 0) return cache[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+        cudaGetLastError();
+        return 1;
+    }
+    cache[dev] = n;
+    return n;
+}
+
+uintptr_t current_context_id()
+{
+    typedef int (*CtxGetCurrentFn)(void**);
+    static CtxGetCurrentFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &ptr, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<CtxGetCurrentFn>(ptr);
+    });
+    void* ctx = nullptr;
+    if (!fn || fn(&ctx) != 0) return 0;
+    return reinterpret_cast<uintptr_t>(ctx);
+}
+
+void* device_symbol_address(const void* symbol, void* (&cache)[kMaxDevices], uintptr_t (&ctx)[kMaxDevices],
+                            std::mutex& m)
+{
+    const int dev = current_device();
+    if (dev < 0 || dev >= kMaxDevices) return nullptr;
+    const uintptr_t c = current_context_id();
+    std::lock_guard<std::mutex> lock(m);
+    if (!cache[dev] || ctx[dev] != c) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, symbol) != cudaSuccess || !p) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        cache[dev] = p;
+        ctx[dev] = c;
+    }
+    return cache[dev];
+}
+
 int* device_status_word()
 {
-    constexpr int kMaxDev = 64;
-    static int* addr[kMaxDev] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return nullptr;
-    if (!addr[dev]) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
-        addr[dev] = static_cast<int*>(p);
-    }
-    return addr[dev];
+    static void* addr[kMaxDevices] = {};
+    static uintptr_t ctx[kMaxDevices] = {};
+    static std::mutex m;
+    return static_cast<int*>(device_symbol_address(reinterpret_cast<const void*>(&g_status), addr, ctx, m));
 }
 
 namespace {
@@ -125,6 +182,7 @@ size_t ssba_mask_workspace_bytes(const ssba_desc* desc)
 int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K, int32_t* kv_idx, int32_t* kv_cnt,
                     float* scores_opt, void* workspace, size_t ws_bytes, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_build_mask");
     Grid g;
     int keep;
     int rc = check_desc(desc, "ssba_build_mask", &g, &keep);
@@ -161,6 +219,7 @@ int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K, int32_t
 int ssba_qkv_rope_pool(const ssba_desc* desc, const void* X, const void* Wqkv, const float* bias, void* Q, void* K,
                        void* V, float* qb, float* kb, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_qkv_rope_pool");
     Grid g;
     int keep;
     int rc = check_desc(desc, "ssba_qkv_rope_pool", &g, &keep);
@@ -180,6 +239,7 @@ int ssba_qkv_rope_pool(const ssba_desc* desc, const void* X, const void* Wqkv, c
 int ssba_select_mask(const ssba_desc* desc, const float* qb, const float* kb, int32_t* kv_idx, int32_t* kv_cnt,
                      float* scores_opt, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_select_mask");
     Grid g;
     int keep;
     int rc = check_desc(desc, "ssba_select_mask", &g, &keep);
@@ -212,6 +272,7 @@ size_t ssba_forward_workspace_bytes(const ssba_desc* desc)
 int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void* V, const int32_t* kv_idx,
                  const int32_t* kv_cnt, void* O, float* lse, void* workspace, size_t ws_bytes, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_forward");
     Grid g;
     int keep;
     int rc = check_desc(desc, "ssba_forward", &g, &keep);
@@ -240,6 +301,7 @@ int ssba_forward(const ssba_desc* desc, const void* Q, const void* K, const void
 
 int ssba_pool_blocks(const ssba_desc* desc, const void* Q, const void* K, float* qb, float* kb, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_pool_blocks");
     Grid g;
     int keep;
     int rc = check_desc(desc, "ssba_pool_blocks", &g, &keep);
@@ -296,6 +358,7 @@ int ssba_forward_select(const ssba_desc* desc, const void* Q, const void* K, con
                         const float* kb, int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O, float* lse,
                         void* workspace, size_t ws_bytes, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_forward_select");
     return forward_select_impl("ssba_forward_select", false, desc, Q, K, V, qb, kb, kv_idx, kv_cnt, scores_opt, O,
                                lse, workspace, ws_bytes, stream);
 }
@@ -304,6 +367,7 @@ int ssba_forward_fused(const ssba_desc* desc, const void* Q, const void* K, cons
                        int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O, float* lse, void* workspace,
                        size_t ws_bytes, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_forward_fused");
     return forward_select_impl("ssba_forward_fused", true, desc, Q, K, V, qb, kb, kv_idx, kv_cnt, scores_opt, O, lse,
                                workspace, ws_bytes, stream);
 }
@@ -312,6 +376,7 @@ int ssba_forward_joint(const ssba_desc* desc, const void* Q, const void* K, cons
                        const void* V_txt, int32_t T_txt, const int32_t* kv_idx, const int32_t* kv_cnt, void* O,
                        float* lse, void* workspace, size_t ws_bytes, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_forward_joint");
     Grid g;
     int keep;
     int rc = check_desc(desc, "ssba_forward_joint", &g, &keep);
@@ -338,6 +403,7 @@ int ssba_forward_joint(const ssba_desc* desc, const void* Q, const void* K, cons
 int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void* K, const void* V, void* O, float* lse,
                        void* workspace, size_t ws_bytes, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_forward_dense");
     Grid g;
     int keep;
     int rc = check_desc(desc, "ssba_forward_dense", &g, &keep);
@@ -427,6 +493,7 @@ int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, const voi
                   const void* dO, const int32_t* kv_idx, const int32_t* kv_cnt, float* dQ, float* dK, float* dV,
                   void* workspace, size_t ws_bytes, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_backward");
     Grid g;
     int keep;
     int rc = check_desc(desc, "ssba_backward", &g, &keep);
@@ -469,6 +536,7 @@ static int haar_args(const char* who, const void* in, const void* out, int N, in
 int ssba_haar_dwt(const void* x, void* y, int32_t N, int32_t C, int32_t H, int32_t W, int32_t nb, int32_t dtype,
                   void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_haar_dwt");
     int rc = haar_args("ssba_haar_dwt", x, y, N, C, H, W, nb, dtype);
     if (rc != SSBA_OK) return rc;
     return launch_haar(false, x, y, N, C, H, W, nb, dtype, static_cast<cudaStream_t>(stream));
@@ -477,6 +545,7 @@ int ssba_haar_dwt(const void* x, void* y, int32_t N, int32_t C, int32_t H, int32
 int ssba_haar_iwt(const void* y, void* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t nb, int32_t dtype,
                   void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_haar_iwt");
     int rc = haar_args("ssba_haar_iwt", y, x, N, C, H, W, nb, dtype);
     if (rc != SSBA_OK) return rc;
     return launch_haar(true, y, x, N, C, H, W, nb, dtype, static_cast<cudaStream_t>(stream));
@@ -504,6 +573,7 @@ static int pyramid_args(const char* who, const void* x, void* const* y, int N, i
 int ssba_haar_dwt_pyramid(const void* x, void* const* y, int32_t N, int32_t C, int32_t H, int32_t W, int32_t levels,
                           int32_t nb, int32_t dtype, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_haar_dwt_pyramid");
     int rc = pyramid_args("ssba_haar_dwt_pyramid", x, y, N, C, H, W, levels, nb, dtype);
     if (rc != SSBA_OK) return rc;
     return launch_haar_pyramid(false, const_cast<void*>(x), y, N, C, H, W, levels, nb, dtype,
@@ -513,6 +583,7 @@ int ssba_haar_dwt_pyramid(const void* x, void* const* y, int32_t N, int32_t C, i
 int ssba_haar_iwt_pyramid(void* const* y, void* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t levels,
                           int32_t nb, int32_t dtype, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_haar_iwt_pyramid");
     int rc = pyramid_args("ssba_haar_iwt_pyramid", x, y, N, C, H, W, levels, nb, dtype);
     if (rc != SSBA_OK) return rc;
     return launch_haar_pyramid(true, x, y, N, C, H, W, levels, nb, dtype, static_cast<cudaStream_t>(stream));

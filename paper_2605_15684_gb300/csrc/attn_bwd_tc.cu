@@ -510,12 +510,11 @@ int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale,
         set_error("ssba_backward: could not resolve the device status word");
         return SSBA_ERR_CUDA;
     }
-    static bool attr_set = false;
-    if (!attr_set) {
+    static PerDeviceOnce attr;  // shared-memory attributes, set once per device
+    attr.run([] {
         cudaFuncSetAttribute(ssba_bwd_dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
         cudaFuncSetAttribute(ssba_bwd_dkdv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
-        attr_set = true;
-    }
+    });
     dim3 grid(g.Tb(), d.B * d.heads);
     ssba_bwd_dq_tc_kernel<<<grid, kThreads, kSmemBytes, st>>>(p);
     cudaError_t e = cudaGetLastError();

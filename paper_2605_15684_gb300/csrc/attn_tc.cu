@@ -4,7 +4,7 @@
 //
 // Work item = one query block (64 tokens, an 8x8 window of the shifted grid) of one
 // (batch, head); it visits only the key blocks listed for it. Persistent CTAs, one per SM
-// (a kernel that uses tensor memory gets one CTA per SM), each running two independent
+// (its 205 KB of shared memory fills the SM), each running two independent
 // pipelines of 12 warps (768 threads), warp-specialised by warpgroup:
 //   warp 0      TMA producer (Q, K). Q of each item and K, V of each listed key block arrive as
 //               8 KB tiles cut from [B*heads, H, W, d] tensor maps (128-byte swizzle): one
@@ -292,6 +292,16 @@ __device__ __forceinline__ void tmem_st_16x32bx2_x16_off32(uint32_t taddr, const
 }
 
 __device__ __forceinline__ int clamp_label(int j, int Tb) { return j < 0 ? 0 : (j >= Tb ? Tb - 1 : j); }
+
+// Checked build (-DSSBA_CHECKED, build.py variant "checked"): the invariants of the index lists
+// the kernel reads (every label in [0, Tb), each row strictly ascending, every count in [0, keep])
+// are tested, and a violation is reported as SSBA_ERR_CHECK in the device status word; the value
+// is still clamped as in the default build, which tests nothing.
+#ifdef SSBA_CHECKED
+constexpr bool kChecked = true;
+#else
+constexpr bool kChecked = false;
+#endif
 
 // Block means of the whole layer inside the launch: unit u is (tensor u & 1, item u >> 1), one
 // unit per warp and round, assigned warp-major over the grid so that the CTAs get equal
@@ -785,6 +795,21 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 const int j = list ? clamp_label(ld_list(p, list + t), Tb) : ti0 - p.ntxt + t;
                 lab[t] = j < kWinCap ? cs.win[j] : window_entry(p.g, j);
             }
+            if (kChecked && is_k && list) {
+                // this piece's entries ascending and in range (the one before it too, for a second
+                // part), and the item's count in [0, keep]
+                bool bad = false;
+                for (int t = lane; t < nimg; t += 32) {
+                    const int raw = ld_list(p, list + t);
+                    bad |= raw < 0 || raw >= Tb;
+                    if (t > 0 || ti0 > p.ntxt) bad |= raw <= ld_list(p, list + t - 1);
+                }
+                if (lane == 0 && !p.sel_qb) {
+                    const int c = __ldg(p.cnt + pc.item);
+                    bad |= c < 0 || c > p.keep;
+                }
+                if (__any_sync(0xffffffffu, bad) && lane == 0) atomicExch(p.status, SSBA_ERR_CHECK);
+            }
             __syncwarp();
             if (lane == 0) {
                 if (is_k) {
@@ -1260,19 +1285,8 @@ bool encode_rows_map(CUtensorMap* m, const void* base, int BH, int T)
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int num_sms()
-{
-    static int n = 0;
-    if (n > 0) return n;
-    int dev = 0, m = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&m, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || m <= 0) {
-        cudaGetLastError();
-        return 1;
-    }
-    n = m;
-    return n;
-}
+int num_sms() { return device_sm_count(); }
+PerDeviceOnce g_attn_attr;  // the kernel's shared-memory attributes, set once per device
 
 }  // namespace
 
@@ -1357,15 +1371,13 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
         return SSBA_ERR_CUDA;
     }
     const size_t smem = sizeof(SmemLayout) + 1024;
-    static bool attr_set = false;
-    if (!attr_set) {
+    g_attn_attr.run([smem] {
         cudaFuncSetAttribute(ssba_attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         cudaFuncSetAttribute(ssba_attn_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared);
-        attr_set = true;
-    }
-    // A kernel that uses tensor memory gets one CTA per SM, so each CTA runs kSlots
-    // pipelines; the persistent grid has one CTA per SM (fewer for small problems).
+    });
+    // One CTA fits an SM (shared memory), so each CTA runs kSlots pipelines; the persistent
+    // grid has one CTA per SM (fewer for small problems).
     const int want = (p.num_items + kSlots - 1) / kSlots;
     const int grid = want < max_grid() ? want : max_grid();
     p.split = 0;

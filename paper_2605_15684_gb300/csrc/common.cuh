@@ -1,12 +1,65 @@
 // common.cuh -- shared definitions of the CUDA library (not shared with the oracle).
 #pragma once
 #include <cstdint>
+#include <mutex>
+#include <utility>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 
 #include "ssba.h"
 
 namespace ssba {
+
+// NVTX ranges around the entry points that launch work (named after the entry point), so that a
+// timeline profiler shows each call's host span beside its kernels; -DSSBA_NO_NVTX removes them.
+// The markers cost a few nanoseconds when no profiler is attached.
+#ifndef SSBA_NO_NVTX
+#include <nvtx3/nvToolsExt.h>
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange&) = delete;
+    NvtxRange& operator=(const NvtxRange&) = delete;
+};
+#define SSBA_NVTX_RANGE(name) ::ssba::NvtxRange ssba_nvtx_range_(name)
+#else
+#define SSBA_NVTX_RANGE(name) do { } while (0)
+#endif
+
+// Per-device host state. Devices are told apart by their ordinal (up to kMaxDevices); a launcher
+// that caches something about a device (its SM count, a function attribute it has set, a
+// symbol's address) keeps one entry per ordinal.
+constexpr int kMaxDevices = 64;
+// The current device's ordinal, or -1 if it cannot be read.
+int current_device();
+// SM count of the current device (1 when it cannot be read; not cached then).
+int device_sm_count();
+// Opaque identity of the current context (0 if unknown): a cached device address is valid only
+// in the context it was looked up in (cudaDeviceReset replaces the primary context).
+uintptr_t current_context_id();
+// Device address of a __device__ symbol on the current device, cached per device and context;
+// nullptr on failure.
+void* device_symbol_address(const void* symbol, void* (&cache)[kMaxDevices], uintptr_t (&ctx)[kMaxDevices],
+                            std::mutex& m);
+
+// Runs a function once per device (the current one), thread-safe: for settings such as
+// cudaFuncSetAttribute that hold per device.
+class PerDeviceOnce {
+public:
+    template <class F>
+    void run(F&& f)
+    {
+        const int dev = current_device();
+        if (dev < 0 || dev >= kMaxDevices) {
+            f();
+            return;
+        }
+        std::call_once(flags_[dev], std::forward<F>(f));
+    }
+
+private:
+    std::once_flag flags_[kMaxDevices];
+};
 
 // Device address of the status word (SSBA_OK or SSBA_ERR_TIMEOUT) of the current
 // device, read by ssba_get_status(); kernels that wait receive it as a parameter.

@@ -16,11 +16,13 @@ namespace {
 // Every GPU that loads this library holds these bytes until the process exits.
 static __device__ __align__(256) unsigned char g_mask_scratch[SSBA_NOALLOC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mutex;
 void* g_scratch_addr[kMaxDevices] = {};
+uintptr_t g_scratch_ctx[kMaxDevices] = {};
 
-// Device address of g_mask_scratch on the current device (looked up on first use).
+// Device address of g_mask_scratch on the current device, looked up with that device current on
+// the first call there, and again if the device's context has changed since (a cudaDeviceReset
+// replaces the primary context, and the old address means nothing in the new one).
 int scratch_address(void** out)
 {
     int dev = 0;
@@ -33,8 +35,9 @@ int scratch_address(void** out)
         set_error("ssba_build_mask_noalloc: device ordinal %d out of range", dev);
         return SSBA_ERR_CUDA;
     }
+    const uintptr_t ctx = current_context_id();
     std::lock_guard<std::mutex> lock(g_scratch_mutex);
-    if (!g_scratch_addr[dev]) {
+    if (!g_scratch_addr[dev] || g_scratch_ctx[dev] != ctx) {
         void* p = nullptr;
         e = cudaGetSymbolAddress(&p, g_mask_scratch);
         if (e != cudaSuccess || !p) {
@@ -42,6 +45,7 @@ int scratch_address(void** out)
             return SSBA_ERR_CUDA;
         }
         g_scratch_addr[dev] = p;
+        g_scratch_ctx[dev] = ctx;
     }
     *out = g_scratch_addr[dev];
     return SSBA_OK;
@@ -53,6 +57,7 @@ int scratch_address(void** out)
 extern "C" int ssba_build_mask_noalloc(const ssba_desc* desc, const void* Q, const void* K, int32_t* kv_idx,
                                        int32_t* kv_cnt, float* scores_opt, void* stream)
 {
+    SSBA_NVTX_RANGE("ssba_build_mask_noalloc");
     using namespace ssba;
     const size_t need = ssba_mask_workspace_bytes(desc);
     if (need == 0)  // invalid descriptor: let the regular entry point report why, before any launch

@@ -595,19 +595,7 @@ bool encode_maps(QkvMaps& m, const void* X, const void* Wqkv, int B, int H, int 
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int sm_count()
-{
-    static int n = 0;
-    if (n > 0) return n;
-    int dev = 0, m = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&m, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || m <= 0) {
-        cudaGetLastError();
-        return 1;
-    }
-    n = m;
-    return n;
-}
+int sm_count() { return device_sm_count(); }
 
 }  // namespace
 
@@ -653,12 +641,11 @@ int launch_qkv_rope_pool(const ssba_desc& d, const Grid& g, const void* X, const
         return SSBA_ERR_CUDA;
     }
     const size_t smem = sizeof(QkvSmem) + 1024;
-    static bool attr_set = false;
-    if (!attr_set) {
+    static PerDeviceOnce attr;  // shared-memory attributes, set once per device
+    attr.run([smem] {
         cudaFuncSetAttribute(ssba_qkv_rope_pool_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         cudaFuncSetAttribute(ssba_qkv_rope_pool_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        attr_set = true;
-    }
+    });
     const int grid = p.tiles < sm_count() ? p.tiles : sm_count();
     if (g.H <= kRopeCap && g.W <= kRopeCap)
         ssba_qkv_rope_pool_kernel<true><<<grid, kThreads, smem, st>>>(maps, p);
