@@ -615,7 +615,7 @@ def run_ours(args, rank, world):
     # ---- the other workloads of the paper's range, outside the timed region: the 512 px model
     #      (24 layers), the elastic sweep at 1024 px (32x32 and 64x64 grids x sparsity x batch)
     #      and the 2048 px stress (24 layers, 84 % and 90 %). Per config: the time per layer on
-    #      its path (the fused launch for Tb <= 128, else ssba_build_mask + ssba_forward), the
+    #      its path (the fused launch for Tb <= 256, else ssba_build_mask + ssba_forward), the
     #      effective TFLOP/s over kept blocks and its fraction of the measured peak, and the
     #      same-build dense kernel. Inputs: N(0,1) (512 px: x 1/8) drawn on the device from a
     #      seeded generator, alternating shifts, and enough distinct layers that one pass over
@@ -636,7 +636,7 @@ def run_ours(args, rank, world):
             lc = torch.empty(shp_c[:3], dtype=torch.float32, device=dev)
             ic = torch.empty((Bc, w.heads, Tbc, kc), dtype=torch.int32, device=dev)
             cc = torch.empty((Bc, w.heads, Tbc), dtype=torch.int32, device=dev)
-            if Tbc <= 128:
+            if Tbc <= 256:
                 pq = torch.empty((Bc, w.heads, Tbc, w.head_dim), dtype=torch.float32, device=dev)
                 pk = torch.empty_like(pq)
                 lys = [api.BoundSelectLayer(dsc[l], *ins[l], pq, pk, ic, cc, Oc, lc, stream) for l in range(layers)]

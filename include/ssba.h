@@ -208,7 +208,7 @@ SSBA_API int ssba_pool_blocks(const ssba_desc* desc, const void* Q, const void* 
  *   qb, kb      device, fp32 block means from ssba_pool_blocks (or ssba_qkv_rope_pool).
  *   scores_opt  device out or NULL, fp32 [B][heads][Tb][Tb]: the scores of the selection.
  *   Q, K, V, O, lse, workspace as for ssba_forward.
- * bf16 only; Tb <= 128 (else SSBA_ERR_UNSUPPORTED: use ssba_build_mask + ssba_forward). */
+ * bf16 only; Tb <= 256 (else SSBA_ERR_UNSUPPORTED: use ssba_build_mask + ssba_forward). */
 SSBA_API int ssba_forward_select(const ssba_desc* desc, const void* Q, const void* K, const void* V,
                                  const float* qb, const float* kb, int32_t* kv_idx, int32_t* kv_cnt,
                                  float* scores_opt, void* O, float* lse, void* workspace, size_t ws_bytes,
@@ -228,7 +228,7 @@ SSBA_API int ssba_forward_select(const ssba_desc* desc, const void* Q, const voi
  * The barrier needs every CTA of the grid (one per SM, at most the SM count) resident at once:
  * work on other streams that holds SMs for longer than the wait budget (2 s) makes the call end
  * with SSBA_ERR_TIMEOUT instead of waiting for it.
- * bf16 only; Tb <= 128 (else SSBA_ERR_UNSUPPORTED); SSBA_ERR_WORKSPACE without a workspace. */
+ * bf16 only; Tb <= 256 (else SSBA_ERR_UNSUPPORTED); SSBA_ERR_WORKSPACE without a workspace. */
 SSBA_API int ssba_forward_fused(const ssba_desc* desc, const void* Q, const void* K, const void* V, float* qb,
                                 float* kb, int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O,
                                 float* lse, void* workspace, size_t ws_bytes, void* stream);

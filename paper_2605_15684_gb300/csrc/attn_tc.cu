@@ -745,7 +745,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 }
                 if (Tb <= 32) select_item<1>(p, item, lane, staged(hi), qs, keys);
                 else if (Tb <= 64) select_item<2>(p, item, lane, staged(hi), qs, keys);
-                else select_item<4>(p, item, lane, staged(hi), qs, keys);
+                else if (Tb <= 128) select_item<4>(p, item, lane, staged(hi), qs, keys);
+                else select_item<8>(p, item, lane, staged(hi), qs, keys);
             }
             __syncthreads();
         }
@@ -1314,8 +1315,8 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
         set_error("ssba_forward_fused: needs a forward workspace and the block-mean buffers");
         return SSBA_ERR_WORKSPACE;
     }
-    if (sel_qb && (g.Tb() > 128 || t_txt > 0 || !idx || !cnt)) {
-        set_error("ssba_forward_select: needs Tb <= 128, no text segment and list outputs");
+    if (sel_qb && (g.Tb() > kWinCap || t_txt > 0 || !idx || !cnt)) {
+        set_error("ssba_forward_select: needs Tb <= 256, no text segment and list outputs");
         return SSBA_ERR_UNSUPPORTED;
     }
     if (d.head_dim != kD || g.blk != 8 || (g.sr % 4) || (g.sc % 4)) {

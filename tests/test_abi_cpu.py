@@ -219,9 +219,9 @@ def test_pool_and_select_forward_validation(lib):
     assert fs(d, bad) == api.SSBA_ERR_INVALID
     assert fs(desc(dtype=api.SSBA_FP32), good) == api.SSBA_ERR_UNSUPPORTED
     assert b"bf16" in lib.ssba_last_error()
-    # rows longer than 128 blocks: the two-launch path
-    assert fs(desc(H_tok=96, W_tok=96), good) == api.SSBA_ERR_UNSUPPORTED
-    assert b"Tb <= 128" in lib.ssba_last_error()
+    # rows longer than 256 blocks: the two-launch path
+    assert fs(desc(H_tok=136, W_tok=136), good) == api.SSBA_ERR_UNSUPPORTED
+    assert b"Tb <= 256" in lib.ssba_last_error()
     # the fused launch: the same checks, and a workspace is required (it holds the barrier)
     ff = lambda dd, v, n=0: lib.ssba_forward_fused(ctypes.byref(dd), *v, n, None)
     bad = list(good)
@@ -232,8 +232,8 @@ def test_pool_and_select_forward_validation(lib):
     bad[4] = FAKE + 4  # misaligned kb
     assert ff(d, bad) == api.SSBA_ERR_INVALID
     assert ff(desc(dtype=api.SSBA_FP32), good) == api.SSBA_ERR_UNSUPPORTED
-    assert ff(desc(H_tok=96, W_tok=96), good) == api.SSBA_ERR_UNSUPPORTED
-    assert b"Tb <= 128" in lib.ssba_last_error()
+    assert ff(desc(H_tok=136, W_tok=136), good) == api.SSBA_ERR_UNSUPPORTED
+    assert b"Tb <= 256" in lib.ssba_last_error()
     # its failure-detection hook: the same checks before any launch (workspace required)
     ft = lambda dd, v: lib.ssba_test_fused_timeout(ctypes.byref(dd), *v[:3], *v[3:5], *v[5:7], *v[8:11], 0,
                                                    2_000_000, None)

@@ -157,10 +157,60 @@ def test_forward_select_without_workspace_matches_default():
 
 
 def test_forward_select_rejects_long_rows():
-    q, k, v = (t.cuda() for t in synthetic.qkv(1, 1, 96 * 96, 64, torch.bfloat16, 0))  # Tb = 144
-    desc = api.SsbaDesc(1, 1, 96, 96, rho=0.8, dtype=torch.bfloat16)
+    q, k, v = (t.cuda() for t in synthetic.qkv(1, 1, 136 * 136, 64, torch.bfloat16, 0))  # Tb = 289
+    desc = api.SsbaDesc(1, 1, 136, 136, rho=0.8, dtype=torch.bfloat16)
     qb, kb = api.pool_blocks(desc, q, k)
-    with pytest.raises(api.SsbaError, match="Tb <= 128"):
+    with pytest.raises(api.SsbaError, match="Tb <= 256"):
         api.forward_select(desc, q, k, v, qb, kb)
-    with pytest.raises(api.SsbaError, match="Tb <= 128"):
+    with pytest.raises(api.SsbaError, match="Tb <= 256"):
         api.forward_fused(desc, q, k, v)
+
+
+@pytest.mark.parametrize("B,h,H,W,shift,rho", [
+    (1, 4, 96, 96, (4, 4), 0.8),      # Tb = 144: eight labels per lane in the selection
+    (1, 3, 112, 112, (0, 0), 0.9),    # Tb = 196
+])
+def test_forward_fused_long_rows_matches_oracle(B, h, H, W, shift, rho):
+    """Rows of 129 to 256 blocks on the one-launch path: means, lists (exact on the launch's S,
+    margin-gated against the oracle) and O / lse against the oracle, every head."""
+    q, k, v = synthetic.qkv(B, h, H * W, 64, torch.bfloat16, 7)
+    desc = api.SsbaDesc(B, h, H, W, shift_r=shift[0], shift_c=shift[1], rho=rho, dtype=torch.bfloat16)
+    O, lse, idx, cnt, qb, kb, S = api.forward_fused(desc, q.cuda(), k.cuda(), v.cuda(), scores=True)
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
+    ref_q = oracle.pooled_blocks(q.double().numpy(), H, W, 8, shift)
+    mag = oracle.pooled_blocks(np.abs(q.double().numpy()), H, W, 8, shift)
+    assert np.all(np.abs(qb.cpu().double().numpy() - ref_q) <= 2.0 ** -17 * mag + 1e-12)
+    Tb = H * W // 64
+    keep = oracle.keep_count(Tb, rho)
+    idx_o, _, S_o = oracle.build_mask(q, k, H, W, 8, shift, rho, return_scores=True)
+    near = check_mask(idx.cpu().numpy(), cnt.cpu().numpy(), S.cpu().numpy(), S_o, idx_o, keep)
+    assert near < 0.1 * B * h * Tb
+    Oo, lo = oracle.forward(q, k, v, idx.cpu().numpy(), H, W, 8, shift)
+    check_out(O.float().cpu().numpy(), lse.cpu().numpy(), Oo, lo, "bf16")
+
+
+def test_forward_fused_2048px_matches_oracle():
+    """The 2048 px stress layer (128 x 128 grid, 24 heads, rho 0.84 -> keep 41 of 256) in one
+    launch: every head's lists exact on the launch's S and margin-gated against the oracle; O and
+    lse on 96 sampled query rows of heads 0 and 23 against the oracle; equal to the two-launch
+    path's lists."""
+    H = W = 128
+    q, k, v = synthetic.qkv(1, 24, H * W, 64, torch.bfloat16, 0)
+    qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
+    desc = api.SsbaDesc(1, 24, H, W, shift_r=4, shift_c=4, rho=0.84, dtype=torch.bfloat16)
+    O, lse, idx, cnt, qb, kb, S = api.forward_fused(desc, qd, kd, vd, scores=True)
+    idx2, cnt2 = api.build_mask(desc, qd, kd)
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
+    assert torch.equal(idx, idx2) and torch.equal(cnt, cnt2)
+    keep = oracle.keep_count(256, 0.84)
+    idx_o, _, S_o = oracle.build_mask(q, k, H, W, 8, (4, 4), 0.84, return_scores=True)
+    near = check_mask(idx.cpu().numpy(), cnt.cpu().numpy(), S.cpu().numpy(), S_o, idx_o, keep)
+    assert near < 0.1 * 24 * 256
+    lab = oracle.partition(H, W, 8, (4, 4))
+    rows = np.sort(np.random.default_rng(0).choice(H * W, 96, replace=False)).astype(np.int32)
+    idx_np = idx.cpu().numpy()
+    for head in (0, 23):
+        O_o, lse_o = oracle.attention_rows(q[0, head], k[0, head], v[0, head], lab, idx_np[0, head], rows)
+        check_out(O[0, head].float().cpu().numpy()[rows], lse[0, head].cpu().numpy()[rows], O_o, lse_o, "bf16")
