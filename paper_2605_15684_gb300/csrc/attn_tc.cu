@@ -1440,11 +1440,18 @@ int timeline_read(unsigned long long* cta, unsigned* tile, unsigned* item)
 #endif
 }
 
-// Dense attention from the same kernel: no list, every key block visited in label
-// order with query tiles of one 8x8 block each (unshifted grid).
+// Dense attention: the 128-token-tile kernel (attn_dense.cu) when N is a multiple of 128, else
+// this kernel with no list, every key block visited in label order with query tiles of one 8x8
+// block each (unshifted grid).
 int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V, void* O,
                          float* lse, void* ws, size_t ws_bytes, cudaStream_t st)
 {
+    if (ws && ws_bytes < attn_tc_workspace_bytes()) {  // the rules of ssba_forward, whichever kernel runs
+        set_error("ssba_forward_dense: workspace of %zu bytes, %zu needed", ws_bytes, attn_tc_workspace_bytes());
+        return SSBA_ERR_WORKSPACE;
+    }
+    const int rc = launch_dense_m128(d, scale, Q, K, V, O, lse, st);
+    if (rc != SSBA_ERR_UNSUPPORTED) return rc;
     if (d.head_dim != kD || d.H_tok % 8 || d.W_tok % 8) {
         set_error("ssba_forward_dense: needs head_dim=64 and H_tok, W_tok multiples of 8");
         return SSBA_ERR_UNSUPPORTED;

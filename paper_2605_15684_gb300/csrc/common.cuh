@@ -113,6 +113,10 @@ int launch_attn_tc_bf16(const ssba_desc& d, const Grid& g, int keep, float scale
                         uint64_t budget_ns = kWaitBudgetNs, int withhold = 0, const void* Kt = nullptr,
                         const void* Vt = nullptr, int t_txt = 0, const float* sel_qb = nullptr,
                         const float* sel_kb = nullptr, float* sel_scores = nullptr, bool pool = false);
+// Dense attention with 128-token tiles (M=128 products; head_dim 64, bf16, N a multiple of 128);
+// returns SSBA_ERR_UNSUPPORTED without launching for other shapes.
+int launch_dense_m128(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V, void* O,
+                      float* lse, cudaStream_t st);
 int launch_dense_tc_bf16(const ssba_desc& d, float scale, const void* Q, const void* K, const void* V,
                          void* O, float* lse, void* ws, size_t ws_bytes, cudaStream_t st);
 // Bytes of the split-merge workspace of the bf16 forward on the current device.

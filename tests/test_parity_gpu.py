@@ -181,6 +181,22 @@ def test_forward_dense_bf16():
     check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
 
 
+@pytest.mark.parametrize("B,h,H,W", [
+    (1, 24, 64, 64),   # 1024 px: the 128-token-tile kernel, 32 key tiles a row
+    (2, 16, 32, 32),   # B > 1, units spread over the streams unevenly
+    (1, 3, 24, 40),    # N = 960, not a multiple of 128: the 64-row path
+])
+def test_forward_dense_bf16_shapes(B, h, H, W):
+    """ssba_forward_dense (Table 2's 0 % sparsity baseline) against the oracle's dense attention."""
+    q, k, v, qd, kd, vd = _inputs(B, h, H, W, torch.bfloat16, seed=4)
+    desc = api.SsbaDesc(B, h, H, W)
+    O, lse = api.forward_dense(desc, qd, kd, vd)
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
+    O_o, lse_o = oracle.dense_forward(q, k, v)
+    check_out(O.float().cpu().numpy(), lse.cpu().numpy(), O_o, lse_o, "bf16")
+
+
 def test_end_to_end_layer_with_gpu_mask():
     """build_mask then forward on the GPU (the path bench.py times), against the oracle
     forward run on the GPU's own lists."""
