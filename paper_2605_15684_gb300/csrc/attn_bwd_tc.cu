@@ -4,25 +4,31 @@
 // For the output gradient dO, with p_nm = exp(scale q_n.k_m - lse_n) over the kept pairs:
 //   D_n = dO_n . O_n,  ds_nm = p_nm (dO_n . v_m - D_n),
 //   dQ_n = scale sum_m ds_nm k_m,  dK_m = scale sum_n ds_nm q_n,  dV_m = sum_n p_nm dO_n.
-// Two kernels, as the CUDA-core version, deterministic (no atomics), 128 threads per CTA,
-// one (batch*head, block) per CTA, each 64 x 64 tile product a tcgen05.mma kind::f16 with
-// M=64 (four K=16 steps) issued by one thread:
+// Two kernels, as the CUDA-core version, deterministic (no atomics), one (batch*head, block)
+// per CTA, each 64 x 64 tile product a tcgen05.mma kind::f16 with M=64 (four K=16 steps).
+// 160 threads: warps 0-3 own the TMEM lane quadrants (the exps, the bf16 operands, the tile
+// copies, the epilogue); lane 0 of warp 4 issues every MMA, so that issuing (some 80 cycles
+// an instruction) runs beside the compute warps instead of in front of them. The two sides
+// meet on mbarriers: MMA commits one way, one arrive per compute warp the other.
 //   ssba_bwd_dq_tc_kernel    query block i: for each kept key block j (list order)
 //                              S  = Q_i K_j^T,  dP = dO_i V_j^T        (A, B from shared memory)
-//                              dS = P o (dP - D) in registers, bf16 back into TMEM over S
-//                              dQ += dS K_j                           (A from TMEM, B MN-major)
+//                              dS = P o (dP - D) in registers, bf16 into shared memory
+//                              dQ += dS K_j                           (B read MN-major)
 //                            and writes D for the second kernel.
 //   ssba_bwd_dkdv_tc_kernel  key block j: for each query block i whose list holds j (ascending)
 //                              S^T = K_j Q_i^T,  dP^T = V_j dO_i^T
-//                              P^T, dS^T in registers, bf16 back into TMEM over S^T and dP^T
+//                              P^T, dS^T in registers, bf16 into shared memory
 //                              dV += P^T dO_i,  dK += dS^T Q_i
 // Tiles are gathered token by token (the shifted window) with 16-byte cp.async into the
 // 128-byte-swizzled layout the MMA descriptors read (K-major for A/B, MN-major as the second
-// operand of the accumulating products), the next pair's tiles in flight while the current
-// one computes. TMEM: S, dP, and one or two fp32 accumulators (256 columns, two CTAs per SM).
-// The thread that owns TMEM lane (row) r of the M=64 data path holds half a row: columns
-// [32 h, 32 h + 32), h = lane / 16. Every mbarrier wait is bounded; a timeout is written to the
-// device status word and the CTA drains its MMAs before it exits.
+// operand of the accumulating products), in three buffers: pair t computes, pair t + 1's tiles
+// are resident and pair t + 2's are in flight. S_{t+1} and dP_{t+1} are issued as soon as
+// S_t and dP_t are in registers, so the tensor core runs the next pair's products while the
+// threads form this pair's bf16 operands. TMEM: S, dP and one or two fp32 accumulators
+// (256 columns, two CTAs per SM). The thread that owns TMEM lane (row) r of the M=64 data
+// path holds half a row: columns [32 h, 32 h + 32), h = lane / 16. Every mbarrier wait is
+// bounded; a timeout is written to the device status word and the CTA drains its MMAs before
+// it exits.
 #include <cstdint>
 
 #include "common.cuh"
@@ -36,17 +42,24 @@ using namespace ptx;
 
 constexpr int kD = 64;
 constexpr int kT = 64;                   // tokens per block
-constexpr int kThreads = 128;
+constexpr int kCompute = 128;  // warps 0-3: one TMEM lane quadrant each
+constexpr int kThreads = 160;  // + warp 4, whose lane 0 issues every MMA of the CTA
+constexpr int kIssuer = 128;
 constexpr uint32_t kTile = kT * kD * 2;  // 8 KB
 constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kColS = 0, kColDP = 64, kColA0 = 128, kColA1 = 192;
 constexpr uint32_t kIdescK = idesc_bf16_f32(64, 64, false, false);  // A, B K-major
 constexpr uint32_t kIdescMN = idesc_bf16_f32(64, 64, false, true);  // B MN-major
+constexpr float kLog2e = 1.4426950408889634f;
 constexpr size_t kSmemBytes = 100 * 1024;  // also keeps residency at two CTAs per SM (TMEM)
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src)
 {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
@@ -74,13 +87,14 @@ __device__ __forceinline__ int win_token(const Grid& g, WinOrigin o, int pos)
 }
 
 // Block `label` of a [N][64] bf16 head into a 1024-aligned 8 KB tile: row r = in-window
-// position r, 16-byte chunk c at chunk c ^ (r & 7) (the 128-byte swizzle).
+// position r, 16-byte chunk c at chunk c ^ (r & 7) (the 128-byte swizzle). Called by the
+// compute threads.
 __device__ __forceinline__ void load_tile(uint32_t dst, const __nv_bfloat16* X, const Grid& g, int label)
 {
     const WinOrigin o = win_origin(g, label);
 #pragma unroll
-    for (int i = 0; i < kT * 8 / kThreads; ++i) {
-        const int e = threadIdx.x + i * kThreads, r = e >> 3, c = e & 7;
+    for (int i = 0; i < kT * 8 / kCompute; ++i) {
+        const int e = threadIdx.x + i * kCompute, r = e >> 3, c = e & 7;
         cp_async16(dst + r * 128 + ((c ^ (r & 7)) << 4), X + (size_t)win_token(g, o, r) * kD + c * 8);
     }
 }
@@ -106,26 +120,42 @@ __device__ __forceinline__ void mma_kk(uint32_t col, uint32_t a, uint32_t b)
     for (int k = 0; k < 4; ++k) mma_ss(col, ad + (uint64_t)(k * 2), bd + (uint64_t)(k * 2), kIdescK, k > 0 ? 1u : 0u);
 }
 
-// C (+)= A B with A (64 x 64 bf16, packed pairs) in TMEM at column `acol` and B the shared tile
-// read MN-major (rows = the contraction index).
-__device__ __forceinline__ void mma_tb(uint32_t col, uint32_t acol, uint32_t b, bool accumulate)
+// C (+)= A B with A (64 x 64 bf16) a K-major shared tile and B a shared tile read MN-major
+// (rows = the contraction index).
+__device__ __forceinline__ void mma_sb(uint32_t col, uint32_t a, uint32_t b, bool accumulate)
 {
-    const uint64_t bd = sdesc_sw128(b, 8192, 1024);
+    const uint64_t ad = sdesc_sw128(a, 16, 1024), bd = sdesc_sw128(b, 8192, 1024);
 #pragma unroll
     for (int k = 0; k < 4; ++k)
-        mma_ts(col, acol + k * 8, bd + (uint64_t)(k * 128), kIdescMN, (accumulate || k > 0) ? 1u : 0u);
+        mma_ss(col, ad + (uint64_t)(k * 2), bd + (uint64_t)(k * 128), kIdescMN, (accumulate || k > 0) ? 1u : 0u);
+}
+
+// This thread's half row (row r of the M=64 data path, columns [32 h, 32 h + 32)) of a 64 x 64
+// bf16 tile, 16 packed pairs, into the 128-byte-swizzled K-major layout at dst.
+__device__ __forceinline__ void store_half_row(uint8_t* dst, int r, int h, const uint32_t (&v)[16])
+{
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int c = 4 * h + i;
+        *reinterpret_cast<uint4*>(dst + r * 128 + ((c ^ (r & 7)) << 4)) =
+            make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    }
 }
 
 struct alignas(1024) BwdSmem {
     uint8_t a[kTile];        // dq: Q_i;  dkdv: K_j
     uint8_t b[kTile];        // dq: dO_i; dkdv: V_j
-    uint8_t x[2][kTile];     // dq: K_j;  dkdv: Q_i   (double-buffered)
-    uint8_t y[2][kTile];     // dq: V_j;  dkdv: dO_i
-    float ls[2][kT];         // dkdv: lse * log2(e) of the query block
-    float ds[2][kT];         // dkdv: D of the query block
+    uint8_t x[3][kTile];     // dq: K_j;  dkdv: Q_i   (three buffers: pair t computes, t + 1 is
+    uint8_t y[3][kTile];     // dq: V_j;  dkdv: dO_i   loaded, t + 2 is being copied)
+    uint8_t e[2][kTile];     // dq: dS (e[0]); dkdv: P^T, dS^T -- bf16, the A operands of the
+                             // accumulating products, written from registers
+    float ls[3][kT];         // dkdv: lse of the query block
+    float ds[3][kT];         // dkdv: D of the query block
     int list[256];           // dkdv: the query blocks holding this key block, ascending
     int wcount[kThreads / 32];
-    uint64_t bar_s, bar_a, drain;
+    uint64_t bar_s, bar_a, drain;  // MMA commits: S and dP ready; accumulators updated; drain
+    uint64_t full_s, full_a;       // compute warps (one arrive each): S, dP read and the next
+                                   // tiles landed; the bf16 operands stored
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -157,6 +187,8 @@ __device__ __forceinline__ void setup(BwdSmem& sm)
         mbar_init(smem_u32(&sm.bar_s), 1);
         mbar_init(smem_u32(&sm.bar_a), 1);
         mbar_init(smem_u32(&sm.drain), 1);
+        mbar_init(smem_u32(&sm.full_s), kCompute / 32);
+        mbar_init(smem_u32(&sm.full_a), kCompute / 32);
         fence_mbar_init();
     }
     if (threadIdx.x < 32) {
@@ -172,20 +204,33 @@ __device__ __forceinline__ void teardown(BwdSmem& sm, const BwdParams& p, bool d
 {
     cp_async_wait<0>();
     if (dead) {
-        if (threadIdx.x == 0) {
-            if (issued) {  // the MMAs still in flight
-                mma_commit(smem_u32(&sm.drain));
-                const uint64_t t0 = globaltimer_ns();
-                while (!mbar_try_wait(smem_u32(&sm.drain), 0) && globaltimer_ns() - t0 < p.budget_ns) {
-                }
+        if (threadIdx.x == kIssuer && issued) {  // the MMAs still in flight
+            mma_commit(smem_u32(&sm.drain));
+            const uint64_t t0 = globaltimer_ns();
+            while (!mbar_try_wait(smem_u32(&sm.drain), 0) && globaltimer_ns() - t0 < p.budget_ns) {
             }
-            atomicExch(p.status, SSBA_ERR_TIMEOUT);
         }
+        if (threadIdx.x == 0) atomicExch(p.status, SSBA_ERR_TIMEOUT);
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     if (threadIdx.x < 32) tmem_dealloc(sm.tmem_base, kTmemCols);
+}
+
+// A compute warp's bounded wait: the warp goes on only if every lane saw the phase, so that a
+// timeout takes the whole warp out of the loop at once.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abortf, uint64_t budget_ns)
+{
+    const bool ok = mbar_wait(bar, parity, abortf, budget_ns);
+    return __all_sync(0xffffffffu, ok);
+}
+
+// One arrive per compute warp, after every lane's TMEM loads and shared-memory writes.
+__device__ __forceinline__ void warp_arrive(uint32_t bar)
+{
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
 }
 
 // Writes the 64 x 64 fp32 accumulator at TMEM column `col`, times `mul`, to rows
@@ -212,115 +257,134 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dq_tc_kernel(const BwdParam
     const Grid g = p.g;
     const int Tb = g.Tb(), N = g.H * g.W;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = lane >> 4;
-    const int r = warp * 16 + (lane & 15);
+    const int r = (warp & 3) * 16 + (lane & 15);  // tile row of a compute thread
     const size_t head = (size_t)bh * N * kD;
     const size_t row = (size_t)bh * N + g.token(label, r);
     volatile int* abortf = &sm.abort_flag;
-    setup(sm);
-    const uint32_t tb = sm.tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
-    const uint32_t tb0 = sm.tmem_base;
-
-    // D for this row (both halves of the row's threads hold it) and the log2-domain lse
-    float Dr = 0.f;
-    {
-        const uint4* go = reinterpret_cast<const uint4*>(p.dO + row * kD + 32 * h);
-        const uint4* oo = reinterpret_cast<const uint4*>(p.O + row * kD + 32 * h);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const uint4 a = __ldg(go + i), b = __ldg(oo + i);
-            const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const float2 fa = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&aw[k]));
-                const float2 fb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&bw[k]));
-                Dr = fmaf(fa.x, fb.x, Dr);
-                Dr = fmaf(fa.y, fb.y, Dr);
-            }
-        }
-    }
-    Dr += __shfl_xor_sync(0xffffffffu, Dr, 16);
-    if (h == 0) p.Dbuf[row] = Dr;
-    const float c = p.scale * 1.4426950408889634f;
-    const float L2 = p.lse[row] * 1.4426950408889634f;
-
+    // the kept key blocks into shared memory (visible after the set-up's barrier)
     const int32_t* list = p.idx + ((size_t)bh * Tb + label) * p.keep;
     const int n = min(max(p.cnt[(size_t)bh * Tb + label], 0), p.keep);
-    load_tile(smem_u32(sm.a), p.Q + head, g, label);
-    load_tile(smem_u32(sm.b), p.dO + head, g, label);
-    if (n > 0) {
-        const int j0 = min(max(list[0], 0), Tb - 1);
-        load_tile(smem_u32(sm.x[0]), p.K + head, g, j0);
-        load_tile(smem_u32(sm.y[0]), p.V + head, g, j0);
-    }
-    cp_async_commit();
+    for (int i = threadIdx.x; i < n; i += kThreads) sm.list[i] = min(max(__ldg(list + i), 0), Tb - 1);
+    setup(sm);
+    const uint32_t tb = sm.tmem_base + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    const uint32_t tb0 = sm.tmem_base;
     bool dead = false;
     uint32_t issued = 0;
-    for (int t = 0; t < n && !dead; ++t) {
-        const int buf = t & 1;
-        // pair t-1's dQ product has read dS (TMEM over S) and the other buffers: only then may
-        // S be overwritten and those buffers refilled (every wait ends in a CTA-wide vote, so
-        // that no thread leaves the loop while another waits at a barrier in it)
-        if (t >= 1) {
-            const bool ok = mbar_wait(smem_u32(&sm.bar_a), (t - 1) & 1, abortf, p.budget_ns);
-            if (__syncthreads_or(!ok)) {
-                dead = true;
-                break;
-            }
-        }
-        if (t + 1 < n) {
-            const int jn = min(max(list[t + 1], 0), Tb - 1);
-            load_tile(smem_u32(sm.x[buf ^ 1]), p.K + head, g, jn);
-            load_tile(smem_u32(sm.y[buf ^ 1]), p.V + head, g, jn);
+
+    if (threadIdx.x < kCompute) {
+        // tiles of pair t in buffer t % 3: K_j in x, V_j in y
+        auto fetch = [&](int t) {
+            const int j = sm.list[t];
+            load_tile(smem_u32(sm.x[t % 3]), p.K + head, g, j);
+            load_tile(smem_u32(sm.y[t % 3]), p.V + head, g, j);
             cp_async_commit();
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
-        }
-        fence_proxy_async_smem();  // the tiles this thread copied, visible to the tensor cores
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            tc_fence_after();
-            mma_kk(tb0 + kColS, smem_u32(sm.a), smem_u32(sm.x[buf]));   // S = Q K^T
-            mma_kk(tb0 + kColDP, smem_u32(sm.b), smem_u32(sm.y[buf]));  // dP = dO V^T
-            mma_commit(smem_u32(&sm.bar_s));
-        }
-        issued = 1;
+        };
+        load_tile(smem_u32(sm.a), p.Q + head, g, label);
+        load_tile(smem_u32(sm.b), p.dO + head, g, label);
+        cp_async_commit();
+        if (n > 0) fetch(0);
+        if (n > 1) fetch(1);
+
+        // D for this row (both halves of the row's threads hold it) and the log2-domain lse,
+        // while the tiles are in flight
+        float Dr = 0.f;
         {
-            const bool ok = mbar_wait(smem_u32(&sm.bar_s), t & 1, abortf, p.budget_ns);
-            if (__syncthreads_or(!ok)) {
+            const uint4* go = reinterpret_cast<const uint4*>(p.dO + row * kD + 32 * h);
+            const uint4* oo = reinterpret_cast<const uint4*>(p.O + row * kD + 32 * h);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint4 a = __ldg(go + i), b = __ldg(oo + i);
+                const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const float2 fa = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&aw[k]));
+                    const float2 fb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&bw[k]));
+                    Dr = fmaf(fa.x, fb.x, Dr);
+                    Dr = fmaf(fa.y, fb.y, Dr);
+                }
+            }
+        }
+        Dr += __shfl_xor_sync(0xffffffffu, Dr, 16);
+        if (h == 0) p.Dbuf[row] = Dr;
+        const float c = p.scale * kLog2e;
+        const float L2 = p.lse[row] * kLog2e;
+        if (n > 0) {  // Q, dO and the tiles of pair 0 landed
+            if (n > 1) cp_async_wait<1>(); else cp_async_wait<0>();
+            fence_proxy_async_smem();
+            warp_arrive(smem_u32(&sm.full_s));
+        }
+        // Pair t: S_t, dP_t into registers, then the issuer may overwrite them with pair t + 1's
+        // products; dS_t goes to shared memory once dQ_{t-1} has read the last one.
+        for (int t = 0; t < n; ++t) {
+            if (!warp_wait(smem_u32(&sm.bar_s), t & 1, abortf, p.budget_ns)) {
                 dead = true;
                 break;
             }
-        }
-        tc_fence_after();
-        uint32_t s[32], dp[32];
-        tmem_ld_16x32bx2_x16_off32(tb + kColS, *reinterpret_cast<uint32_t(*)[16]>(&s[0]));
-        tmem_ld_16x32bx2_x16_off32(tb + kColS + 16, *reinterpret_cast<uint32_t(*)[16]>(&s[16]));
-        tmem_ld_16x32bx2_x16_off32(tb + kColDP, *reinterpret_cast<uint32_t(*)[16]>(&dp[0]));
-        tmem_ld_16x32bx2_x16_off32(tb + kColDP + 16, *reinterpret_cast<uint32_t(*)[16]>(&dp[16]));
-        tmem_wait_ld();
-        uint32_t pk[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            const float p0 = fast_exp2(fmaf(__uint_as_float(s[2 * i]), c, -L2));
-            const float p1 = fast_exp2(fmaf(__uint_as_float(s[2 * i + 1]), c, -L2));
-            pk[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - Dr), p1 * (__uint_as_float(dp[2 * i + 1]) - Dr));
-        }
-        tmem_st_16x32bx2_x16_off16(tb + kColS, pk);  // dS (bf16 pairs) over S
-        tmem_wait_st();
-        tc_fence_before();
-        __syncthreads();
-        if (threadIdx.x == 0) {
             tc_fence_after();
-            mma_tb(tb0 + kColA0, tb0 + kColS, smem_u32(sm.x[buf]), t > 0);  // dQ += dS K
-            mma_commit(smem_u32(&sm.bar_a));
+            uint32_t s[32], dp[32];
+            tmem_ld_16x32bx2_x16_off32(tb + kColS, *reinterpret_cast<uint32_t(*)[16]>(&s[0]));
+            tmem_ld_16x32bx2_x16_off32(tb + kColS + 16, *reinterpret_cast<uint32_t(*)[16]>(&s[16]));
+            tmem_ld_16x32bx2_x16_off32(tb + kColDP, *reinterpret_cast<uint32_t(*)[16]>(&dp[0]));
+            tmem_ld_16x32bx2_x16_off32(tb + kColDP + 16, *reinterpret_cast<uint32_t(*)[16]>(&dp[16]));
+            tmem_wait_ld();
+            tc_fence_before();
+            if (t + 1 < n) {  // the tiles of pair t + 1 (copied during pair t - 1)
+                cp_async_wait<0>();
+                fence_proxy_async_smem();
+            }
+            warp_arrive(smem_u32(&sm.full_s));
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const float p0 = fast_exp2(fmaf(__uint_as_float(s[2 * i]), c, -L2));
+                const float p1 = fast_exp2(fmaf(__uint_as_float(s[2 * i + 1]), c, -L2));
+                pk[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - Dr), p1 * (__uint_as_float(dp[2 * i + 1]) - Dr));
+            }
+            // dQ_{t-1} has read the last dS and the tiles of pair t - 1
+            if (t >= 1 && !warp_wait(smem_u32(&sm.bar_a), (t - 1) & 1, abortf, p.budget_ns)) {
+                dead = true;
+                break;
+            }
+            if (t + 2 < n) fetch(t + 2);  // into the buffers of pair t - 1
+            store_half_row(sm.e[0], r, h, pk);
+            fence_proxy_async_smem();
+            warp_arrive(smem_u32(&sm.full_a));
+        }
+        if (!dead && n > 0 && !warp_wait(smem_u32(&sm.bar_a), (n - 1) & 1, abortf, p.budget_ns)) dead = true;
+    } else if (threadIdx.x == kIssuer && n > 0) {
+        // S_0, dP_0; then per pair t: S_{t+1}, dP_{t+1} once S_t, dP_t are in registers, and
+        // dQ += dS_t K_t once dS_t is stored
+        if (mbar_wait(smem_u32(&sm.full_s), 0, abortf, p.budget_ns)) {
+            tc_fence_after();
+            mma_kk(tb0 + kColS, smem_u32(sm.a), smem_u32(sm.x[0]));   // S = Q K^T
+            mma_kk(tb0 + kColDP, smem_u32(sm.b), smem_u32(sm.y[0]));  // dP = dO V^T
+            mma_commit(smem_u32(&sm.bar_s));
+            issued = 1;
+            for (int t = 0; t < n; ++t) {
+                if (!mbar_wait(smem_u32(&sm.full_s), (t + 1) & 1, abortf, p.budget_ns)) {
+                    dead = true;
+                    break;
+                }
+                tc_fence_after();
+                if (t + 1 < n) {
+                    mma_kk(tb0 + kColS, smem_u32(sm.a), smem_u32(sm.x[(t + 1) % 3]));
+                    mma_kk(tb0 + kColDP, smem_u32(sm.b), smem_u32(sm.y[(t + 1) % 3]));
+                    mma_commit(smem_u32(&sm.bar_s));
+                }
+                if (!mbar_wait(smem_u32(&sm.full_a), t & 1, abortf, p.budget_ns)) {
+                    dead = true;
+                    break;
+                }
+                tc_fence_after();
+                mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.x[t % 3]), t > 0);  // dQ += dS K
+                mma_commit(smem_u32(&sm.bar_a));
+            }
+        } else {
+            dead = true;
         }
     }
-    if (!dead && n > 0) {
-        const bool ok = mbar_wait(smem_u32(&sm.bar_a), (n - 1) & 1, abortf, p.budget_ns);
-        dead = __syncthreads_or(!ok);
-    }
-    if (!dead) {
+    dead = __syncthreads_or(dead);
+    if (!dead && threadIdx.x < kCompute) {
         tc_fence_after();
         if (n > 0) {
             store_acc(tb + kColA0, p.dQ + head, g, label, p.scale);
@@ -340,16 +404,16 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dkdv_tc_kernel(const BwdPar
     const Grid g = p.g;
     const int Tb = g.Tb(), N = g.H * g.W;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = lane >> 4;
+    const int r = (warp & 3) * 16 + (lane & 15);  // tile row of a compute thread
     const size_t head = (size_t)bh * N * kD;
     volatile int* abortf = &sm.abort_flag;
-    setup(sm);
-    const uint32_t tb = sm.tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
-    const uint32_t tb0 = sm.tmem_base;
-    const float c = p.scale * 1.4426950408889634f;
+    const float c = p.scale * kLog2e;
 
-    load_tile(smem_u32(sm.a), p.K + head, g, label);
-    load_tile(smem_u32(sm.b), p.V + head, g, label);
-    cp_async_commit();
+    if (threadIdx.x < kCompute) {
+        load_tile(smem_u32(sm.a), p.K + head, g, label);
+        load_tile(smem_u32(sm.b), p.V + head, g, label);
+        cp_async_commit();
+    }
 
     // the query blocks whose lists hold this key block, ascending
     int total = 0;
@@ -377,97 +441,114 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dkdv_tc_kernel(const BwdPar
         if (has) sm.list[off + __popc(b & ((1u << lane) - 1u))] = i;
         for (int w = 0; w < kThreads / 32; ++w) total += sm.wcount[w];
     }
-    __syncthreads();
     const int n = total;
-
-    auto prefetch = [&](int t, int buf) {
-        const int qi = sm.list[t];
-        load_tile(smem_u32(sm.x[buf]), p.Q + head, g, qi);
-        load_tile(smem_u32(sm.y[buf]), p.dO + head, g, qi);
-        if (threadIdx.x < kT) {
-            const size_t qrow = (size_t)bh * N + win_token(g, win_origin(g, qi), threadIdx.x);
-            sm.ls[buf][threadIdx.x] = __ldg(p.lse + qrow) * 1.4426950408889634f;
-            sm.ds[buf][threadIdx.x] = p.Dbuf[qrow];
-        }
-        cp_async_commit();
-    };
-    if (n > 0) prefetch(0, 0);
+    setup(sm);  // its barrier also publishes the list
+    const uint32_t tb = sm.tmem_base + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    const uint32_t tb0 = sm.tmem_base;
     bool dead = false;
     uint32_t issued = 0;
-    for (int t = 0; t < n && !dead; ++t) {
-        const int buf = t & 1;
-        // pair t-1's products have read P^T, dS^T (TMEM over S^T, dP^T) and the other buffers
-        if (t >= 1) {
-            const bool ok = mbar_wait(smem_u32(&sm.bar_a), (t - 1) & 1, abortf, p.budget_ns);
-            if (__syncthreads_or(!ok)) {
+
+    if (threadIdx.x < kCompute) {
+        // tiles of pair t in buffer t % 3: Q_i in x, dO_i in y, and the block's lse and D
+        auto fetch = [&](int t) {
+            const int qi = sm.list[t], buf = t % 3;
+            load_tile(smem_u32(sm.x[buf]), p.Q + head, g, qi);
+            load_tile(smem_u32(sm.y[buf]), p.dO + head, g, qi);
+            if (threadIdx.x < kT) {
+                const size_t qrow = (size_t)bh * N + win_token(g, win_origin(g, qi), threadIdx.x);
+                cp_async4(smem_u32(&sm.ls[buf][threadIdx.x]), p.lse + qrow);
+                cp_async4(smem_u32(&sm.ds[buf][threadIdx.x]), p.Dbuf + qrow);
+            }
+            cp_async_commit();
+        };
+        if (n > 0) fetch(0);
+        if (n > 1) fetch(1);
+        if (n > 0) {  // K, V and the tiles of pair 0 landed
+            if (n > 1) cp_async_wait<1>(); else cp_async_wait<0>();
+            fence_proxy_async_smem();
+            warp_arrive(smem_u32(&sm.full_s));
+        }
+        // Pair t as in the dQ kernel, with P^T_t and dS^T_t as the stored operands.
+        for (int t = 0; t < n; ++t) {
+            const int buf = t % 3;
+            if (!warp_wait(smem_u32(&sm.bar_s), t & 1, abortf, p.budget_ns)) {
                 dead = true;
                 break;
             }
-        }
-        if (t + 1 < n) {
-            prefetch(t + 1, buf ^ 1);
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
-        }
-        fence_proxy_async_smem();
-        __syncthreads();
-        if (threadIdx.x == 0) {
             tc_fence_after();
-            mma_kk(tb0 + kColS, smem_u32(sm.a), smem_u32(sm.x[buf]));   // S^T = K Q^T
-            mma_kk(tb0 + kColDP, smem_u32(sm.b), smem_u32(sm.y[buf]));  // dP^T = V dO^T
-            mma_commit(smem_u32(&sm.bar_s));
-        }
-        issued = 1;
-        {
-            const bool ok = mbar_wait(smem_u32(&sm.bar_s), t & 1, abortf, p.budget_ns);
-            if (__syncthreads_or(!ok)) {
-                dead = true;
-                break;
+            uint32_t s[32], dp[32];
+            tmem_ld_16x32bx2_x16_off32(tb + kColS, *reinterpret_cast<uint32_t(*)[16]>(&s[0]));
+            tmem_ld_16x32bx2_x16_off32(tb + kColS + 16, *reinterpret_cast<uint32_t(*)[16]>(&s[16]));
+            tmem_ld_16x32bx2_x16_off32(tb + kColDP, *reinterpret_cast<uint32_t(*)[16]>(&dp[0]));
+            tmem_ld_16x32bx2_x16_off32(tb + kColDP + 16, *reinterpret_cast<uint32_t(*)[16]>(&dp[16]));
+            tmem_wait_ld();
+            tc_fence_before();
+            if (t + 1 < n) {
+                cp_async_wait<0>();
+                fence_proxy_async_smem();
             }
-        }
-        tc_fence_after();
-        uint32_t s[32], dp[32];
-        tmem_ld_16x32bx2_x16_off32(tb + kColS, *reinterpret_cast<uint32_t(*)[16]>(&s[0]));
-        tmem_ld_16x32bx2_x16_off32(tb + kColS + 16, *reinterpret_cast<uint32_t(*)[16]>(&s[16]));
-        tmem_ld_16x32bx2_x16_off32(tb + kColDP, *reinterpret_cast<uint32_t(*)[16]>(&dp[0]));
-        tmem_ld_16x32bx2_x16_off32(tb + kColDP + 16, *reinterpret_cast<uint32_t(*)[16]>(&dp[16]));
-        tmem_wait_ld();
-        // columns are the query rows 32 h + i of the block
-        const float* Lq = sm.ls[buf] + 32 * h;
-        const float* Dq = sm.ds[buf] + 32 * h;
-        uint32_t pp[16], dd[16];
+            warp_arrive(smem_u32(&sm.full_s));
+            // columns are the query rows 32 h + i of the block
+            const float* Lq = sm.ls[buf] + 32 * h;
+            const float* Dq = sm.ds[buf] + 32 * h;
+            uint32_t pp[16], dd[16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            const float p0 = fast_exp2(fmaf(__uint_as_float(s[2 * i]), c, -Lq[2 * i]));
-            const float p1 = fast_exp2(fmaf(__uint_as_float(s[2 * i + 1]), c, -Lq[2 * i + 1]));
-            pp[i] = pack_bf16(p0, p1);
-            dd[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - Dq[2 * i]),
-                              p1 * (__uint_as_float(dp[2 * i + 1]) - Dq[2 * i + 1]));
+            for (int i = 0; i < 16; ++i) {
+                const float p0 = fast_exp2(fmaf(__uint_as_float(s[2 * i]), c, -Lq[2 * i] * kLog2e));
+                const float p1 = fast_exp2(fmaf(__uint_as_float(s[2 * i + 1]), c, -Lq[2 * i + 1] * kLog2e));
+                pp[i] = pack_bf16(p0, p1);
+                dd[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - Dq[2 * i]),
+                                  p1 * (__uint_as_float(dp[2 * i + 1]) - Dq[2 * i + 1]));
+            }
+            if (t >= 1 && !warp_wait(smem_u32(&sm.bar_a), (t - 1) & 1, abortf, p.budget_ns)) {
+                dead = true;
+                break;
+            }
+            if (t + 2 < n) fetch(t + 2);  // into the buffers of pair t - 1
+            store_half_row(sm.e[0], r, h, pp);
+            store_half_row(sm.e[1], r, h, dd);
+            fence_proxy_async_smem();
+            warp_arrive(smem_u32(&sm.full_a));
         }
-        tmem_st_16x32bx2_x16_off16(tb + kColS, pp);   // P^T over S^T
-        tmem_st_16x32bx2_x16_off16(tb + kColDP, dd);  // dS^T over dP^T
-        tmem_wait_st();
-        tc_fence_before();
-        __syncthreads();
-        if (threadIdx.x == 0) {
+        if (!dead && n > 0 && !warp_wait(smem_u32(&sm.bar_a), (n - 1) & 1, abortf, p.budget_ns)) dead = true;
+    } else if (threadIdx.x == kIssuer && n > 0) {
+        if (mbar_wait(smem_u32(&sm.full_s), 0, abortf, p.budget_ns)) {
             tc_fence_after();
-            mma_tb(tb0 + kColA0, tb0 + kColS, smem_u32(sm.y[buf]), t > 0);   // dV += P^T dO
-            mma_tb(tb0 + kColA1, tb0 + kColDP, smem_u32(sm.x[buf]), t > 0);  // dK += dS^T Q
-            mma_commit(smem_u32(&sm.bar_a));
+            mma_kk(tb0 + kColS, smem_u32(sm.a), smem_u32(sm.x[0]));   // S^T = K Q^T
+            mma_kk(tb0 + kColDP, smem_u32(sm.b), smem_u32(sm.y[0]));  // dP^T = V dO^T
+            mma_commit(smem_u32(&sm.bar_s));
+            issued = 1;
+            for (int t = 0; t < n; ++t) {
+                if (!mbar_wait(smem_u32(&sm.full_s), (t + 1) & 1, abortf, p.budget_ns)) {
+                    dead = true;
+                    break;
+                }
+                tc_fence_after();
+                if (t + 1 < n) {
+                    mma_kk(tb0 + kColS, smem_u32(sm.a), smem_u32(sm.x[(t + 1) % 3]));
+                    mma_kk(tb0 + kColDP, smem_u32(sm.b), smem_u32(sm.y[(t + 1) % 3]));
+                    mma_commit(smem_u32(&sm.bar_s));
+                }
+                if (!mbar_wait(smem_u32(&sm.full_a), t & 1, abortf, p.budget_ns)) {
+                    dead = true;
+                    break;
+                }
+                tc_fence_after();
+                mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.y[t % 3]), t > 0);  // dV += P^T dO
+                mma_sb(tb0 + kColA1, smem_u32(sm.e[1]), smem_u32(sm.x[t % 3]), t > 0);  // dK += dS^T Q
+                mma_commit(smem_u32(&sm.bar_a));
+            }
+        } else {
+            dead = true;
         }
     }
-    if (!dead && n > 0) {
-        const bool ok = mbar_wait(smem_u32(&sm.bar_a), (n - 1) & 1, abortf, p.budget_ns);
-        dead = __syncthreads_or(!ok);
-    }
-    if (!dead) {
+    dead = __syncthreads_or(dead);
+    if (!dead && threadIdx.x < kCompute) {
         tc_fence_after();
         if (n > 0) {
             store_acc(tb + kColA0, p.dV + head, g, label, 1.0f);
             store_acc(tb + kColA1, p.dK + head, g, label, p.scale);
         } else {
-            const int r = warp * 16 + (lane & 15);
             const size_t krow = (size_t)bh * N + g.token(label, r);
             float4* a = reinterpret_cast<float4*>(p.dV + krow * kD + 32 * h);
             float4* b = reinterpret_cast<float4*>(p.dK + krow * kD + 32 * h);

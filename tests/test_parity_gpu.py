@@ -381,7 +381,11 @@ def test_backward_fp32_tiny(shift, rho):
 
 
 @pytest.mark.parametrize("H,W,h,rho,shift", [(32, 32, 4, 0.75, (4, 4)), (64, 64, 4, 0.8416, (4, 4)),
-                                            (24, 40, 3, 0.6, (4, -4))])
+                                            (24, 40, 3, 0.6, (4, -4)),
+                                            # one, two and three kept blocks a row: the pipelined
+                                            # loops with fewer pairs than tile buffers
+                                            (16, 16, 4, 0.75, (4, 4)), (16, 16, 4, 0.5, (3, -5)),
+                                            (16, 24, 2, 0.5, (0, 0))])
 def test_backward_bf16(H, W, h, rho, shift):
     _bwd_case_gpu(1, h, H, W, rho, shift, torch.bfloat16, 31)
 
