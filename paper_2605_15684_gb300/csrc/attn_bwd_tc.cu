@@ -4,18 +4,19 @@
 // For the output gradient dO, with p_nm = exp(scale q_n.k_m - lse_n) over the kept pairs:
 //   D_n = dO_n . O_n,  ds_nm = p_nm (dO_n . v_m - D_n),
 //   dQ_n = scale sum_m ds_nm k_m,  dK_m = scale sum_n ds_nm q_n,  dV_m = sum_n p_nm dO_n.
-// Two kernels, as the CUDA-core version, deterministic (no atomics), one (batch*head, block)
-// per CTA, each 64 x 64 tile product a tcgen05.mma kind::f16 with M=64 (four K=16 steps).
+// Deterministic (no atomics). A row kernel writes D for every row; then one grid holds both
+// gradient roles, one (batch*head, block) per CTA, launched as a programmatic dependent of the
+// row kernel (only the key-block role waits for D). Each 64 x 64 tile product is a
+// tcgen05.mma kind::f16 with M=64 (four K=16 steps).
 // 160 threads: warps 0-3 own the TMEM lane quadrants (the exps, the bf16 operands, the tile
 // copies, the epilogue); lane 0 of warp 4 issues every MMA, so that issuing (some 80 cycles
 // an instruction) runs beside the compute warps instead of in front of them. The two sides
 // meet on mbarriers: MMA commits one way, one arrive per compute warp the other.
-//   ssba_bwd_dq_tc_kernel    query block i: for each kept key block j (list order)
+//   dq_block     query block i: for each kept key block j (list order)
 //                              S  = Q_i K_j^T,  dP = dO_i V_j^T        (A, B from shared memory)
 //                              dS = P o (dP - D) in registers, bf16 into shared memory
 //                              dQ += dS K_j                           (B read MN-major)
-//                            and writes D for the second kernel.
-//   ssba_bwd_dkdv_tc_kernel  key block j: for each query block i whose list holds j (ascending)
+//   dkdv_block   key block j: for each query block i whose list holds j (ascending)
 //                              S^T = K_j Q_i^T,  dP^T = V_j dO_i^T
 //                              P^T, dS^T in registers, bf16 into shared memory
 //                              dV += P^T dO_i,  dK += dS^T Q_i
@@ -250,10 +251,11 @@ __device__ __forceinline__ void store_acc(uint32_t taddr, float* out, const Grid
                              __uint_as_float(v[4 * i + 2]) * mul, __uint_as_float(v[4 * i + 3]) * mul);
 }
 
-__global__ void __launch_bounds__(kThreads) ssba_bwd_dq_tc_kernel(const BwdParams p)
+// dQ of query block `label` of head bh (D comes from the row kernel; computed here again
+// for this block's own rows, so that this role needs nothing from that kernel).
+__device__ __forceinline__ void dq_block(const BwdParams& p, const int label, const int bh)
 {
     BwdSmem& sm = smem_layout();
-    const int label = blockIdx.x, bh = blockIdx.y;
     const Grid g = p.g;
     const int Tb = g.Tb(), N = g.H * g.W;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = lane >> 4;
@@ -305,7 +307,6 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dq_tc_kernel(const BwdParam
             }
         }
         Dr += __shfl_xor_sync(0xffffffffu, Dr, 16);
-        if (h == 0) p.Dbuf[row] = Dr;
         const float c = p.scale * kLog2e;
         const float L2 = p.lse[row] * kLog2e;
         if (n > 0) {  // Q, dO and the tiles of pair 0 landed
@@ -397,10 +398,10 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dq_tc_kernel(const BwdParam
     teardown(sm, p, dead, issued);
 }
 
-__global__ void __launch_bounds__(kThreads) ssba_bwd_dkdv_tc_kernel(const BwdParams p)
+// dK, dV of key block `label` of head bh.
+__device__ __forceinline__ void dkdv_block(const BwdParams& p, const int label, const int bh)
 {
     BwdSmem& sm = smem_layout();
-    const int label = blockIdx.x, bh = blockIdx.y;
     const Grid g = p.g;
     const int Tb = g.Tb(), N = g.H * g.W;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = lane >> 4;
@@ -461,6 +462,7 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dkdv_tc_kernel(const BwdPar
             }
             cp_async_commit();
         };
+        grid_dep_wait();  // D of every row, from the row kernel
         if (n > 0) fetch(0);
         if (n > 1) fetch(1);
         if (n > 0) {  // K, V and the tiles of pair 0 landed
@@ -562,6 +564,48 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_dkdv_tc_kernel(const BwdPar
     teardown(sm, p, dead, issued);
 }
 
+// D_n = dO_n . O_n for every row, two threads a row (32 dims each).
+__global__ void __launch_bounds__(256) ssba_bwd_rows_kernel(const BwdParams p, const int rows)
+{
+    grid_dep_launch();  // the gradient kernel's prologues need nothing from here
+    const int t = blockIdx.x * 256 + threadIdx.x;
+    const int row = t >> 1, h = t & 1;
+    float Dr = 0.f;
+    if (row < rows) {
+        const uint4* go = reinterpret_cast<const uint4*>(p.dO + (size_t)row * kD + 32 * h);
+        const uint4* oo = reinterpret_cast<const uint4*>(p.O + (size_t)row * kD + 32 * h);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint4 a = __ldg(go + i), b = __ldg(oo + i);
+            const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 fa = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&aw[k]));
+                const float2 fb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&bw[k]));
+                Dr = fmaf(fa.x, fb.x, Dr);
+                Dr = fmaf(fa.y, fb.y, Dr);
+            }
+        }
+    }
+    Dr += __shfl_xor_sync(0xffffffffu, Dr, 1);
+    if (row < rows && h == 0) p.Dbuf[row] = Dr;
+}
+
+// Both gradient roles in one grid: CTAs [0, BH Tb) are key blocks (dK, dV; their list lengths
+// vary), the rest query blocks (dQ; all the same length), so that the query blocks fill in
+// behind the key blocks instead of ending in a partial wave of their own.
+__global__ void __launch_bounds__(kThreads) ssba_bwd_tc_kernel(const BwdParams p)
+{
+    const int Tb = p.g.Tb();
+    const int nk = (int)(gridDim.x >> 1);
+    const int item = blockIdx.x < nk ? blockIdx.x : blockIdx.x - nk;
+    const int bh = item / Tb, label = item - bh * Tb;
+    if ((int)blockIdx.x < nk)
+        dkdv_block(p, label, bh);
+    else
+        dq_block(p, label, bh);
+}
+
 }  // namespace
 
 int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
@@ -591,17 +635,27 @@ int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale,
         set_error("ssba_backward: could not resolve the device status word");
         return SSBA_ERR_CUDA;
     }
-    static PerDeviceOnce attr;  // shared-memory attributes, set once per device
+    static PerDeviceOnce attr;  // shared-memory attribute, set once per device
     attr.run([] {
-        cudaFuncSetAttribute(ssba_bwd_dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
-        cudaFuncSetAttribute(ssba_bwd_dkdv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        cudaFuncSetAttribute(ssba_bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     });
-    dim3 grid(g.Tb(), d.B * d.heads);
-    ssba_bwd_dq_tc_kernel<<<grid, kThreads, kSmemBytes, st>>>(p);
+    const int BH = d.B * d.heads, rows = BH * g.H * g.W;
+    ssba_bwd_rows_kernel<<<(unsigned)((2 * (size_t)rows + 255) / 256), 256, 0, st>>>(p, rows);
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess) {
-        ssba_bwd_dkdv_tc_kernel<<<grid, kThreads, kSmemBytes, st>>>(p);
-        e = cudaGetLastError();
+        // launched as a programmatic dependent of the row kernel: only the key-block role waits
+        // for it (grid_dep_wait before it reads D)
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)(2 * BH * g.Tb()));
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = kSmemBytes;
+        cfg.stream = st;
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        at[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, ssba_bwd_tc_kernel, p);
     }
     if (e != cudaSuccess) {
         set_error("ssba_backward (tensor cores) launch: %s", cudaGetErrorString(e));
