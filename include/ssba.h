@@ -179,7 +179,8 @@ SSBA_API int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void
  *   kv_idx, kv_cnt  the lists of the forward.
  *   dQ, dK, dV      device out, fp32 [B][heads][N][head_dim], every element written.
  *   workspace       device scratch of at least ssba_backward_workspace_bytes(desc) bytes
- *                   (the D_n values), 16-byte aligned.
+ *                   (the D_n values and the key blocks' transposed lists), 16-byte aligned,
+ *                   one per stream (a call's kernels read what its own first kernel wrote).
  * bf16 inputs with head_dim = 64, 8x8 blocks and Tb <= 256 run on the tensor cores (tcgen05
  * products of 64-row tiles with fp32 accumulation in tensor memory; P and dS rounded to bf16
  * before their products, as the forward rounds P); fp32 inputs, and other shapes, on CUDA cores
@@ -189,7 +190,10 @@ SSBA_API int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, 
                            const float* lse, const void* dO, const int32_t* kv_idx, const int32_t* kv_cnt,
                            float* dQ, float* dK, float* dV, void* workspace, size_t ws_bytes, void* stream);
 
-/* Bytes of the ssba_backward workspace: B * heads * N * 4 (0 for an invalid descriptor). */
+/* Bytes of the ssba_backward workspace (0 for an invalid descriptor): D of every row
+ * (B * heads * N * 4, rounded up to 256), then 256 bytes for a work counter and the transposed
+ * lists, three int arrays of B * heads * Tb, B * heads * Tb and B * heads * Tb * keep entries
+ * (each rounded up to 256 bytes). Every part is rewritten by each call: no zero-fill needed. */
 SSBA_API size_t ssba_backward_workspace_bytes(const ssba_desc* desc);
 
 /* Block compression alone (Sec. 2.2, the means q_b, k_b; Algorithm 1 MeanPool): the first

@@ -6,11 +6,48 @@
 #include <cstdio>
 #include <cstring>
 
+#include "bwd_tile.cuh"
 #include "common.cuh"
+#include "window.cuh"
 
 namespace ssba {
 
 __device__ int g_status = 0;
+
+EncodeTiledFn tensor_map_encoder()
+{
+    static EncodeTiledFn fn = [] {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            cudaGetLastError();
+            return static_cast<EncodeTiledFn>(nullptr);
+        }
+        return reinterpret_cast<EncodeTiledFn>(ptr);
+    }();
+    return fn;
+}
+
+bool encode_window_maps(CUtensorMap* m4, const void* base, int BH, int H, int W)
+{
+    EncodeTiledFn fn = tensor_map_encoder();
+    if (!fn) return false;
+    constexpr cuuint64_t d = 64;
+    const cuuint32_t cols[4] = {8, 8, 4, 4}, rows[4] = {8, 4, 8, 4};
+    for (int s = 0; s < 4; ++s) {
+        cuuint64_t dims[4] = {d, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)BH};
+        cuuint64_t strides[3] = {d * 2, (cuuint64_t)W * d * 2, (cuuint64_t)H * W * d * 2};
+        cuuint32_t box[4] = {(cuuint32_t)d, cols[s], rows[s], 1};
+        cuuint32_t es[4] = {1, 1, 1, 1};
+        CUresult r = fn(&m4[s], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return false;
+    }
+    return true;
+}
 
 int current_device()
 {
@@ -486,7 +523,7 @@ size_t ssba_backward_workspace_bytes(const ssba_desc* desc)
     Grid g;
     int keep;
     if (check_desc(desc, "ssba_backward_workspace_bytes", &g, &keep) != SSBA_OK) return 0;
-    return (size_t)desc->B * desc->heads * desc->H_tok * desc->W_tok * sizeof(float);
+    return bwd::bwd_layout(*desc, g, keep).bytes;
 }
 
 int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, const void* V, const void* O, const float* lse,

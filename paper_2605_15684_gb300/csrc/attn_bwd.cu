@@ -211,7 +211,9 @@ int launch_backward(const ssba_desc& d, const Grid& g, int keep, float scale, co
         return SSBA_ERR_UNSUPPORTED;
     }
     if (d.dtype == SSBA_BF16) {
-        const int rc = launch_backward_tc(d, g, keep, scale, Q, K, V, O, lse, dO, idx, cnt, dQ, dK, dV, Dbuf, st);
+        int rc = launch_backward_ws(d, g, keep, scale, Q, K, V, O, lse, dO, idx, cnt, dQ, dK, dV, Dbuf, st);
+        if (rc != SSBA_ERR_UNSUPPORTED) return rc;
+        rc = launch_backward_tc(d, g, keep, scale, Q, K, V, O, lse, dO, idx, cnt, dQ, dK, dV, Dbuf, st);
         if (rc != SSBA_ERR_UNSUPPORTED) return rc;
         return launch_bwd_t<__nv_bfloat16>(d, g, keep, scale, Q, K, V, O, lse, dO, idx, cnt, dQ, dK, dV, Dbuf, st);
     }

@@ -33,6 +33,7 @@
 #include <cstdint>
 
 #include "common.cuh"
+#include "bwd_tile.cuh"
 #include "ptx.cuh"
 
 namespace ssba {
@@ -41,17 +42,13 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kD = 64;
-constexpr int kT = 64;                   // tokens per block
+using namespace bwd;
+
 constexpr int kCompute = 128;  // warps 0-3: one TMEM lane quadrant each
 constexpr int kThreads = 160;  // + warp 4, whose lane 0 issues every MMA of the CTA
 constexpr int kIssuer = 128;
-constexpr uint32_t kTile = kT * kD * 2;  // 8 KB
 constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kColS = 0, kColDP = 64, kColA0 = 128, kColA1 = 192;
-constexpr uint32_t kIdescK = idesc_bf16_f32(64, 64, false, false);  // A, B K-major
-constexpr uint32_t kIdescMN = idesc_bf16_f32(64, 64, false, true);  // B MN-major
-constexpr float kLog2e = 1.4426950408889634f;
 constexpr size_t kSmemBytes = 100 * 1024;  // also keeps residency at two CTAs per SM (TMEM)
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src)
@@ -100,49 +97,6 @@ __device__ __forceinline__ void load_tile(uint32_t dst, const __nv_bfloat16* X, 
     }
 }
 
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
-{
-    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t*>(&v);
-}
-
-__device__ __forceinline__ float fast_exp2(float x)
-{
-    float y;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-    return y;
-}
-
-// C (64 x 64, fp32 TMEM at column `col`) = A B^T with A, B K-major 64 x 64 tiles in shared memory.
-__device__ __forceinline__ void mma_kk(uint32_t col, uint32_t a, uint32_t b)
-{
-    const uint64_t ad = sdesc_sw128(a, 16, 1024), bd = sdesc_sw128(b, 16, 1024);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) mma_ss(col, ad + (uint64_t)(k * 2), bd + (uint64_t)(k * 2), kIdescK, k > 0 ? 1u : 0u);
-}
-
-// C (+)= A B with A (64 x 64 bf16) a K-major shared tile and B a shared tile read MN-major
-// (rows = the contraction index).
-__device__ __forceinline__ void mma_sb(uint32_t col, uint32_t a, uint32_t b, bool accumulate)
-{
-    const uint64_t ad = sdesc_sw128(a, 16, 1024), bd = sdesc_sw128(b, 8192, 1024);
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        mma_ss(col, ad + (uint64_t)(k * 2), bd + (uint64_t)(k * 128), kIdescMN, (accumulate || k > 0) ? 1u : 0u);
-}
-
-// This thread's half row (row r of the M=64 data path, columns [32 h, 32 h + 32)) of a 64 x 64
-// bf16 tile, 16 packed pairs, into the 128-byte-swizzled K-major layout at dst.
-__device__ __forceinline__ void store_half_row(uint8_t* dst, int r, int h, const uint32_t (&v)[16])
-{
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int c = 4 * h + i;
-        *reinterpret_cast<uint4*>(dst + r * 128 + ((c ^ (r & 7)) << 4)) =
-            make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-    }
-}
-
 struct alignas(1024) BwdSmem {
     uint8_t a[kTile];        // dq: Q_i;  dkdv: K_j
     uint8_t b[kTile];        // dq: dO_i; dkdv: V_j
@@ -161,19 +115,6 @@ struct alignas(1024) BwdSmem {
     int abort_flag;
 };
 static_assert(sizeof(BwdSmem) + 1024 <= kSmemBytes, "shared memory");
-
-struct BwdParams {
-    const __nv_bfloat16 *Q, *K, *V, *O, *dO;
-    const float* lse;
-    const int32_t* idx;
-    const int32_t* cnt;
-    float *dQ, *dK, *dV, *Dbuf;
-    Grid g;
-    int keep;
-    float scale;
-    int* status;
-    uint64_t budget_ns;
-};
 
 __device__ __forceinline__ BwdSmem& smem_layout()
 {
@@ -564,10 +505,67 @@ __device__ __forceinline__ void dkdv_block(const BwdParams& p, const int label, 
     teardown(sm, p, dead, issued);
 }
 
-// D_n = dO_n . O_n for every row, two threads a row (32 dims each).
-__global__ void __launch_bounds__(256) ssba_bwd_rows_kernel(const BwdParams p, const int rows)
+// Head bh's transposed lists (see BwdParams): a bit per (key block j, query block i) in shared
+// memory, then per key block its count, an exclusive scan over the key blocks, and its query
+// blocks written in ascending order. Thread j owns key block j (Tb <= 256 = the block size).
+__device__ __forceinline__ void build_transposed(const BwdParams& p, const int bh)
+{
+    __shared__ uint32_t bits[256 * 8];  // [j][i / 32]
+    __shared__ int wsum[8];
+    const int Tb = p.g.Tb(), nw = (Tb + 31) >> 5;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int w = threadIdx.x; w < Tb * nw; w += 256) bits[w] = 0;
+    if (bh == 0 && threadIdx.x == 0) *p.ctr = 0;  // read by the gradient kernel after its wait
+    __syncthreads();
+    const int32_t* idx = p.idx + (size_t)bh * Tb * p.keep;
+    const int32_t* cnt = p.cnt + (size_t)bh * Tb;
+    for (int e = threadIdx.x; e < Tb * p.keep; e += 256) {
+        const int i = e / p.keep, t = e - i * p.keep;
+        if (t < min(max(__ldg(cnt + i), 0), p.keep)) {
+            const int j = min(max(__ldg(idx + e), 0), Tb - 1);
+            atomicOr(&bits[j * nw + (i >> 5)], 1u << (i & 31));
+        }
+    }
+    __syncthreads();
+    const int j = threadIdx.x;
+    int c = 0;
+    if (j < Tb)
+        for (int w = 0; w < nw; ++w) c += __popc(bits[j * nw + w]);
+    int v = c;  // inclusive scan within the warp, then over the warps
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += u;
+    }
+    if (lane == 31) wsum[warp] = v;
+    __syncthreads();
+    int off = v - c;
+    for (int w = 0; w < warp; ++w) off += wsum[w];
+    if (j < Tb) {
+        const size_t row = (size_t)bh * Tb + j;
+        p.toff[row] = (int)((size_t)bh * Tb * p.keep) + off;
+        p.tcnt[row] = c;
+        int* out = p.tlist + (size_t)bh * Tb * p.keep + off;
+        for (int w = 0; w < nw; ++w) {
+            uint32_t m = bits[j * nw + w];
+            while (m) {
+                const int b = __ffs(m) - 1;
+                m &= m - 1;
+                *out++ = w * 32 + b;
+            }
+        }
+    }
+}
+
+// D_n = dO_n . O_n for every row, two threads a row (32 dims each); CTAs past row_blocks
+// build the transposed lists, one head each.
+__global__ void __launch_bounds__(256) ssba_bwd_rows_kernel(const BwdParams p, const int rows, const int row_blocks)
 {
     grid_dep_launch();  // the gradient kernel's prologues need nothing from here
+    if ((int)blockIdx.x >= row_blocks) {
+        build_transposed(p, (int)blockIdx.x - row_blocks);
+        return;
+    }
     const int t = blockIdx.x * 256 + threadIdx.x;
     const int row = t >> 1, h = t & 1;
     float Dr = 0.f;
@@ -608,6 +606,32 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_tc_kernel(const BwdParams p
 
 }  // namespace
 
+namespace bwd {
+
+BwdLayout bwd_layout(const ssba_desc& d, const Grid& g, int keep)
+{
+    auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
+    const size_t BH = (size_t)d.B * d.heads, Tb = (size_t)g.Tb();
+    BwdLayout l;
+    l.ctr = up(BH * g.H * g.W * sizeof(float));
+    l.toff = l.ctr + 256;
+    l.tcnt = l.toff + up(BH * Tb * sizeof(int));
+    l.tlist = l.tcnt + up(BH * Tb * sizeof(int));
+    l.bytes = l.tlist + up(BH * Tb * (size_t)keep * sizeof(int));
+    return l;
+}
+
+cudaError_t launch_bwd_rows(const BwdParams& p, int BH, cudaStream_t st)
+{
+    const int rows = BH * p.g.H * p.g.W;
+    const int row_blocks = (int)((2 * (size_t)rows + 255) / 256);
+    const int extra = p.tlist ? BH : 0;
+    ssba_bwd_rows_kernel<<<(unsigned)(row_blocks + extra), 256, 0, st>>>(p, rows, row_blocks);
+    return cudaGetLastError();
+}
+
+}  // namespace bwd
+
 int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
                        const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
                        const int32_t* cnt, float* dQ, float* dK, float* dV, float* Dbuf, cudaStream_t st)
@@ -626,6 +650,7 @@ int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale,
     p.dK = dK;
     p.dV = dV;
     p.Dbuf = Dbuf;
+    p.ctr = p.toff = p.tcnt = p.tlist = nullptr;
     p.g = g;
     p.keep = keep;
     p.scale = scale;
@@ -639,9 +664,8 @@ int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale,
     attr.run([] {
         cudaFuncSetAttribute(ssba_bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     });
-    const int BH = d.B * d.heads, rows = BH * g.H * g.W;
-    ssba_bwd_rows_kernel<<<(unsigned)((2 * (size_t)rows + 255) / 256), 256, 0, st>>>(p, rows);
-    cudaError_t e = cudaGetLastError();
+    const int BH = d.B * d.heads;
+    cudaError_t e = launch_bwd_rows(p, BH, st);
     if (e == cudaSuccess) {
         // launched as a programmatic dependent of the row kernel: only the key-block role waits
         // for it (grid_dep_wait before it reads D)

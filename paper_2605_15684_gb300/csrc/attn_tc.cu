@@ -50,12 +50,14 @@
 #include "common.cuh"
 #include "ptx.cuh"
 #include "select.cuh"
+#include "window.cuh"
 
 namespace ssba {
 
 namespace {
 
 using namespace ptx;
+using namespace win;
 
 constexpr int kD = 64;
 constexpr int kRows = 64;  // query rows per item = tokens per block
@@ -72,8 +74,6 @@ constexpr uint32_t kColS = 0;    // S buffers: [0,64), [64,128)
 constexpr uint32_t kColP = 128;  // P buffers: [128,160), [160,192)
 constexpr uint32_t kColO = 192;  // O accumulator: [192,256)
 constexpr uint32_t kTileBytes = kRows * kD * 2;  // 8 KB
-// Tensor-map box shapes (d x cols x rows) used to cut a shifted 8x8 window out of the grid.
-enum BoxShape { kBox8x8 = 0, kBox8c4r = 1, kBox4c8r = 2, kBox4x4 = 3 };
 constexpr float kRescaleLog2 = 8.0f;
 constexpr int kLabelCap = 128;  // labels staged per producer warp and piece; the rest are read per block
 constexpr int kCntCap = 64;     // phase-B item counts of a pipeline held in shared memory
@@ -461,74 +461,6 @@ __device__ __noinline__ void select_item(const TcParams& p, int item, int lane, 
     if (stamp) TL_CTA(tl::kWalkDone);
     if (lane == 0) p.sel_cnt[item] = p.keep;
     __syncwarp();
-}
-
-// Origin (row, col) of the shifted 8x8 window `label` in the unshifted grid. With block
-// 8 and a shift that is a multiple of 4, a window either fits (origin <= size - 8) or is
-// split 4 + 4 by the grid edge (origin = size - 4).
-__device__ __forceinline__ void window_origin(const Grid& g, int label, int& r0, int& c0)
-{
-    const int br = label / g.bw, bc = label - br * g.bw;
-    r0 = br * 8 - g.sr;
-    if (r0 < 0) r0 += g.H;
-    c0 = bc * 8 - g.sc;
-    if (c0 < 0) c0 += g.W;
-}
-
-// Window of `label` packed in one word: origin row r0 (bits 0-14), origin column c0 (bits
-// 15-29) and the box shape class (bits 30-31: 0 one 8x8 box, 1 split rows, 2 split columns,
-// 3 both). Tabulated per CTA at kernel start, so that the producers' per-copy work is a
-// shared-memory load and a switch (the producers' issue loop is on the critical path).
-__device__ __forceinline__ uint32_t window_entry(const Grid& g, int label)
-{
-    int r0, c0;
-    window_origin(g, label, r0, c0);
-    const uint32_t wr = r0 + 8 > g.H, wc = c0 + 8 > g.W;
-    return (uint32_t)r0 | ((uint32_t)c0 << 15) | ((wr | (wc << 1)) << 30);
-}
-
-// TMA copies of a window given its packed entry (see window_boxes).
-__device__ __forceinline__ void window_boxes_e(const CUtensorMap* m4, uint32_t dst, uint32_t bar, uint32_t e, int bh)
-{
-    const int r0 = e & 0x7fff, c0 = (e >> 15) & 0x7fff;
-    switch (e >> 30) {
-        case 0:
-            tma_load_4d(dst, &m4[kBox8x8], bar, 0, c0, r0, bh);
-            break;
-        case 1:
-            tma_load_4d(dst, &m4[kBox8c4r], bar, 0, c0, r0, bh);
-            tma_load_4d(dst + 4096, &m4[kBox8c4r], bar, 0, c0, 0, bh);
-            break;
-        case 2:
-            tma_load_4d(dst, &m4[kBox4c8r], bar, 0, c0, r0, bh);
-            tma_load_4d(dst + 4096, &m4[kBox4c8r], bar, 0, 0, r0, bh);
-            break;
-        default:
-            tma_load_4d(dst, &m4[kBox4x4], bar, 0, c0, r0, bh);
-            tma_load_4d(dst + 2048, &m4[kBox4x4], bar, 0, 0, r0, bh);
-            tma_load_4d(dst + 4096, &m4[kBox4x4], bar, 0, c0, 0, bh);
-            tma_load_4d(dst + 6144, &m4[kBox4x4], bar, 0, 0, 0, bh);
-            break;
-    }
-}
-
-// A window is one 8x8 box when it does not cross the grid edge, else two 8-col x 4-row boxes
-// (split rows), two 4-col x 8-row boxes (split columns) or four 4x4 boxes; the tile row
-// order is set by the shape class and decoded by tile_row_pos(); K and V of one label
-// always share it.
-// Tile row r of window `label` -> in-window position (row-major over the 8x8 window).
-__device__ __forceinline__ int tile_row_pos(const Grid& g, int label, int r)
-{
-    int r0, c0;
-    window_origin(g, label, r0, c0);
-    const bool wr = r0 + 8 > g.H, wc = c0 + 8 > g.W;
-    if (!wc) return r;  // 8-wide rows, row-major (one box or two row halves)
-    if (!wr) {          // two 8x4 column halves
-        const int h = r >> 5, a = (r >> 2) & 7, b = r & 3;
-        return a * 8 + 4 * h + b;
-    }
-    const int q = r >> 4, a = (r >> 2) & 3, b = r & 3;  // four 4x4 quadrants
-    return (4 * (q >> 1) + a) * 8 + 4 * (q & 1) + b;
 }
 
 // Piece k of pipeline v (V pipelines) from the schedule in shared memory.
@@ -1232,50 +1164,11 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
     if (threadIdx.x == 0) TL_CTA(tl::kEnd);
 }
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn get_encode_fn()
-{
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
-        void* ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
-    return fn;
-}
-
-// [B*heads][H][W][d] bf16 viewed as 4-D tensor maps, one per box shape (BoxShape order:
-// 8x8, 8 cols x 4 rows, 4 cols x 8 rows, 4x4), 128-byte swizzle.
-bool encode_window_maps(CUtensorMap* m4, const void* base, int BH, int H, int W)
-{
-    EncodeTiledFn fn = get_encode_fn();
-    if (!fn) return false;
-    const cuuint32_t cols[4] = {8, 8, 4, 4}, rows[4] = {8, 4, 8, 4};
-    for (int s = 0; s < 4; ++s) {
-        cuuint64_t dims[4] = {(cuuint64_t)kD, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)BH};
-        cuuint64_t strides[3] = {(cuuint64_t)kD * 2, (cuuint64_t)W * kD * 2, (cuuint64_t)H * W * kD * 2};
-        cuuint32_t box[4] = {kD, cols[s], rows[s], 1};
-        cuuint32_t es[4] = {1, 1, 1, 1};
-        CUresult r = fn(&m4[s], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-        if (r != CUDA_SUCCESS) return false;
-    }
-    return true;
-}
-
-// SM count of the current device (1 when it cannot be read; not cached then).
 // [B*heads][T][d] bf16 as a 3-D map with 64-row boxes (128-byte swizzle); rows past T read
 // as zeros.
 bool encode_rows_map(CUtensorMap* m, const void* base, int BH, int T)
 {
-    EncodeTiledFn fn = get_encode_fn();
+    EncodeTiledFn fn = tensor_map_encoder();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)T, (cuuint64_t)BH};
     cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)T * kD * 2};

@@ -3,6 +3,7 @@
 #include <cstdint>
 #include <mutex>
 #include <utility>
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 
@@ -34,6 +35,11 @@ constexpr int kMaxDevices = 64;
 int current_device();
 // SM count of the current device (1 when it cannot be read; not cached then).
 int device_sm_count();
+// The driver's cuTensorMapEncodeTiled, looked up once through the runtime (null if absent).
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
 // Opaque identity of the current context (0 if unknown): a cached device address is valid only
 // in the context it was looked up in (cudaDeviceReset replaces the primary context).
 uintptr_t current_context_id();
@@ -133,6 +139,12 @@ int launch_backward(const ssba_desc& d, const Grid& g, int keep, float scale, co
 int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
                        const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
                        const int32_t* cnt, float* dQ, float* dK, float* dV, float* Dbuf, cudaStream_t st);
+// The persistent warp-specialised tensor-core backward (bf16, head_dim 64, shifts that are
+// multiples of 4, Tb <= 256); SSBA_ERR_UNSUPPORTED otherwise. workspace = the caller's
+// ssba_backward workspace (bwd_layout).
+int launch_backward_ws(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
+                       const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
+                       const int32_t* cnt, float* dQ, float* dK, float* dV, void* workspace, cudaStream_t st);
 
 int launch_haar(bool inverse, const void* in, void* out, int N, int C, int H, int W, int nb, int dtype,
                 cudaStream_t st);

@@ -554,27 +554,9 @@ __global__ void __launch_bounds__(kThreads, 1) ssba_qkv_rope_pool_kernel(const _
     if (warp == 1) tmem_dealloc(tbase, kTmemCols);
 }
 
-typedef CUresult (*EncodeTiledFnQ)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFnQ encode_fn()
-{
-    static EncodeTiledFnQ fn = nullptr;
-    if (!fn) {
-        void* ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFnQ>(ptr);
-    }
-    return fn;
-}
-
 bool encode_maps(QkvMaps& m, const void* X, const void* Wqkv, int B, int H, int W, int Dm)
 {
-    EncodeTiledFnQ fn = encode_fn();
+    EncodeTiledFn fn = tensor_map_encoder();
     if (!fn) return false;
     for (int s = 0; s < 8; ++s) {
         cuuint64_t dims[3] = {(cuuint64_t)Dm, (cuuint64_t)W, (cuuint64_t)H * B};
