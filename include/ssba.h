@@ -191,9 +191,10 @@ SSBA_API int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, 
                            float* dQ, float* dK, float* dV, void* workspace, size_t ws_bytes, void* stream);
 
 /* Bytes of the ssba_backward workspace (0 for an invalid descriptor): D of every row
- * (B * heads * N * 4, rounded up to 256), then 256 bytes for a work counter and the transposed
- * lists, three int arrays of B * heads * Tb, B * heads * Tb and B * heads * Tb * keep entries
- * (each rounded up to 256 bytes). Every part is rewritten by each call: no zero-fill needed. */
+ * (B * heads * N * 4, rounded up to 256), then 256 bytes for a work counter, the transposed
+ * lists (three int arrays of B * heads * Tb, B * heads * Tb and B * heads * Tb * keep entries)
+ * and the rows' (lse, D) pairs by block (B * heads * N * 8 bytes), each part rounded up to 256
+ * bytes. Every part is rewritten by each call: no zero-fill needed. */
 SSBA_API size_t ssba_backward_workspace_bytes(const ssba_desc* desc);
 
 /* Block compression alone (Sec. 2.2, the means q_b, k_b; Algorithm 1 MeanPool): the first

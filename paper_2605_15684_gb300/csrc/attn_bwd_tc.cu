@@ -35,6 +35,7 @@
 #include "common.cuh"
 #include "bwd_tile.cuh"
 #include "ptx.cuh"
+#include "window.cuh"
 
 namespace ssba {
 
@@ -586,7 +587,16 @@ __global__ void __launch_bounds__(256) ssba_bwd_rows_kernel(const BwdParams p, c
         }
     }
     Dr += __shfl_xor_sync(0xffffffffu, Dr, 1);
-    if (row < rows && h == 0) p.Dbuf[row] = Dr;
+    if (row < rows && h == 0) {
+        p.Dbuf[row] = Dr;
+        if (p.ld) {  // the same row by block, at its tile row, beside its log2-domain lse
+            const int N = p.g.H * p.g.W, bh = row / N;
+            int label, pos;
+            win::token_block(p.g, row - bh * N, label, pos);
+            const int r = win::tile_row_of(p.g, label, pos);
+            p.ld[((size_t)bh * p.g.Tb() + label) * kT + r] = make_float2(__ldg(p.lse + row) * kLog2e, Dr);
+        }
+    }
 }
 
 // Both gradient roles in one grid: CTAs [0, BH Tb) are key blocks (dK, dV; their list lengths
@@ -617,7 +627,8 @@ BwdLayout bwd_layout(const ssba_desc& d, const Grid& g, int keep)
     l.toff = l.ctr + 256;
     l.tcnt = l.toff + up(BH * Tb * sizeof(int));
     l.tlist = l.tcnt + up(BH * Tb * sizeof(int));
-    l.bytes = l.tlist + up(BH * Tb * (size_t)keep * sizeof(int));
+    l.ld = l.tlist + up(BH * Tb * (size_t)keep * sizeof(int));
+    l.bytes = l.ld + up(BH * g.H * g.W * 2 * sizeof(float));
     return l;
 }
 
@@ -651,6 +662,7 @@ int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale,
     p.dV = dV;
     p.Dbuf = Dbuf;
     p.ctr = p.toff = p.tcnt = p.tlist = nullptr;
+    p.ld = nullptr;
     p.g = g;
     p.keep = keep;
     p.scale = scale;

@@ -10,8 +10,9 @@
 //   warp 5     producer: publishes each item (role, head, block, count and its list of other
 //              blocks: the forward's list for dQ, the transposed list the row kernel built for
 //              dK, dV) in one of two item slots; copies the item's resident tiles by TMA (two
-//              buffers, by item parity) and each pair's streamed tiles (a ring of three), and
-//              the lse and D values the compute warps use (cp.async, counted on mbarriers).
+//              buffers, by item parity) and each pair's streamed tiles (a ring of three), each
+//              with the 512-byte row of (lse, D) values of its block that the compute warps
+//              use (the row kernel writes them by block, in tile order: one bulk copy).
 //   warp 4     lane 0 issues every MMA: per pair S, dP into the same TMEM columns once the
 //              compute warps hold the last ones in registers, then the accumulating products
 //              of the previous pair once its bf16 operands are in shared memory.
@@ -57,20 +58,17 @@ struct alignas(1024) WsSmem {
     uint8_t x[kRing][kTile];  // pair tiles: dQ item K_j, dK/dV item Q_i
     uint8_t y[kRing][kTile];  //             V_j,         dO_i
     uint8_t e[2][kTile];      // bf16 operands: dS (e[0]); P^T and dS^T
-    float pls[kRing][kT];     // dK/dV pair: lse of its query rows (tile order)
-    float pds[kRing][kT];     //             D of its query rows
-    float ils[2][kT];         // dQ item: lse of its rows
-    float ids[2][kT];         //          D of its rows
+    float2 pld[kRing][kT];    // dK/dV pair: (lse log2(e), D) of its query rows (tile order)
+    float2 ild[2][kT];        // dQ item: (lse log2(e), D) of its rows
     int list[2][256];         // the item's other blocks, in pair order (producer only)
+    uint32_t win[256];        // label -> packed window entry (window_entry)
     int4 info[2];             // role (0 dQ, 1 dK/dV, kDone), bh, label, n
     uint64_t item_full[2];    // producer lane 0, after the slot is written
     uint64_t item_empty[2];   // the 4 compute warps and the issuer have read the slot
-    uint64_t ild_full[2];     // 32 producer lanes' cp.async of ils, ids
-    uint64_t ab_full[2];      // TMA bytes of the item tiles
+    uint64_t ab_full[2];      // TMA bytes of the item tiles (and, for dQ, of its ild row)
     uint64_t ab_empty[2];     // MMA commit after the item's last S, dP
-    uint64_t tile_full[kRing];   // TMA bytes of a pair's tiles
+    uint64_t tile_full[kRing];   // TMA bytes of a pair's tiles (and, for dK/dV, of its pld row)
     uint64_t tile_empty[kRing];  // MMA commit after the pair's accumulating products
-    uint64_t lsd_full[kRing];    // 32 producer lanes' cp.async of pls, pds
     uint64_t bar_s;           // MMA commit: S, dP of the pair in TMEM
     uint64_t s_free;          // 4 compute warps: S, dP in registers
     uint64_t e_full;          // 4 compute warps: the pair's bf16 operands stored
@@ -86,19 +84,6 @@ __device__ __forceinline__ WsSmem& smem_layout()
     extern __shared__ uint8_t raw[];
     return *reinterpret_cast<WsSmem*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023));
 }
-
-__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src)
-{
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
-}
-
-// Counts one arrival on bar once this thread's earlier cp.async copies have landed.
-__device__ __forceinline__ void cp_async_arrive(uint32_t bar)
-{
-    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 // A warp's bounded wait: every lane must see the phase, so a timeout takes the warp out whole.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abortf, uint64_t budget_ns)
@@ -119,6 +104,8 @@ __device__ __forceinline__ int tile_token(const Grid& g, int label, int r)
 {
     return g.token(label, tile_row_pos(g, label, r));
 }
+
+constexpr uint32_t kLdRow = kT * sizeof(float2);  // 512 bytes of (lse, D) per block
 
 // An item slot's shape, read after its mbarrier wait.
 __device__ __forceinline__ int4 read_info(const int4* q)
@@ -142,7 +129,7 @@ __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, cons
 {
     const int lane = threadIdx.x & 31;
     const Grid& g = p.g;
-    const int Tb = g.Tb(), N = g.H * g.W;
+    const int Tb = g.Tb();
     volatile int* abortf = &sm.abort_flag;
     grid_dep_wait();  // D, the counter and the transposed lists come from the row kernel
     int w = blockIdx.x;
@@ -171,14 +158,6 @@ __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, cons
             src = p.idx + brow * p.keep;
         }
         for (int i = lane; i < n; i += 32) sm.list[s][i] = min(max(__ldg(src + i), 0), Tb - 1);
-        if (role == 0) {  // lse and D of the item's own rows
-            for (int r = lane; r < kT; r += 32) {
-                const size_t tok = (size_t)bh * N + tile_token(g, label, r);
-                cp_async4(smem_u32(&sm.ils[s][r]), p.lse + tok);
-                cp_async4(smem_u32(&sm.ids[s][r]), p.Dbuf + tok);
-            }
-        }
-        cp_async_arrive(smem_u32(&sm.ild_full[s]));
         __syncwarp();
         if (lane == 0) {
             sm.info[s] = make_int4(role, bh, label, n);
@@ -187,10 +166,11 @@ __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, cons
         // the item's resident tiles, once the item two back has issued its last S, dP
         if (k >= 2 && !warp_wait(smem_u32(&sm.ab_empty[s]), ((k >> 1) + 1) & 1, abortf, p.budget_ns)) return false;
         if (lane == 0) {
-            const uint32_t bar = smem_u32(&sm.ab_full[s]), e = window_entry(g, label);
-            mbar_arrive_expect_tx(bar, 2 * kTile);
+            const uint32_t bar = smem_u32(&sm.ab_full[s]), e = sm.win[label];
+            mbar_arrive_expect_tx(bar, 2 * kTile + (role ? 0 : kLdRow));
             window_boxes_e(role ? maps.k : maps.q, smem_u32(sm.a[s]), bar, e, bh);
             window_boxes_e(role ? maps.v : maps.o, smem_u32(sm.b[s]), bar, e, bh);
+            if (!role) bulk_load(smem_u32(sm.ild[s]), p.ld + brow * kT, kLdRow, bar);
         }
         ++kab;
         // the pairs' streamed tiles, each once the pair three back has finished its products
@@ -200,19 +180,12 @@ __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, cons
                 return false;
             const int j = sm.list[s][t];
             if (lane == 0) {
-                const uint32_t bar = smem_u32(&sm.tile_full[r]), e = window_entry(g, j);
-                mbar_arrive_expect_tx(bar, 2 * kTile);
+                const uint32_t bar = smem_u32(&sm.tile_full[r]), e = sm.win[j];
+                mbar_arrive_expect_tx(bar, 2 * kTile + (role ? kLdRow : 0));
                 window_boxes_e(role ? maps.q : maps.k, smem_u32(sm.x[r]), bar, e, bh);
                 window_boxes_e(role ? maps.o : maps.v, smem_u32(sm.y[r]), bar, e, bh);
+                if (role) bulk_load(smem_u32(sm.pld[r]), p.ld + ((size_t)bh * Tb + j) * kT, kLdRow, bar);
             }
-            if (role == 1) {  // lse and D of the pair's query rows
-                for (int rr = lane; rr < kT; rr += 32) {
-                    const size_t tok = (size_t)bh * N + tile_token(g, j, rr);
-                    cp_async4(smem_u32(&sm.pls[r][rr]), p.lse + tok);
-                    cp_async4(smem_u32(&sm.pds[r][rr]), p.Dbuf + tok);
-                }
-            }
-            cp_async_arrive(smem_u32(&sm.lsd_full[r]));
         }
         int next = 0;
         if (lane == 0) next = (int)gridDim.x + atomicAdd(p.ctr, 1);
@@ -315,10 +288,10 @@ __device__ bool compute(const BwdParams& p, WsSmem& sm)
         if (!warp_wait(smem_u32(&sm.item_full[s]), (k >> 1) & 1, abortf, p.budget_ns)) return false;
         const int4 inf = read_info(&sm.info[s]);
         float L2 = 0.f, Dr = 0.f;
-        if (inf.x == 0) {
-            if (!warp_wait(smem_u32(&sm.ild_full[s]), (k >> 1) & 1, abortf, p.budget_ns)) return false;
-            L2 = sm.ils[s][r] * kLog2e;
-            Dr = sm.ids[s][r];
+        if (inf.x == 0) {  // the row's statistics came with the item's tiles
+            if (!warp_wait(smem_u32(&sm.ab_full[s]), (k >> 1) & 1, abortf, p.budget_ns)) return false;
+            L2 = sm.ild[s][r].x;
+            Dr = sm.ild[s][r].y;
         }
         warp_arrive(smem_u32(&sm.item_empty[s]));
         if (inf.x == kDone) return true;
@@ -337,17 +310,16 @@ __device__ bool compute(const BwdParams& p, WsSmem& sm)
             warp_arrive(smem_u32(&sm.s_free));
             if (role == 1) {
                 // S^T, dP^T: columns are the query rows 32 h + i of the pair's query block
-                if (!warp_wait(smem_u32(&sm.lsd_full[slot]), (P / kRing) & 1, abortf, p.budget_ns)) return false;
-                const float* Lq = sm.pls[slot] + 32 * h;
-                const float* Dq = sm.pds[slot] + 32 * h;
+                if (!warp_wait(smem_u32(&sm.tile_full[slot]), (P / kRing) & 1, abortf, p.budget_ns)) return false;
+                const float4* ld = reinterpret_cast<const float4*>(sm.pld[slot] + 32 * h);
                 uint32_t pp[16], dd[16];
 #pragma unroll
                 for (int i = 0; i < 16; ++i) {
-                    const float p0 = fast_exp2(fmaf(__uint_as_float(sv[2 * i]), c, -Lq[2 * i] * kLog2e));
-                    const float p1 = fast_exp2(fmaf(__uint_as_float(sv[2 * i + 1]), c, -Lq[2 * i + 1] * kLog2e));
+                    const float4 q = ld[i];  // (lse, D) of query rows 32 h + 2 i and 32 h + 2 i + 1
+                    const float p0 = fast_exp2(fmaf(__uint_as_float(sv[2 * i]), c, -q.x));
+                    const float p1 = fast_exp2(fmaf(__uint_as_float(sv[2 * i + 1]), c, -q.z));
                     pp[i] = pack_bf16(p0, p1);
-                    dd[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - Dq[2 * i]),
-                                      p1 * (__uint_as_float(dp[2 * i + 1]) - Dq[2 * i + 1]));
+                    dd[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - q.y), p1 * (__uint_as_float(dp[2 * i + 1]) - q.w));
                 }
                 // the last pair's products have read e[] (and the tiles of its slot)
                 if (P > 0 && !warp_wait(smem_u32(&sm.bar_a), (P - 1) & 1, abortf, p.budget_ns)) return false;
@@ -403,14 +375,12 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_ws_kernel(const __grid_cons
         for (int i = 0; i < 2; ++i) {
             mbar_init(smem_u32(&sm.item_full[i]), 1);
             mbar_init(smem_u32(&sm.item_empty[i]), kCompute / 32 + 1);
-            mbar_init(smem_u32(&sm.ild_full[i]), 32);
             mbar_init(smem_u32(&sm.ab_full[i]), 1);
             mbar_init(smem_u32(&sm.ab_empty[i]), 1);
         }
         for (int i = 0; i < kRing; ++i) {
             mbar_init(smem_u32(&sm.tile_full[i]), 1);
             mbar_init(smem_u32(&sm.tile_empty[i]), 1);
-            mbar_init(smem_u32(&sm.lsd_full[i]), 32);
         }
         mbar_init(smem_u32(&sm.bar_s), 1);
         mbar_init(smem_u32(&sm.s_free), kCompute / 32);
@@ -419,6 +389,7 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_ws_kernel(const __grid_cons
         mbar_init(smem_u32(&sm.drain), 1);
         fence_mbar_init();
     }
+    for (int l = threadIdx.x; l < p.g.Tb(); l += kThreads) sm.win[l] = window_entry(p.g, l);
     if (warp == kProducer && lane < 16) {
         const CUtensorMap* m = lane < 4 ? &maps.q[lane] : lane < 8 ? &maps.k[lane - 4] : lane < 12 ? &maps.v[lane - 8]
                                                                                                   : &maps.o[lane - 12];
@@ -466,7 +437,6 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_ws_kernel(const __grid_cons
         }
         if (threadIdx.x == 0) atomicExch(p.status, SSBA_ERR_TIMEOUT);
     }
-    cp_async_wait_all();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -505,6 +475,7 @@ int launch_backward_ws(const ssba_desc& d, const Grid& g, int keep, float scale,
     p.toff = reinterpret_cast<int*>(ws + lay.toff);
     p.tcnt = reinterpret_cast<int*>(ws + lay.tcnt);
     p.tlist = reinterpret_cast<int*>(ws + lay.tlist);
+    p.ld = reinterpret_cast<float2*>(ws + lay.ld);
     p.g = g;
     p.keep = keep;
     p.scale = scale;

@@ -60,10 +60,10 @@ __device__ __forceinline__ void store_half_row(uint8_t* dst, int r, int h, const
     }
 }
 
-// Arguments of the backward kernels (device pointers). ctr, toff, tcnt and tlist are the
-// persistent kernel's: its work counter and the transposed lists (CSR per head: for key block j
-// of head bh, tcnt[bh Tb + j] query blocks, ascending, at tlist + toff[bh Tb + j]); null for the
-// per-block kernel.
+// Arguments of the backward kernels (device pointers). ctr, toff, tcnt, tlist and ld are the
+// persistent kernel's: its work counter, the transposed lists (CSR per head: for key block j of
+// head bh, tcnt[bh Tb + j] query blocks, ascending, at tlist + toff[bh Tb + j]) and the row
+// statistics by block; null for the per-block kernel.
 struct BwdParams {
     const __nv_bfloat16 *Q, *K, *V, *O, *dO;
     const float* lse;
@@ -71,6 +71,7 @@ struct BwdParams {
     const int32_t* cnt;
     float *dQ, *dK, *dV, *Dbuf;
     int *ctr, *toff, *tcnt, *tlist;
+    float2* ld;  // [B*heads][Tb][64]: (lse log2(e), D) of each block's rows in TMA tile order
     Grid g;
     int keep;
     float scale;
@@ -81,12 +82,12 @@ struct BwdParams {
 // Byte offsets in the ssba_backward workspace: D of every row first (every path), then the
 // persistent kernel's counter and transposed lists.
 struct BwdLayout {
-    size_t ctr, toff, tcnt, tlist, bytes;
+    size_t ctr, toff, tcnt, tlist, ld, bytes;
 };
 BwdLayout bwd_layout(const ssba_desc& d, const Grid& g, int keep);
 
-// The row kernel: D for every row and, when p.tlist is set, the counter reset and the
-// transposed lists (one extra CTA per head). Launched plainly (it depends on all earlier work);
+// The row kernel: D for every row and, when p.tlist is set, the rows' (lse log2(e), D) by block
+// in tile order, the counter reset and the transposed lists (one extra CTA per head). Launched plainly (it depends on all earlier work);
 // the gradient kernel that follows is its programmatic dependent.
 cudaError_t launch_bwd_rows(const BwdParams& p, int BH, cudaStream_t st);
 

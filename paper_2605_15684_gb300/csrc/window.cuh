@@ -84,6 +84,29 @@ __device__ __forceinline__ int tile_row_pos(const Grid& g, int label, int r)
     return (4 * (q >> 1) + a) * 8 + 4 * (q & 1) + b;
 }
 
+// Inverse of tile_row_pos: the tile row that holds in-window position pos of block `label`.
+__device__ __forceinline__ int tile_row_of(const Grid& g, int label, int pos)
+{
+    int r0, c0;
+    window_origin(g, label, r0, c0);
+    const bool wr = r0 + 8 > g.H, wc = c0 + 8 > g.W;
+    if (!wc) return pos;
+    const int a = pos >> 3, c = pos & 7;
+    if (!wr) return (c >> 2) * 32 + a * 4 + (c & 3);
+    return ((a >> 2) * 2 + (c >> 2)) * 16 + (a & 3) * 4 + (c & 3);
+}
+
+// Block label and in-window position of token t (the inverse of Grid::token).
+__device__ __forceinline__ void token_block(const Grid& g, int t, int& label, int& pos)
+{
+    const int r = t / g.W, c = t - r * g.W;
+    int R = r + g.sr, C = c + g.sc;
+    R -= R >= g.H ? g.H : 0;
+    C -= C >= g.W ? g.W : 0;
+    label = (R >> 3) * g.bw + (C >> 3);
+    pos = (R & 7) * 8 + (C & 7);
+}
+
 }  // namespace win
 
 // [B*heads][H][W][64] bf16 viewed as 4-D tensor maps, one per box shape (BoxShape order),

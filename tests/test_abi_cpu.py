@@ -137,11 +137,11 @@ def test_backward_validation(lib):
     """The backward entry point checks its workspace and shape before any launch."""
     d = desc()
     need = lib.ssba_backward_workspace_bytes(ctypes.byref(d))
-    # D per row, a 256-byte counter, then the transposed lists (offsets, counts, entries), each
-    # part rounded up to 256 bytes
+    # D per row, a 256-byte counter, the transposed lists (offsets, counts, entries), then the
+    # rows' (lse, D) pairs by block, each part rounded up to 256 bytes
     up = lambda x: (x + 255) // 256 * 256
     BH, N, Tb, keep = 1 * 2, 16 * 16, 4, lib.ssba_keep_count(ctypes.byref(d))
-    assert need == up(BH * N * 4) + 256 + 2 * up(BH * Tb * 4) + up(BH * Tb * keep * 4)
+    assert need == up(BH * N * 4) + 256 + 2 * up(BH * Tb * 4) + up(BH * Tb * keep * 4) + up(BH * N * 8)
     args = [ctypes.byref(d)] + [FAKE] * 11
     assert lib.ssba_backward(*args, FAKE, need - 4, None) == api.SSBA_ERR_WORKSPACE
     assert lib.ssba_backward(*args, None, need, None) == api.SSBA_ERR_WORKSPACE
