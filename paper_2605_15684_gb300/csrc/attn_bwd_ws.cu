@@ -7,15 +7,16 @@
 // Work items: a key block's dK, dV or a query block's dQ, of one (batch, head). The first item
 // of a CTA is its index; the others come from a counter in the workspace that the row kernel
 // zeroes. Key-block items come first (their lengths vary), query-block items fill in behind.
-//   warp 5     producer: publishes each item (role, head, block, count and its list of other
+//   warp 6     producer: publishes each item (role, head, block, count and its list of other
 //              blocks: the forward's list for dQ, the transposed list the row kernel built for
 //              dK, dV) in one of two item slots; copies the item's resident tiles by TMA (two
 //              buffers, by item parity) and each pair's streamed tiles (a ring of three), each
 //              with the 512-byte row of (lse, D) values of its block that the compute warps
 //              use (the row kernel writes them by block, in tile order: one bulk copy).
-//   warp 4     lane 0 issues every MMA: per pair S, dP into the same TMEM columns once the
-//              compute warps hold the last ones in registers, then the accumulating products
-//              of the previous pair once its bf16 operands are in shared memory.
+//   warps 4-5  lane 0 of each issues one side of the MMAs (S and the products reading the
+//              pair's x tile; dP and the one reading its y tile): per pair S, dP into the same
+//              TMEM columns once the compute warps hold the last ones in registers, then the
+//              accumulating products of the previous pair once its bf16 operands are stored.
 //   warps 0-3  the exps and the bf16 operands of each pair, one TMEM lane quadrant each, and
 //              each item's epilogue (the accumulators to global memory, fp32).
 // Pairs are counted across items: the next item's tiles arrive while the last item computes,
@@ -39,9 +40,11 @@ using namespace win;
 using namespace bwd;
 
 constexpr int kCompute = 128;   // warps 0-3
-constexpr int kIssuer = 128;    // lane 0 of warp 4
-constexpr int kProducer = 5;    // warp
-constexpr int kThreads = 192;
+constexpr int kIssuer0 = 128;   // lane 0 of warp 4: S and the products that read the x tiles
+constexpr int kIssuer1 = 160;   // lane 0 of warp 5: dP and the products that read the y tiles
+constexpr int kIssuers = 2;
+constexpr int kProducer = 6;    // warp
+constexpr int kThreads = 224;
 constexpr int kRing = 3;        // streamed tile slots
 constexpr int kDone = -1;       // role of the item slot that ends a CTA's work
 constexpr uint32_t kTmemCols = 256;
@@ -64,15 +67,15 @@ struct alignas(1024) WsSmem {
     uint32_t win[256];        // label -> packed window entry (window_entry)
     int4 info[2];             // role (0 dQ, 1 dK/dV, kDone), bh, label, n
     uint64_t item_full[2];    // producer lane 0, after the slot is written
-    uint64_t item_empty[2];   // the 4 compute warps and the issuer have read the slot
+    uint64_t item_empty[2];   // the 4 compute warps and the 2 issuers have read the slot
     uint64_t ab_full[2];      // TMA bytes of the item tiles (and, for dQ, of its ild row)
-    uint64_t ab_empty[2];     // MMA commit after the item's last S, dP
+    uint64_t ab_empty[2];     // MMA commits (both issuers) after the item's last S, dP
     uint64_t tile_full[kRing];   // TMA bytes of a pair's tiles (and, for dK/dV, of its pld row)
-    uint64_t tile_empty[kRing];  // MMA commit after the pair's accumulating products
-    uint64_t bar_s;           // MMA commit: S, dP of the pair in TMEM
+    uint64_t tile_empty[kRing];  // MMA commits (both issuers) after the pair's products
+    uint64_t bar_s;           // MMA commits (both issuers): S, dP of the pair in TMEM
     uint64_t s_free;          // 4 compute warps: S, dP in registers
     uint64_t e_full;          // 4 compute warps: the pair's bf16 operands stored
-    uint64_t bar_a;           // MMA commit: the pair's accumulating products done
+    uint64_t bar_a;           // MMA commits (both issuers): the pair's accumulating products
     uint64_t drain;
     uint32_t tmem_base;
     int abort_flag;
@@ -122,7 +125,7 @@ __device__ __forceinline__ int4 decode_item(int w, int nk, int Tb)
     return make_int4(key ? 1 : 0, bh, u - bh * Tb, 0);
 }
 
-// Warp 5. nk = number of key-block items (B * heads * Tb), total = 2 nk. Returns false on a
+// Warp 6. nk = number of key-block items (B * heads * Tb), total = 2 nk. Returns false on a
 // timeout. P counts the pairs whose tiles were issued, kab the items whose tiles were issued
 // (after a timeout the teardown waits for the last copies of each barrier).
 __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, const int nk, uint32_t& P, int& kab)
@@ -193,28 +196,33 @@ __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, cons
     }
 }
 
-// The accumulating products of pair q (role and whether it opens its item from the pair's
-// bookkeeping), once its bf16 operands are stored; frees the pair's ring slot when done.
-__device__ __forceinline__ bool issue_acc(const BwdParams& p, WsSmem& sm, uint32_t q, int role, bool first)
+// Issuer `which`'s share of the accumulating products of pair q (its role, and whether it opens
+// its item), once the pair's bf16 operands are stored: issuer 0 dQ += dS K or dK += dS^T Q
+// (x tiles), issuer 1 dV += P^T dO (y tiles). Each commits, so the barriers count two.
+__device__ __forceinline__ bool issue_acc(const BwdParams& p, WsSmem& sm, uint32_t q, int role, bool first, int which)
 {
     if (!mbar_wait(smem_u32(&sm.e_full), q & 1, &sm.abort_flag, p.budget_ns)) return false;
     tc_fence_after();
     const uint32_t tb0 = sm.tmem_base;
     const int r = (int)(q % kRing);
-    if (role == 1) {
+    if (which == 0) {
+        if (role == 1)
+            mma_sb(tb0 + kColA1, smem_u32(sm.e[1]), smem_u32(sm.x[r]), !first);  // dK += dS^T Q
+        else
+            mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.x[r]), !first);  // dQ += dS K
+    } else if (role == 1) {
         mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.y[r]), !first);  // dV += P^T dO
-        mma_sb(tb0 + kColA1, smem_u32(sm.e[1]), smem_u32(sm.x[r]), !first);  // dK += dS^T Q
-    } else {
-        mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.x[r]), !first);  // dQ += dS K
     }
     mma_commit(smem_u32(&sm.bar_a));
     mma_commit(smem_u32(&sm.tile_empty[r]));
     return true;
 }
 
-// Lane 0 of warp 4. Returns false on a timeout; `issued` tells the teardown that MMAs may be in
-// flight.
-__device__ bool issue(const BwdParams& p, WsSmem& sm, bool& issued)
+// Lane 0 of warp 4 (which = 0) or 5 (which = 1): the products of one side of every pair, so
+// that two threads share the issue latency of a tcgen05.mma (about 57 cycles from one thread,
+// 44 a product when several issue). Returns false on a timeout; `issued` tells the teardown
+// that MMAs may be in flight.
+__device__ bool issue(const BwdParams& p, WsSmem& sm, const int which, bool& issued)
 {
     volatile int* abortf = &sm.abort_flag;
     const uint32_t tb0 = sm.tmem_base;
@@ -227,7 +235,7 @@ __device__ bool issue(const BwdParams& p, WsSmem& sm, bool& issued)
         // the last item's final products first: its epilogue waits for them, and the next
         // item's tiles may still be on their way
         if (pending) {
-            if (!issue_acc(p, sm, P - 1, prole, pfirst)) return false;
+            if (!issue_acc(p, sm, P - 1, prole, pfirst, which)) return false;
             pending = false;
         }
         if (!mbar_wait(smem_u32(&sm.item_full[s]), (k >> 1) & 1, abortf, p.budget_ns)) return false;
@@ -236,18 +244,20 @@ __device__ bool issue(const BwdParams& p, WsSmem& sm, bool& issued)
         if (inf.x == kDone) return true;
         const int role = inf.x, n = inf.w;
         if (!mbar_wait(smem_u32(&sm.ab_full[s]), (k >> 1) & 1, abortf, p.budget_ns)) return false;
-        const uint32_t a = smem_u32(sm.a[s]), b = smem_u32(sm.b[s]);
+        const uint32_t ab = smem_u32(which ? sm.b[s] : sm.a[s]);
         for (int t = 0; t < n; ++t, ++P) {
             const int r = (int)(P % kRing);
             if (!mbar_wait(smem_u32(&sm.tile_full[r]), (P / kRing) & 1, abortf, p.budget_ns)) return false;
             if (P > 0 && !mbar_wait(smem_u32(&sm.s_free), (P - 1) & 1, abortf, p.budget_ns)) return false;
             tc_fence_after();
-            mma_kk(tb0 + kColS, a, smem_u32(sm.x[r]));   // S = Q K^T (dK/dV item: S^T = K Q^T)
-            mma_kk(tb0 + kColDP, b, smem_u32(sm.y[r]));  // dP = dO V^T (dP^T = V dO^T)
+            if (which == 0)
+                mma_kk(tb0 + kColS, ab, smem_u32(sm.x[r]));  // S = Q K^T (dK/dV item: S^T = K Q^T)
+            else
+                mma_kk(tb0 + kColDP, ab, smem_u32(sm.y[r]));  // dP = dO V^T (dP^T = V dO^T)
             mma_commit(smem_u32(&sm.bar_s));
             issued = true;
             if (t == n - 1) mma_commit(smem_u32(&sm.ab_empty[s]));
-            if (pending && !issue_acc(p, sm, P - 1, prole, pfirst)) return false;
+            if (pending && !issue_acc(p, sm, P - 1, prole, pfirst, which)) return false;
             pending = true;
             prole = role;
             pfirst = t == 0;
@@ -374,19 +384,19 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_ws_kernel(const __grid_cons
         sm.abort_flag = 0;
         for (int i = 0; i < 2; ++i) {
             mbar_init(smem_u32(&sm.item_full[i]), 1);
-            mbar_init(smem_u32(&sm.item_empty[i]), kCompute / 32 + 1);
+            mbar_init(smem_u32(&sm.item_empty[i]), kCompute / 32 + kIssuers);
             mbar_init(smem_u32(&sm.ab_full[i]), 1);
-            mbar_init(smem_u32(&sm.ab_empty[i]), 1);
+            mbar_init(smem_u32(&sm.ab_empty[i]), kIssuers);
         }
         for (int i = 0; i < kRing; ++i) {
             mbar_init(smem_u32(&sm.tile_full[i]), 1);
-            mbar_init(smem_u32(&sm.tile_empty[i]), 1);
+            mbar_init(smem_u32(&sm.tile_empty[i]), kIssuers);
         }
-        mbar_init(smem_u32(&sm.bar_s), 1);
+        mbar_init(smem_u32(&sm.bar_s), kIssuers);
         mbar_init(smem_u32(&sm.s_free), kCompute / 32);
         mbar_init(smem_u32(&sm.e_full), kCompute / 32);
-        mbar_init(smem_u32(&sm.bar_a), 1);
-        mbar_init(smem_u32(&sm.drain), 1);
+        mbar_init(smem_u32(&sm.bar_a), kIssuers);
+        mbar_init(smem_u32(&sm.drain), kIssuers);
         fence_mbar_init();
     }
     for (int l = threadIdx.x; l < p.g.Tb(); l += kThreads) sm.win[l] = window_entry(p.g, l);
@@ -408,8 +418,8 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_ws_kernel(const __grid_cons
     int kab = 0;
     if (warp < kCompute / 32)
         ok = compute(p, sm);
-    else if (threadIdx.x == kIssuer)
-        ok = issue(p, sm, issued);
+    else if (threadIdx.x == kIssuer0 || threadIdx.x == kIssuer1)
+        ok = issue(p, sm, threadIdx.x == kIssuer1 ? 1 : 0, issued);
     else if (warp == kProducer)
         ok = produce(maps, p, sm, nk, P, kab);
     const bool dead = __syncthreads_or(!ok);
@@ -429,7 +439,7 @@ __global__ void __launch_bounds__(kThreads) ssba_bwd_ws_kernel(const __grid_cons
                 settle(smem_u32(&sm.tile_full[q % kRing]), (q / kRing) & 1);
             }
         }
-        if (threadIdx.x == kIssuer && issued) {
+        if (threadIdx.x == kIssuer0 || threadIdx.x == kIssuer1) {  // both commit: the barrier counts two
             mma_commit(smem_u32(&sm.drain));
             const uint64_t t0 = globaltimer_ns();
             while (!mbar_try_wait(smem_u32(&sm.drain), 0) && globaltimer_ns() - t0 < p.budget_ns) {
