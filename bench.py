@@ -34,7 +34,8 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "SSBA fwd latency (ms) and effective TFLOP/s @4096 tok, 84% sparse, bf16"
-ATTN_SOURCES = ("paper_2605_15684_gb300/csrc/attn_tc.cu", "paper_2605_15684_gb300/csrc/ptx.cuh")
+ATTN_SOURCES = ("paper_2605_15684_gb300/csrc/attn_tc.cu", "paper_2605_15684_gb300/csrc/ptx.cuh",
+                "paper_2605_15684_gb300/csrc/window.cuh")
 ATTN_PROFILE = os.path.join(ROOT, "profiles", "ssba_attn_tc_kernel_1024px.md")
 
 
@@ -525,8 +526,10 @@ def run_ours(args, rank, world):
         tb = e0.elapsed_time(e1) / reps
         F_b = 2.5 * F_layer
         bwd = {"ms_per_layer": tb, "effective_tflops": F_b / (tb * 1e-3) / 1e12, "flops_per_layer": F_b,
-               "how": "ssba_backward (tcgen05 kernels: dQ and D per query block, then dK, dV per key block) "
-                      "per layer on the layer's forward O and lse and a synthetic dO, CUDA events"}
+               "how": "ssba_backward per layer (a row kernel: D, the rows' (lse, D) by block, the key "
+                      "blocks' transposed lists; then the persistent warp-specialised tcgen05 kernel, "
+                      "dQ per query block and dK, dV per key block) on the layer's forward O and lse "
+                      "and a synthetic dO, CUDA events"}
     except Exception as exc:  # reported, not fatal
         bwd = f"failed: {exc}"
 
