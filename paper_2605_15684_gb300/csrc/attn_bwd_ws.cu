@@ -7,18 +7,19 @@
 // Work items: a key block's dK, dV or a query block's dQ, of one (batch, head). The first item
 // of a CTA is its index; the others come from a counter in the workspace that the row kernel
 // zeroes. Key-block items come first (their lengths vary), query-block items fill in behind.
-//   warp 6     producer: publishes each item (role, head, block, count and its list of other
+//   warp 10    producer: publishes each item (role, head, block, count and its list of other
 //              blocks: the forward's list for dQ, the transposed list the row kernel built for
 //              dK, dV) in one of two item slots; copies the item's resident tiles by TMA (two
 //              buffers, by item parity) and each pair's streamed tiles (a ring of three), each
 //              with the 512-byte row of (lse, D) values of its block that the compute warps
 //              use (the row kernel writes them by block, in tile order: one bulk copy).
-//   warps 4-5  lane 0 of each issues one side of the MMAs (S and the products reading the
+//   warps 8-9  lane 0 of each issues one side of the MMAs (S and the products reading the
 //              pair's x tile; dP and the one reading its y tile): per pair S, dP into the same
 //              TMEM columns once the compute warps hold the last ones in registers, then the
 //              accumulating products of the previous pair once its bf16 operands are stored.
-//   warps 0-3  the exps and the bf16 operands of each pair, one TMEM lane quadrant each, and
-//              each item's epilogue (the accumulators to global memory, fp32).
+//   warps 0-7  the exps and the bf16 operands of each pair, two warps per TMEM lane quadrant
+//              (16 of a row's 64 columns a thread), and each item's epilogue (the accumulators
+//              to global memory, fp32).
 // Pairs are counted across items: the next item's tiles arrive while the last item computes,
 // and its first products run while the compute warps store the last item's gradients.
 // Tile rows follow the TMA box order (tile_row_pos). Every wait is bounded; on a timeout the
@@ -39,12 +40,12 @@ using namespace ptx;
 using namespace win;
 using namespace bwd;
 
-constexpr int kCompute = 128;   // warps 0-3
-constexpr int kIssuer0 = 128;   // lane 0 of warp 4: S and the products that read the x tiles
-constexpr int kIssuer1 = 160;   // lane 0 of warp 5: dP and the products that read the y tiles
+constexpr int kCompute = 256;   // warps 0-7, two per TMEM lane quadrant
+constexpr int kIssuer0 = 256;   // lane 0 of warp 8: S and the products that read the x tiles
+constexpr int kIssuer1 = 288;   // lane 0 of warp 9: dP and the products that read the y tiles
 constexpr int kIssuers = 2;
-constexpr int kProducer = 6;    // warp
-constexpr int kThreads = 224;
+constexpr int kProducer = 10;   // warp
+constexpr int kThreads = 352;
 constexpr int kRing = 3;        // streamed tile slots
 constexpr int kDone = -1;       // role of the item slot that ends a CTA's work
 constexpr uint32_t kTmemCols = 256;
@@ -67,14 +68,14 @@ struct alignas(1024) WsSmem {
     uint32_t win[256];        // label -> packed window entry (window_entry)
     int4 info[2];             // role (0 dQ, 1 dK/dV, kDone), bh, label, n
     uint64_t item_full[2];    // producer lane 0, after the slot is written
-    uint64_t item_empty[2];   // the 4 compute warps and the 2 issuers have read the slot
+    uint64_t item_empty[2];   // the 8 compute warps and the 2 issuers have read the slot
     uint64_t ab_full[2];      // TMA bytes of the item tiles (and, for dQ, of its ild row)
     uint64_t ab_empty[2];     // MMA commits (both issuers) after the item's last S, dP
     uint64_t tile_full[kRing];   // TMA bytes of a pair's tiles (and, for dK/dV, of its pld row)
     uint64_t tile_empty[kRing];  // MMA commits (both issuers) after the pair's products
     uint64_t bar_s;           // MMA commits (both issuers): S, dP of the pair in TMEM
-    uint64_t s_free;          // 4 compute warps: S, dP in registers
-    uint64_t e_full;          // 4 compute warps: the pair's bf16 operands stored
+    uint64_t s_free;          // 8 compute warps: S, dP in registers
+    uint64_t e_full;          // 8 compute warps: the pair's bf16 operands stored
     uint64_t bar_a;           // MMA commits (both issuers): the pair's accumulating products
     uint64_t drain;
     uint32_t tmem_base;
@@ -125,7 +126,7 @@ __device__ __forceinline__ int4 decode_item(int w, int nk, int Tb)
     return make_int4(key ? 1 : 0, bh, u - bh * Tb, 0);
 }
 
-// Warp 6. nk = number of key-block items (B * heads * Tb), total = 2 nk. Returns false on a
+// Warp 10. nk = number of key-block items (B * heads * Tb), total = 2 nk. Returns false on a
 // timeout. P counts the pairs whose tiles were issued, kab the items whose tiles were issued
 // (after a timeout the teardown waits for the last copies of each barrier).
 __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, const int nk, uint32_t& P, int& kab)
@@ -218,7 +219,7 @@ __device__ __forceinline__ bool issue_acc(const BwdParams& p, WsSmem& sm, uint32
     return true;
 }
 
-// Lane 0 of warp 4 (which = 0) or 5 (which = 1): the products of one side of every pair, so
+// Lane 0 of warp 8 (which = 0) or 9 (which = 1): the products of one side of every pair, so
 // that two threads share the issue latency of a tcgen05.mma (about 57 cycles from one thread,
 // 44 a product when several issue). Returns false on a timeout; `issued` tells the teardown
 // that MMAs may be in flight.
@@ -266,29 +267,44 @@ __device__ bool issue(const BwdParams& p, WsSmem& sm, const int which, bool& iss
     }
 }
 
-// Half row (columns [32 h, 32 h + 32)) of the fp32 accumulator at TMEM address taddr, times
-// mul, to row `token` of out (one [N][64] head).
-__device__ __forceinline__ void store_row(uint32_t taddr, float* out, int token, int h, float mul)
+// Columns [col0, col0 + 16) of this thread's row of the fp32 accumulator whose 16-column
+// group starts at TMEM address taddr, times mul, to row `token` of out (one [N][64] head).
+__device__ __forceinline__ void store_cols(uint32_t taddr, float* out, int token, int col0, float mul)
 {
-    uint32_t v[32];
-    tmem_ld_16x32bx2_x16_off32(taddr, *reinterpret_cast<uint32_t(*)[16]>(&v[0]));
-    tmem_ld_16x32bx2_x16_off32(taddr + 16, *reinterpret_cast<uint32_t(*)[16]>(&v[16]));
+    uint32_t v[16];
+    tmem_ld_16x32bx2_x16_off32(taddr, v);
     tmem_wait_ld();
-    float4* dst = reinterpret_cast<float4*>(out + (size_t)token * kD + 32 * h);
+    float4* dst = reinterpret_cast<float4*>(out + (size_t)token * kD + col0);
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < 4; ++i)
         dst[i] = make_float4(__uint_as_float(v[4 * i]) * mul, __uint_as_float(v[4 * i + 1]) * mul,
                              __uint_as_float(v[4 * i + 2]) * mul, __uint_as_float(v[4 * i + 3]) * mul);
 }
 
-// Warps 0-3: thread (warp, lane) owns TMEM lane (row) r = 16 warp + lane % 16 of the M=64 data
-// path, columns [32 h, 32 h + 32), h = lane / 16. Returns false on a timeout.
+// Sixteen bf16 values (8 packed pairs) of row r, 16-byte chunks c0 and c0 + 1, into the
+// 128-byte-swizzled K-major tile at dst.
+__device__ __forceinline__ void store_cols_bf16(uint8_t* dst, int r, int c0, const uint32_t (&v)[8])
+{
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        const int c = c0 + i;
+        *reinterpret_cast<uint4*>(dst + r * 128 + ((c ^ (r & 7)) << 4)) =
+            make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    }
+}
+
+// Warps 0-7: warp w reads TMEM lane quadrant w % 4; thread (w, lane) owns row
+// r = 16 (w % 4) + lane % 16 of the M=64 data path and its columns [col0, col0 + 16),
+// col0 = 32 (lane / 16) + 16 (w / 4): two warps share each quadrant's exps. Returns false on a
+// timeout.
 __device__ bool compute(const BwdParams& p, WsSmem& sm)
 {
     volatile int* abortf = &sm.abort_flag;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = lane >> 4;
-    const int r = warp * 16 + (lane & 15);
-    const uint32_t tb = sm.tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int q = warp & 3, col0 = 32 * (lane >> 4) + 16 * (warp >> 2);
+    const int r = q * 16 + (lane & 15);
+    // lanes 16-31 of a 16x32bx2 load read 32 columns further on: one address serves the warp
+    const uint32_t tb = sm.tmem_base + (static_cast<uint32_t>(q * 32) << 16) + 16 * (warp >> 2);
     const Grid& g = p.g;
     const int N = g.H * g.W;
     const float c = p.scale * kLog2e;
@@ -310,41 +326,39 @@ __device__ bool compute(const BwdParams& p, WsSmem& sm)
             const int slot = (int)(P % kRing);
             if (!warp_wait(smem_u32(&sm.bar_s), P & 1, abortf, p.budget_ns)) return false;
             tc_fence_after();
-            uint32_t sv[32], dp[32];
-            tmem_ld_16x32bx2_x16_off32(tb + kColS, *reinterpret_cast<uint32_t(*)[16]>(&sv[0]));
-            tmem_ld_16x32bx2_x16_off32(tb + kColS + 16, *reinterpret_cast<uint32_t(*)[16]>(&sv[16]));
-            tmem_ld_16x32bx2_x16_off32(tb + kColDP, *reinterpret_cast<uint32_t(*)[16]>(&dp[0]));
-            tmem_ld_16x32bx2_x16_off32(tb + kColDP + 16, *reinterpret_cast<uint32_t(*)[16]>(&dp[16]));
+            uint32_t sv[16], dp[16];
+            tmem_ld_16x32bx2_x16_off32(tb + kColS, sv);
+            tmem_ld_16x32bx2_x16_off32(tb + kColDP, dp);
             tmem_wait_ld();
             tc_fence_before();
             warp_arrive(smem_u32(&sm.s_free));
             if (role == 1) {
-                // S^T, dP^T: columns are the query rows 32 h + i of the pair's query block
+                // S^T, dP^T: columns are the query rows col0 + i of the pair's query block
                 if (!warp_wait(smem_u32(&sm.tile_full[slot]), (P / kRing) & 1, abortf, p.budget_ns)) return false;
-                const float4* ld = reinterpret_cast<const float4*>(sm.pld[slot] + 32 * h);
-                uint32_t pp[16], dd[16];
+                const float4* ld = reinterpret_cast<const float4*>(sm.pld[slot] + col0);
+                uint32_t pp[8], dd[8];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const float4 q = ld[i];  // (lse, D) of query rows 32 h + 2 i and 32 h + 2 i + 1
-                    const float p0 = fast_exp2(fmaf(__uint_as_float(sv[2 * i]), c, -q.x));
-                    const float p1 = fast_exp2(fmaf(__uint_as_float(sv[2 * i + 1]), c, -q.z));
+                for (int i = 0; i < 8; ++i) {
+                    const float4 qd = ld[i];  // (lse, D) of query rows col0 + 2 i and col0 + 2 i + 1
+                    const float p0 = fast_exp2(fmaf(__uint_as_float(sv[2 * i]), c, -qd.x));
+                    const float p1 = fast_exp2(fmaf(__uint_as_float(sv[2 * i + 1]), c, -qd.z));
                     pp[i] = pack_bf16(p0, p1);
-                    dd[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - q.y), p1 * (__uint_as_float(dp[2 * i + 1]) - q.w));
+                    dd[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - qd.y), p1 * (__uint_as_float(dp[2 * i + 1]) - qd.w));
                 }
                 // the last pair's products have read e[] (and the tiles of its slot)
                 if (P > 0 && !warp_wait(smem_u32(&sm.bar_a), (P - 1) & 1, abortf, p.budget_ns)) return false;
-                store_half_row(sm.e[0], r, h, pp);
-                store_half_row(sm.e[1], r, h, dd);
+                store_cols_bf16(sm.e[0], r, col0 >> 3, pp);
+                store_cols_bf16(sm.e[1], r, col0 >> 3, dd);
             } else {
-                uint32_t pk[16];
+                uint32_t pk[8];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
+                for (int i = 0; i < 8; ++i) {
                     const float p0 = fast_exp2(fmaf(__uint_as_float(sv[2 * i]), c, -L2));
                     const float p1 = fast_exp2(fmaf(__uint_as_float(sv[2 * i + 1]), c, -L2));
                     pk[i] = pack_bf16(p0 * (__uint_as_float(dp[2 * i]) - Dr), p1 * (__uint_as_float(dp[2 * i + 1]) - Dr));
                 }
                 if (P > 0 && !warp_wait(smem_u32(&sm.bar_a), (P - 1) & 1, abortf, p.budget_ns)) return false;
-                store_half_row(sm.e[0], r, h, pk);
+                store_cols_bf16(sm.e[0], r, col0 >> 3, pk);
             }
             fence_proxy_async_smem();
             warp_arrive(smem_u32(&sm.e_full));
@@ -356,26 +370,26 @@ __device__ bool compute(const BwdParams& p, WsSmem& sm)
             if (!warp_wait(smem_u32(&sm.bar_a), (P - 1) & 1, abortf, p.budget_ns)) return false;
             tc_fence_after();
             if (role == 1) {
-                store_row(tb + kColA0, p.dV + head, tok, h, 1.0f);
-                store_row(tb + kColA1, p.dK + head, tok, h, p.scale);
+                store_cols(tb + kColA0, p.dV + head, tok, col0, 1.0f);
+                store_cols(tb + kColA1, p.dK + head, tok, col0, p.scale);
             } else {
-                store_row(tb + kColA0, p.dQ + head, tok, h, p.scale);
+                store_cols(tb + kColA0, p.dQ + head, tok, col0, p.scale);
             }
             tc_fence_before();  // the next item's first products overwrite the accumulators
         } else {
-            float4* a = reinterpret_cast<float4*>((role == 1 ? p.dV : p.dQ) + head + (size_t)tok * kD + 32 * h);
+            float4* a = reinterpret_cast<float4*>((role == 1 ? p.dV : p.dQ) + head + (size_t)tok * kD + col0);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) a[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int i = 0; i < 4; ++i) a[i] = make_float4(0.f, 0.f, 0.f, 0.f);
             if (role == 1) {
-                float4* b = reinterpret_cast<float4*>(p.dK + head + (size_t)tok * kD + 32 * h);
+                float4* b = reinterpret_cast<float4*>(p.dK + head + (size_t)tok * kD + col0);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) b[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int i = 0; i < 4; ++i) b[i] = make_float4(0.f, 0.f, 0.f, 0.f);
             }
         }
     }
 }
 
-__global__ void __launch_bounds__(kThreads) ssba_bwd_ws_kernel(const __grid_constant__ WsMaps maps, const BwdParams p,
+__global__ void __launch_bounds__(kThreads, 2) ssba_bwd_ws_kernel(const __grid_constant__ WsMaps maps, const BwdParams p,
                                                                const int nk)
 {
     WsSmem& sm = smem_layout();

@@ -390,6 +390,25 @@ def test_backward_bf16(H, W, h, rho, shift):
     _bwd_case_gpu(1, h, H, W, rho, shift, torch.bfloat16, 31)
 
 
+def test_backward_is_deterministic():
+    """Repeated calls give bitwise-equal gradients: no atomics, and the work counter only decides
+    which CTA runs an item, not the order of any sum (1024 px layer, 24 heads, shift 4)."""
+    H = W = 64
+    q, k, v = synthetic.qkv(1, 24, H * W, 64, torch.bfloat16, 33)
+    go = synthetic.qkv(1, 24, H * W, 64, torch.bfloat16, 133)[0].cuda()
+    desc = api.SsbaDesc(1, 24, H, W, shift_r=4, shift_c=4, rho=0.8416)
+    qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
+    idx, cnt = api.build_mask(desc, qd, kd)
+    O, lse = api.forward(desc, qd, kd, vd, idx, cnt)
+    first = [g.clone() for g in api.backward(desc, qd, kd, vd, O, lse, go, idx, cnt)]
+    for _ in range(3):
+        again = api.backward(desc, qd, kd, vd, O, lse, go, idx, cnt)
+        torch.cuda.synchronize()
+        for a, b in zip(first, again):
+            assert torch.equal(a, b)
+    assert api.get_status() == api.SSBA_OK
+
+
 def test_backward_after_gpu_forward():
     """The training order: GPU mask, GPU forward, then the backward on the forward's own O
     and lse, against the oracle backward on the same lists."""
