@@ -349,6 +349,20 @@ SSBA_API int ssba_test_fused_timeout(const ssba_desc* desc, const void* Q, const
                                      float* kb, int32_t* kv_idx, int32_t* kv_cnt, void* O, float* lse,
                                      void* workspace, size_t ws_bytes, uint64_t budget_ns, void* stream);
 
+/* Test hook for failure detection in the backward (no counterpart in the paper): runs the
+ * persistent tensor-core kernel of ssba_backward with every wait limited to budget_ns of wall
+ * time (clamped to [1 ms, 2 s]) and CTA 0 announcing its first pair's tile copies without
+ * issuing them, so that the waits on them run out. That CTA stops all its roles, waits
+ * (bounded) for its own copies and MMAs in flight, frees its tensor memory and returns; the
+ * other CTAs finish their items. The device status word reads SSBA_ERR_TIMEOUT (ssba_get_status,
+ * after a synchronize), dQ, dK and dV are undefined, and the context stays usable. No fault,
+ * trap or endless wait is involved. Arguments as ssba_backward (workspace required); bf16,
+ * head_dim 64, shifts that are multiples of 4 and Tb <= 256, else SSBA_ERR_UNSUPPORTED. */
+SSBA_API int ssba_test_backward_timeout(const ssba_desc* desc, const void* Q, const void* K, const void* V,
+                                        const void* O, const float* lse, const void* dO, const int32_t* kv_idx,
+                                        const int32_t* kv_cnt, float* dQ, float* dK, float* dV, void* workspace,
+                                        size_t ws_bytes, uint64_t budget_ns, void* stream);
+
 /* Reads and clears the device status word of the current device (SSBA_OK or
  * SSBA_ERR_TIMEOUT). Synchronous: call after the caller's stream sync. Returns
  * SSBA_OK, or SSBA_ERR_CUDA if the read failed. */

@@ -28,7 +28,7 @@ _STATUS_NAMES = {0: "SSBA_OK", 1: "SSBA_ERR_INVALID", 2: "SSBA_ERR_UNSUPPORTED",
 
 EXPORTED = ("ssba_keep_count", "ssba_mask_workspace_bytes", "ssba_build_mask", "ssba_build_mask_noalloc",
             "ssba_forward", "ssba_forward_joint", "ssba_forward_workspace_bytes", "ssba_forward_dense",
-            "ssba_test_forward_timeout", "ssba_test_fused_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
+            "ssba_test_forward_timeout", "ssba_test_fused_timeout", "ssba_test_backward_timeout", "ssba_backward", "ssba_backward_workspace_bytes", "ssba_haar_dwt",
             "ssba_haar_iwt", "ssba_haar_dwt_pyramid", "ssba_haar_iwt_pyramid", "ssba_qkv_rope_pool",
             "ssba_select_mask", "ssba_pool_blocks", "ssba_forward_select", "ssba_forward_fused",
             "ssba_get_status", "ssba_last_error", "ssba_timeline_read")
@@ -134,6 +134,9 @@ def load_library(path: str | None = None):
         lib.ssba_test_fused_timeout.restype = ctypes.c_int
         lib.ssba_backward.argtypes = [DP, P, P, P, P, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
         lib.ssba_backward.restype = ctypes.c_int
+        lib.ssba_test_backward_timeout.argtypes = [DP, P, P, P, P, P, P, P, P, P, P, P, P, ctypes.c_size_t,
+                                                   ctypes.c_uint64, P]
+        lib.ssba_test_backward_timeout.restype = ctypes.c_int
         lib.ssba_backward_workspace_bytes.argtypes = [DP]
         lib.ssba_backward_workspace_bytes.restype = ctypes.c_size_t
         I = ctypes.c_int32
@@ -566,8 +569,10 @@ def backward_workspace_bytes(desc: SsbaDesc) -> int:
 
 
 def backward(desc: SsbaDesc, Q, K, V, O, lse, dO, kv_idx, kv_cnt, dQ=None, dK=None, dV=None, workspace=None,
-             stream=None):
-    """ssba_backward: gradients (dQ, dK, dV) in fp32 of the sparse forward for output gradient dO."""
+             stream=None, _timeout_budget_ns=None):
+    """ssba_backward: gradients (dQ, dK, dV) in fp32 of the sparse forward for output gradient dO.
+    With _timeout_budget_ns set it calls the failure-detection test hook ssba_test_backward_timeout
+    instead (see include/ssba.h): the gradients are then undefined."""
     lib = load_library()
     d = desc.c()
     keep = lib.ssba_keep_count(ctypes.byref(d))
@@ -589,11 +594,20 @@ def backward(desc: SsbaDesc, Q, K, V, O, lse, dO, kv_idx, kv_cnt, dQ=None, dK=No
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=Q.device)
     wp, wn = _ws_args(workspace)
-    rc = lib.ssba_backward(ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), O.data_ptr(), lse.data_ptr(),
-                           dO.data_ptr(), kv_idx.data_ptr(), kv_cnt.data_ptr(), outs[0].data_ptr(),
-                           outs[1].data_ptr(), outs[2].data_ptr(), wp, wn, _stream_ptr(stream))
+    args = (ctypes.byref(d), Q.data_ptr(), K.data_ptr(), V.data_ptr(), O.data_ptr(), lse.data_ptr(), dO.data_ptr(),
+            kv_idx.data_ptr(), kv_cnt.data_ptr(), outs[0].data_ptr(), outs[1].data_ptr(), outs[2].data_ptr(), wp, wn)
+    if _timeout_budget_ns is None:
+        rc = lib.ssba_backward(*args, _stream_ptr(stream))
+    else:
+        rc = lib.ssba_test_backward_timeout(*args, int(_timeout_budget_ns), _stream_ptr(stream))
     _raise_on(rc)
     return tuple(outs)
+
+
+def test_backward_timeout(desc: SsbaDesc, Q, K, V, O, lse, dO, kv_idx, kv_cnt, budget_ns: int = 2_000_000,
+                          stream=None) -> None:
+    """ssba_test_backward_timeout: the backward's failure-detection test hook (include/ssba.h)."""
+    backward(desc, Q, K, V, O, lse, dO, kv_idx, kv_cnt, stream=stream, _timeout_budget_ns=budget_ns)
 
 
 def _dtype_code(t: torch.Tensor) -> int:

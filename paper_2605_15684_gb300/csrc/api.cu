@@ -555,6 +555,40 @@ int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, const voi
                            static_cast<float*>(workspace), static_cast<cudaStream_t>(stream));
 }
 
+int ssba_test_backward_timeout(const ssba_desc* desc, const void* Q, const void* K, const void* V, const void* O,
+                               const float* lse, const void* dO, const int32_t* kv_idx, const int32_t* kv_cnt,
+                               float* dQ, float* dK, float* dV, void* workspace, size_t ws_bytes, uint64_t budget_ns,
+                               void* stream)
+{
+    Grid g;
+    int keep;
+    int rc = check_desc(desc, "ssba_test_backward_timeout", &g, &keep);
+    if (rc != SSBA_OK) return rc;
+    if (!Q || !K || !V || !O || !lse || !dO || !kv_idx || !kv_cnt || !dQ || !dK || !dV) {
+        set_error("ssba_test_backward_timeout: every pointer must be non-null");
+        return SSBA_ERR_INVALID;
+    }
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(dO, 16) ||
+        !aligned(lse, 4) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) || !aligned(dQ, 16) || !aligned(dK, 16) ||
+        !aligned(dV, 16)) {
+        set_error("ssba_test_backward_timeout: tensors 16-byte aligned; lse, kv_idx, kv_cnt 4-byte aligned");
+        return SSBA_ERR_INVALID;
+    }
+    const size_t need = ssba_backward_workspace_bytes(desc);
+    if (!workspace || ws_bytes < need || !aligned(workspace, 16)) {
+        set_error("ssba_test_backward_timeout: workspace of %zu bytes (16-byte aligned) required, got %zu", need,
+                  ws_bytes);
+        return SSBA_ERR_WORKSPACE;
+    }
+    const uint64_t b = budget_ns < 1000000ull ? 1000000ull : (budget_ns > kWaitBudgetNs ? kWaitBudgetNs : budget_ns);
+    rc = launch_backward_ws(*desc, g, keep, resolve_scale(desc), Q, K, V, O, lse, dO, kv_idx, kv_cnt, dQ, dK, dV,
+                            workspace, static_cast<cudaStream_t>(stream), b, 1);
+    if (rc == SSBA_ERR_UNSUPPORTED)
+        set_error("ssba_test_backward_timeout: needs the persistent kernel (bf16, head_dim 64, shifts that are "
+                  "multiples of 4, Tb <= 256)");
+    return rc;
+}
+
 static int haar_args(const char* who, const void* in, const void* out, int N, int C, int H, int W, int nb,
                      int dtype)
 {

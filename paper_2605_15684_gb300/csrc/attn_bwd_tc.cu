@@ -663,6 +663,7 @@ int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale,
     p.Dbuf = Dbuf;
     p.ctr = p.toff = p.tcnt = p.tlist = nullptr;
     p.ld = nullptr;
+    p.withhold = 0;
     p.g = g;
     p.keep = keep;
     p.scale = scale;

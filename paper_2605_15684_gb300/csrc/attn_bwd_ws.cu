@@ -183,12 +183,17 @@ __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, cons
             if (P >= kRing && !warp_wait(smem_u32(&sm.tile_empty[r]), ((P / kRing) + 1) & 1, abortf, p.budget_ns))
                 return false;
             const int j = sm.list[s][t];
+            // test hook: CTA 0 announces its first pair's bytes and copies nothing, so that the
+            // waits on them run out
+            const bool hold = p.withhold == 1 && P == 0 && blockIdx.x == 0;
             if (lane == 0) {
                 const uint32_t bar = smem_u32(&sm.tile_full[r]), e = sm.win[j];
                 mbar_arrive_expect_tx(bar, 2 * kTile + (role ? kLdRow : 0));
-                window_boxes_e(role ? maps.q : maps.k, smem_u32(sm.x[r]), bar, e, bh);
-                window_boxes_e(role ? maps.o : maps.v, smem_u32(sm.y[r]), bar, e, bh);
-                if (role) bulk_load(smem_u32(sm.pld[r]), p.ld + ((size_t)bh * Tb + j) * kT, kLdRow, bar);
+                if (!hold) {
+                    window_boxes_e(role ? maps.q : maps.k, smem_u32(sm.x[r]), bar, e, bh);
+                    window_boxes_e(role ? maps.o : maps.v, smem_u32(sm.y[r]), bar, e, bh);
+                    if (role) bulk_load(smem_u32(sm.pld[r]), p.ld + ((size_t)bh * Tb + j) * kT, kLdRow, bar);
+                }
             }
         }
         int next = 0;
@@ -471,7 +476,8 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_bwd_ws_kernel(const __grid_c
 
 int launch_backward_ws(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
                        const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
-                       const int32_t* cnt, float* dQ, float* dK, float* dV, void* workspace, cudaStream_t st)
+                       const int32_t* cnt, float* dQ, float* dK, float* dV, void* workspace, cudaStream_t st,
+                       uint64_t budget_ns, int withhold)
 {
     if (d.head_dim != kD || g.blk != 8 || d.dtype != SSBA_BF16 || g.Tb() > 256 || (g.sr % 4) || (g.sc % 4))
         return SSBA_ERR_UNSUPPORTED;
@@ -503,7 +509,8 @@ int launch_backward_ws(const ssba_desc& d, const Grid& g, int keep, float scale,
     p.g = g;
     p.keep = keep;
     p.scale = scale;
-    p.budget_ns = kWaitBudgetNs;
+    p.budget_ns = budget_ns;
+    p.withhold = withhold;
     p.status = device_status_word();
     if (!p.status) {
         set_error("ssba_backward: could not resolve the device status word");

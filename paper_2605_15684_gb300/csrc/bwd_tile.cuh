@@ -77,6 +77,8 @@ struct BwdParams {
     float scale;
     int* status;
     uint64_t budget_ns;
+    int withhold;  // failure-detection test hook: 1, CTA 0 announces its first pair's tiles
+                   // and never copies them (ssba_test_backward_timeout)
 };
 
 // Byte offsets in the ssba_backward workspace: D of every row first (every path), then the

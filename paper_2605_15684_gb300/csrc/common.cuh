@@ -144,7 +144,8 @@ int launch_backward_tc(const ssba_desc& d, const Grid& g, int keep, float scale,
 // ssba_backward workspace (bwd_layout).
 int launch_backward_ws(const ssba_desc& d, const Grid& g, int keep, float scale, const void* Q, const void* K,
                        const void* V, const void* O, const float* lse, const void* dO, const int32_t* idx,
-                       const int32_t* cnt, float* dQ, float* dK, float* dV, void* workspace, cudaStream_t st);
+                       const int32_t* cnt, float* dQ, float* dK, float* dV, void* workspace, cudaStream_t st,
+                       uint64_t budget_ns = kWaitBudgetNs, int withhold = 0);
 
 int launch_haar(bool inverse, const void* in, void* out, int N, int C, int H, int W, int nb, int dtype,
                 cudaStream_t st);

@@ -4,7 +4,8 @@ issues, so the waits on that tile run out; the kernel must stop, drain what it i
 free its tensor memory and report SSBA_ERR_TIMEOUT in the device status word, and the
 CUDA context must stay usable (a normal forward right after matches the oracle). A second
 hook makes one CTA of the fused launch withhold its arrival at the grid barrier, so that
-every CTA's barrier wait runs out, with the same requirements."""
+every CTA's barrier wait runs out, with the same requirements. A third makes one CTA of the
+persistent backward announce a pair's tile copies without issuing them."""
 import pytest
 import torch
 
@@ -76,3 +77,36 @@ def test_grid_barrier_timeout_reports_status_and_context_survives():
     assert api.get_status() == api.SSBA_OK
     assert torch.equal(i2, i3) and torch.equal(O2, O3) and torch.equal(l2, l3)
     assert int(ws[-256:].count_nonzero()) == 0
+
+
+def test_backward_timeout_reports_status_and_context_survives():
+    """CTA 0 of the persistent backward never receives its first pair's tiles: its issuers'
+    waits run out, it drains and reports SSBA_ERR_TIMEOUT, the other CTAs finish; a normal
+    backward right after matches the oracle."""
+    build.build()
+    api.load_library()
+    H = W = 32
+    q, k, v = synthetic.qkv(1, 4, H * W, 64, torch.bfloat16, 13)
+    go = synthetic.qkv(1, 4, H * W, 64, torch.bfloat16, 113)[0]
+    desc = api.SsbaDesc(1, 4, H, W, shift_r=4, shift_c=4, rho=0.75)
+    qd, kd, vd, god = q.cuda(), k.cuda(), v.cuda(), go.cuda()
+    idx_o, cnt_o = oracle.build_mask(q, k, H, W, 8, (4, 4), 0.75)
+    O_o, lse_o = oracle.forward(q, k, v, idx_o, H, W, 8, (4, 4))
+    idx, cnt = torch.from_numpy(idx_o).cuda(), torch.from_numpy(cnt_o).cuda()
+    O = torch.from_numpy(O_o).to(torch.bfloat16).cuda()
+    lse = torch.from_numpy(lse_o).float().cuda()
+    torch.cuda.synchronize()
+    assert api.get_status() == api.SSBA_OK
+
+    api.test_backward_timeout(desc, qd, kd, vd, O, lse, god, idx, cnt, budget_ns=2_000_000)
+    torch.cuda.synchronize()  # the kernel returns: no hang, no CUDA error
+    assert api.get_status() == api.SSBA_ERR_TIMEOUT
+    assert api.get_status() == api.SSBA_OK
+
+    grads = api.backward(desc, qd, kd, vd, O, lse, god, idx, cnt)
+    torch.cuda.synchronize()
+    ref = oracle.backward(q, k, v, go, idx_o, H, W, 8, (4, 4))
+    for got, want in zip(grads, ref):  # the bf16 bound of the parity tests
+        g = got.cpu().double().numpy()
+        assert abs(g - want).max() / max(1.0, abs(want).max()) <= 5e-3
+    assert api.get_status() == api.SSBA_OK
