@@ -232,7 +232,9 @@ SSBA_API int ssba_forward_select(const ssba_desc* desc, const void* Q, const voi
  *   the rest    as ssba_forward_select.
  * The barrier needs every CTA of the grid (one per SM, at most the SM count) resident at once:
  * work on other streams that holds SMs for longer than the wait budget (2 s) makes the call end
- * with SSBA_ERR_TIMEOUT instead of waiting for it.
+ * with SSBA_ERR_TIMEOUT instead of waiting for it. The fallback with no grid-wide wait is
+ * ssba_pool_blocks then ssba_forward_select on the same buffers (the same means, lists and
+ * outputs); after SSBA_ERR_TIMEOUT, zero the workspace again before the next fused call.
  * bf16 only; Tb <= 256 (else SSBA_ERR_UNSUPPORTED); SSBA_ERR_WORKSPACE without a workspace. */
 SSBA_API int ssba_forward_fused(const ssba_desc* desc, const void* Q, const void* K, const void* V, float* qb,
                                 float* kb, int32_t* kv_idx, int32_t* kv_cnt, float* scores_opt, void* O,
