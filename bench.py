@@ -525,7 +525,35 @@ def run_ours(args, rank, world):
         torch.cuda.synchronize()
         tb = e0.elapsed_time(e1) / reps
         F_b = 2.5 * F_layer
+        # the same call at 2048 px (rows of 41 kept blocks of 256), one layer with its own mask
+        # and forward, outside the timed region
+        big = None
+        try:
+            wb = synthetic.PX2048
+            db = api.SsbaDesc(wb.B, wb.heads, wb.H_tok, wb.W_tok, shift_r=4, shift_c=4, rho=wb.rho, dtype=wb.dtype)
+            qb_, kb_, vb_ = (t.to(dev) for t in synthetic.qkv(wb.B, wb.heads, wb.N, wb.head_dim, wb.dtype,
+                                                               seed=900 + 1000 * rank, std=wb.std))
+            gob = synthetic.qkv(wb.B, wb.heads, wb.N, wb.head_dim, wb.dtype, seed=901 + 1000 * rank)[0].to(dev)
+            ib, cb = api.build_mask(db, qb_, kb_)
+            Ob, lb = api.forward(db, qb_, kb_, vb_, ib, cb)
+            wsbb = torch.empty(api.backward_workspace_bytes(db), dtype=torch.uint8, device=dev)
+            gb = [torch.empty((wb.B, wb.heads, wb.N, wb.head_dim), dtype=torch.float32, device=dev) for _ in range(3)]
+            api.backward(db, qb_, kb_, vb_, Ob, lb, gob, ib, cb, *gb, workspace=wsbb)
+            e0.record(stream)
+            for _ in range(4):
+                api.backward(db, qb_, kb_, vb_, Ob, lb, gob, ib, cb, *gb, workspace=wsbb)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            tbb = e0.elapsed_time(e1) / 4
+            keep_b = api.keep_count(db)
+            F_bb = 2.5 * kept_flops(wb.B, wb.heads, db.Tb, keep_b, wb.head_dim)
+            big = {"config": wb.name, "keep": keep_b, "Tb": db.Tb, "ms_per_layer": tbb,
+                   "effective_tflops": F_bb / (tbb * 1e-3) / 1e12, "flops_per_layer": F_bb}
+            del qb_, kb_, vb_, gob, Ob, lb, wsbb, gb
+        except Exception as exc:  # reported, not fatal
+            big = f"failed: {exc}"
         bwd = {"ms_per_layer": tb, "effective_tflops": F_b / (tb * 1e-3) / 1e12, "flops_per_layer": F_b,
+               "px2048": big,
                "how": "ssba_backward per layer (a row kernel: D, the rows' (lse, D) by block, the key "
                       "blocks' transposed lists; then the persistent warp-specialised tcgen05 kernel, "
                       "dQ per query block and dK, dV per key block) on the layer's forward O and lse "

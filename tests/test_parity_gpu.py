@@ -390,6 +390,14 @@ def test_backward_bf16(H, W, h, rho, shift):
     _bwd_case_gpu(1, h, H, W, rho, shift, torch.bfloat16, 31)
 
 
+@pytest.mark.parametrize("B,H,W,h,rho,shift", [(2, 32, 32, 3, 0.75, (4, 4)),
+                                              # 256 blocks a head (the 2048 px grid): long rows
+                                              # and key blocks kept by many query blocks
+                                              (1, 128, 128, 2, 0.84, (4, 4))])
+def test_backward_bf16_batches_and_long_rows(B, H, W, h, rho, shift):
+    _bwd_case_gpu(B, h, H, W, rho, shift, torch.bfloat16, 34)
+
+
 def test_backward_is_deterministic():
     """Repeated calls give bitwise-equal gradients: no atomics, and the work counter only decides
     which CTA runs an item, not the order of any sum (1024 px layer, 24 heads, shift 4)."""
