@@ -226,9 +226,8 @@ __device__ __forceinline__ bool issue_acc(const BwdParams& p, WsSmem& sm, uint32
 
 // Lane 0 of warp 8 (which = 0) or 9 (which = 1): the products of one side of every pair, so
 // that two threads share the issue latency of a tcgen05.mma (about 57 cycles from one thread,
-// 44 a product when several issue). Returns false on a timeout; `issued` tells the teardown
-// that MMAs may be in flight.
-__device__ bool issue(const BwdParams& p, WsSmem& sm, const int which, bool& issued)
+// 44 a product when several issue). Returns false on a timeout.
+__device__ bool issue(const BwdParams& p, WsSmem& sm, const int which)
 {
     volatile int* abortf = &sm.abort_flag;
     const uint32_t tb0 = sm.tmem_base;
@@ -261,7 +260,6 @@ __device__ bool issue(const BwdParams& p, WsSmem& sm, const int which, bool& iss
             else
                 mma_kk(tb0 + kColDP, ab, smem_u32(sm.y[r]));  // dP = dO V^T (dP^T = V dO^T)
             mma_commit(smem_u32(&sm.bar_s));
-            issued = true;
             if (t == n - 1) mma_commit(smem_u32(&sm.ab_empty[s]));
             if (pending && !issue_acc(p, sm, P - 1, prole, pfirst, which)) return false;
             pending = true;
@@ -432,13 +430,13 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_bwd_ws_kernel(const __grid_c
     __syncthreads();
     tc_fence_after();
 
-    bool ok = true, issued = false;
+    bool ok = true;
     uint32_t P = 0;
     int kab = 0;
     if (warp < kCompute / 32)
         ok = compute(p, sm);
     else if (threadIdx.x == kIssuer0 || threadIdx.x == kIssuer1)
-        ok = issue(p, sm, threadIdx.x == kIssuer1 ? 1 : 0, issued);
+        ok = issue(p, sm, threadIdx.x == kIssuer1 ? 1 : 0);
     else if (warp == kProducer)
         ok = produce(maps, p, sm, nk, P, kab);
     const bool dead = __syncthreads_or(!ok);
