@@ -16,16 +16,17 @@
 //   warp 1      QK issuer (one elected lane; warp 1 of the CTA also owns the TMEM allocation):
 //                 S_t = Q K_t^T   tcgen05.mma kind::f16, M=64 N=64, A = Q tile and
 //                                 B = K tile from shared memory (K-major, SW128)
-//               S is double-buffered in TMEM: QK of block t waits only until the softmax
-//               has loaded S_{t-2} into registers.
+//               S is triple-buffered in TMEM: QK of block t waits only until PV_{t-3} has
+//               read P_{t-3} from the same buffer.
 //   warp 2      TMA producer of the V ring (warp 0 keeps Q and K), so that two threads
 //               share the per-box issue latency.
 //   warp 3      PV issuer (one elected lane):
 //                 O  += P_t V_t   tcgen05.mma kind::f16, M=64 N=64, A = P from TMEM,
 //                                 B = V tile (MN-major, SW128)
-//               P has its own two TMEM buffers (bf16 pairs, 32 columns each), so an S
-//               buffer is not held while its P waits for the PV. TMEM of a pipeline:
-//               S 2 x 64 + P 2 x 32 + O 64 = 256 columns. Two issuing threads keep one's
+//               P_t (bf16 pairs, 32 columns) goes into the first half of S_t's buffer, which
+//               the softmax no longer needs once S_t is in its registers, so the softmax never
+//               waits for a P buffer and QK runs up to three blocks ahead. TMEM of a
+//               pipeline: S/P 3 x 64 + O 64 = 256 columns. Two issuing threads keep one's
 //               barrier waits (about 100 cycles per query) off the other's issue path.
 //   warps 4-7   softmax, one TMEM lane quadrant each. The M=64 data path puts tile row r
 //               at lane 32*(r/16) + r%16, so two threads share a row (16x32bx2 TMEM
@@ -63,15 +64,14 @@ constexpr int kD = 64;
 constexpr int kRows = 64;  // query rows per item = tokens per block
 constexpr int kKStages = 5;  // K ring
 constexpr int kVStages = 5;  // V ring
-constexpr int kSBuf = 2;     // S buffers in TMEM (fp32, 64 columns each)
-constexpr int kPBuf = 2;     // P buffers in TMEM (bf16 pairs, 32 columns each)
+constexpr int kSBuf = 3;     // S buffers in TMEM (fp32, 64 columns each); P_t (bf16 pairs) goes
+                             // into the first 32 columns of S_t's buffer
 constexpr int kSlotWarps = 12;                // warps of one pipeline (see the role map above)
 constexpr int kSlots = 2;                     // independent pipelines per CTA
 constexpr int kThreads = kSlots * kSlotWarps * 32;
 constexpr uint32_t kSlotCols = 256;           // TMEM columns of one pipeline
 constexpr uint32_t kTmemCols = kSlots * kSlotCols;
-constexpr uint32_t kColS = 0;    // S buffers: [0,64), [64,128)
-constexpr uint32_t kColP = 128;  // P buffers: [128,160), [160,192)
+constexpr uint32_t kColS = 0;    // S / P buffers: [0,64), [64,128), [128,192)
 constexpr uint32_t kColO = 192;  // O accumulator: [192,256)
 constexpr uint32_t kTileBytes = kRows * kD * 2;  // 8 KB
 constexpr float kRescaleLog2 = 8.0f;
@@ -96,9 +96,9 @@ struct __align__(1024) SlotSmem {
     uint64_t q_full[2];
     uint64_t q_empty[2];
     uint64_t s_full[kSBuf];
-    uint64_t s_free[kSBuf];   // the softmax has loaded S_t: QK_{t+2} may overwrite it
-    uint64_t p_full[kPBuf];
-    uint64_t p_empty[kPBuf];  // PV_t has finished (it read P_t; O holds it)
+    uint64_t s_free[kSBuf];   // PV_t has finished (it read P_t from S_t's buffer): QK_{t+3} may
+                              // overwrite the buffer
+    uint64_t p_full[kSBuf];
     uint64_t stats_full[2];
     uint64_t stats_free[2];
     uint64_t o_full;
@@ -547,11 +547,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         }
         for (int b = 0; b < kSBuf; ++b) {
             mbar_init(smem_u32(&sm.s_full[b]), 1);
-            mbar_init(smem_u32(&sm.s_free[b]), 4);
-        }
-        for (int b = 0; b < kPBuf; ++b) {
+            mbar_init(smem_u32(&sm.s_free[b]), 1);
             mbar_init(smem_u32(&sm.p_full[b]), 4);
-            mbar_init(smem_u32(&sm.p_empty[b]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&sm.q_full[b]), 1);
@@ -810,7 +807,7 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
         __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------------------ QK issuer
-        // S_t = Q K_t^T into S buffer t % 3, once the softmax has loaded S_{t-3} from it.
+        // S_t = Q K_t^T into S buffer t % 3, once PV_{t-3} has read P_{t-3} from it.
         // MMAs and commits are issued under an elect.sync taken at the issue site: the
         // compiler then keeps the descriptors on the uniform datapath (measured: 4 MMAs +
         // commit issue in about 280 cycles, against about 480 under a precomputed lane test).
@@ -875,8 +872,8 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
             const Piece pc = get_piece(p, sm, pi, vcta, vgrid);
             const int nblk = pc.nb;
             for (int t = 0; t < nblk; ++t) {
-                const uint32_t gb = gblk + t, pb = gb % kPBuf, slot = gb % kVStages;
-                if (!mbar_wait(smem_u32(&sm.p_full[pb]), (gb / kPBuf) & 1, abortf, p.budget_ns)) {
+                const uint32_t gb = gblk + t, pb = gb % kSBuf, slot = gb % kVStages;
+                if (!mbar_wait(smem_u32(&sm.p_full[pb]), (gb / kSBuf) & 1, abortf, p.budget_ns)) {
                     dead = true;
                     break;
                 }
@@ -893,13 +890,13 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 tc_fence_after();
                 if (elect_one_sync()) {
                     const uint64_t vdesc = sdesc_sw128(vbase + slot * kTileBytes, 8192, 1024);
-                    const uint32_t pcol = tbase + kColP + pb * 32;
+                    const uint32_t pcol = tbase + kColS + pb * 64;
 #pragma unroll
                     for (int k = 0; k < 4; ++k)
                         mma_ts(tbase + kColO, pcol + k * 8, vdesc + (uint64_t)(k * 128), kIdescPV,
                                (t > 0 || k > 0) ? 1u : 0u);
                     mma_commit(smem_u32(&sm.v_empty[slot]));
-                    mma_commit(smem_u32(&sm.p_empty[pb]));
+                    mma_commit(smem_u32(&sm.s_free[pb]));
                     TL_TILE(gwarp / kSlotWarps, gb, tl::kPVIssue);
                 }
                 __syncwarp();
@@ -954,10 +951,6 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                         for (int i = 0; i < 32; ++i)
                             if (half * 32 + i >= valid) sr[i] = __float_as_uint(-INFINITY);
                 }
-                // S_t is in registers: QK_{t+2} may overwrite its buffer
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&sm.s_free[sb]));
                 float mx;
                 {
                     float t8[8];
@@ -1002,19 +995,14 @@ __global__ void __maxnreg__(80) ssba_attn_tc_kernel(const __grid_constant__ Tile
                 const float2 lsum = __fadd2_rn(ls2[0], ls2[1]);
                 l = fmaf(l, alpha, lsum.x + lsum.y);
                 if (quad == 0 && lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kSmxExp);
-                // P_t (bf16 pairs) into its TMEM buffer once PV_{t-2} has finished reading it
-                const uint32_t pb = gb % kPBuf;
-                if (gb >= (uint32_t)kPBuf &&
-                    !mbar_wait(smem_u32(&sm.p_empty[pb]), ((gb / kPBuf) - 1) & 1, abortf, p.budget_ns)) {
-                    dead = true;
-                    break;
-                }
+                // P_t (bf16 pairs) into the first half of S_t's buffer, which S_t no longer needs
                 if (quad == 0 && lane == 0) TL_TILE(gwarp / kSlotWarps, gb, tl::kPFree);
-                tmem_st_16x32bx2_x16_off16(tbase + lane_off + kColP + pb * 32, pk);
+                const uint32_t pb = sb;
+                tmem_st_16x32bx2_x16_off16(tbase + lane_off + kColS + pb * 64, pk);
                 if (rescale) {
                     // O must hold every earlier PV before it is rescaled; PV_t waits for p_full
-                    const uint32_t qb = (gb - 1) % kPBuf;
-                    if (!mbar_wait(smem_u32(&sm.p_empty[qb]), ((gb - 1) / kPBuf) & 1, abortf, p.budget_ns)) {
+                    const uint32_t qb = (gb - 1) % kSBuf;
+                    if (!mbar_wait(smem_u32(&sm.s_free[qb]), ((gb - 1) / kSBuf) & 1, abortf, p.budget_ns)) {
                         dead = true;
                         break;
                     }
