@@ -7,16 +7,16 @@
 // Work items: a key block's dK, dV or a query block's dQ, of one (batch, head). The first item
 // of a CTA is its index; the others come from a counter in the workspace that the row kernel
 // zeroes. Key-block items come first (their lengths vary), query-block items fill in behind.
-//   warp 10    producer: publishes each item (role, head, block, count and its list of other
+//   warp 11    producer: publishes each item (role, head, block, count and its list of other
 //              blocks: the forward's list for dQ, the transposed list the row kernel built for
 //              dK, dV) in one of two item slots; copies the item's resident tiles by TMA (two
 //              buffers, by item parity) and each pair's streamed tiles (a ring of three), each
 //              with the 512-byte row of (lse, D) values of its block that the compute warps
 //              use (the row kernel writes them by block, in tile order: one bulk copy).
-//   warps 8-9  lane 0 of each issues one side of the MMAs (S and the products reading the
-//              pair's x tile; dP and the one reading its y tile): per pair S, dP into the same
-//              TMEM columns once the compute warps hold the last ones in registers, then the
-//              accumulating products of the previous pair once its bf16 operands are stored.
+//   warps 8-10 lane 0 of each issues a share of the MMAs: warp 8 S and dK += dS^T Q, warp 9
+//              dP and dV += P^T dO, warp 10 dQ += dS K. Per pair S, dP go into the same TMEM
+//              columns once the compute warps hold the last ones in registers; the
+//              accumulating products of a pair follow once its bf16 operands are stored.
 //   warps 0-7  the exps and the bf16 operands of each pair, two warps per TMEM lane quadrant
 //              (16 of a row's 64 columns a thread), and each item's epilogue (the accumulators
 //              to global memory, fp32).
@@ -41,11 +41,13 @@ using namespace win;
 using namespace bwd;
 
 constexpr int kCompute = 256;   // warps 0-7, two per TMEM lane quadrant
-constexpr int kIssuer0 = 256;   // lane 0 of warp 8: S and the products that read the x tiles
-constexpr int kIssuer1 = 288;   // lane 0 of warp 9: dP and the products that read the y tiles
-constexpr int kIssuers = 2;
-constexpr int kProducer = 10;   // warp
-constexpr int kThreads = 352;
+constexpr int kIssuer0 = 256;   // lane 0 of warp 8: S, and dK += dS^T Q
+constexpr int kIssuer1 = 288;   // lane 0 of warp 9: dP, and dV += P^T dO
+constexpr int kIssuer2 = 320;   // lane 0 of warp 10: dQ += dS K
+constexpr int kIssuers = 3;     // commit to bar_a, tile_empty, drain
+constexpr int kSdpIssuers = 2;  // commit to bar_s, ab_empty
+constexpr int kProducer = 11;   // warp
+constexpr int kThreads = 384;
 constexpr int kRing = 3;        // streamed tile slots
 constexpr int kDone = -1;       // role of the item slot that ends a CTA's work
 constexpr uint32_t kTmemCols = 256;
@@ -68,15 +70,15 @@ struct alignas(1024) WsSmem {
     uint32_t win[256];        // label -> packed window entry (window_entry)
     int4 info[2];             // role (0 dQ, 1 dK/dV, kDone), bh, label, n
     uint64_t item_full[2];    // producer lane 0, after the slot is written
-    uint64_t item_empty[2];   // the 8 compute warps and the 2 issuers have read the slot
+    uint64_t item_empty[2];   // the 8 compute warps and the 3 issuers have read the slot
     uint64_t ab_full[2];      // TMA bytes of the item tiles (and, for dQ, of its ild row)
-    uint64_t ab_empty[2];     // MMA commits (both issuers) after the item's last S, dP
+    uint64_t ab_empty[2];     // MMA commits (the S and dP issuers) after the item's last S, dP
     uint64_t tile_full[kRing];   // TMA bytes of a pair's tiles (and, for dK/dV, of its pld row)
-    uint64_t tile_empty[kRing];  // MMA commits (both issuers) after the pair's products
-    uint64_t bar_s;           // MMA commits (both issuers): S, dP of the pair in TMEM
+    uint64_t tile_empty[kRing];  // MMA commits (all three issuers) after the pair's products
+    uint64_t bar_s;           // MMA commits (the S and dP issuers): S, dP of the pair in TMEM
     uint64_t s_free;          // 8 compute warps: S, dP in registers
     uint64_t e_full;          // 8 compute warps: the pair's bf16 operands stored
-    uint64_t bar_a;           // MMA commits (both issuers): the pair's accumulating products
+    uint64_t bar_a;           // MMA commits (all three issuers): the pair's accumulating products
     uint64_t drain;
     uint32_t tmem_base;
     int abort_flag;
@@ -126,7 +128,7 @@ __device__ __forceinline__ int4 decode_item(int w, int nk, int Tb)
     return make_int4(key ? 1 : 0, bh, u - bh * Tb, 0);
 }
 
-// Warp 10. nk = number of key-block items (B * heads * Tb), total = 2 nk. Returns false on a
+// Warp 11. nk = number of key-block items (B * heads * Tb), total = 2 nk. Returns false on a
 // timeout. P counts the pairs whose tiles were issued, kab the items whose tiles were issued
 // (after a timeout the teardown waits for the last copies of each barrier).
 __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, const int nk, uint32_t& P, int& kab)
@@ -203,30 +205,54 @@ __device__ bool produce(const WsMaps& maps, const BwdParams& p, WsSmem& sm, cons
 }
 
 // Issuer `which`'s share of the accumulating products of pair q (its role, and whether it opens
-// its item), once the pair's bf16 operands are stored: issuer 0 dQ += dS K or dK += dS^T Q
-// (x tiles), issuer 1 dV += P^T dO (y tiles). Each commits, so the barriers count two.
+// its item), once the pair's bf16 operands are stored: for a key-block pair issuer 0
+// dK += dS^T Q (x tile), issuer 1 dV += P^T dO (y tile); nothing for a query-block pair, whose
+// dQ is issuer 2's. Each commits, so bar_a and tile_empty count three.
 __device__ __forceinline__ bool issue_acc(const BwdParams& p, WsSmem& sm, uint32_t q, int role, bool first, int which)
 {
     if (!mbar_wait(smem_u32(&sm.e_full), q & 1, &sm.abort_flag, p.budget_ns)) return false;
     tc_fence_after();
     const uint32_t tb0 = sm.tmem_base;
     const int r = (int)(q % kRing);
-    if (which == 0) {
-        if (role == 1)
+    if (role == 1) {
+        if (which == 0)
             mma_sb(tb0 + kColA1, smem_u32(sm.e[1]), smem_u32(sm.x[r]), !first);  // dK += dS^T Q
         else
-            mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.x[r]), !first);  // dQ += dS K
-    } else if (role == 1) {
-        mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.y[r]), !first);  // dV += P^T dO
+            mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.y[r]), !first);  // dV += P^T dO
     }
     mma_commit(smem_u32(&sm.bar_a));
     mma_commit(smem_u32(&sm.tile_empty[r]));
     return true;
 }
 
-// Lane 0 of warp 8 (which = 0) or 9 (which = 1): the products of one side of every pair, so
-// that two threads share the issue latency of a tcgen05.mma (about 57 cycles from one thread,
-// 44 a product when several issue). Returns false on a timeout.
+// Lane 0 of warp 8 (which = 0) or 9 (which = 1): S or dP of every pair and its share of the
+// accumulating products, so that the issue latency of a tcgen05.mma (about 57 cycles from one
+// thread, 44 a product when several issue) is shared. Returns false on a timeout.
+// Lane 0 of warp 10: dQ += dS K of every query-block pair, in pair order, once its operands are
+// stored; for key-block pairs it only commits (bar_a and tile_empty count three commits).
+__device__ bool issue_dq(const BwdParams& p, WsSmem& sm)
+{
+    volatile int* abortf = &sm.abort_flag;
+    const uint32_t tb0 = sm.tmem_base;
+    uint32_t P = 0;
+    for (int k = 0;; ++k) {
+        const int s = k & 1;
+        if (!mbar_wait(smem_u32(&sm.item_full[s]), (k >> 1) & 1, abortf, p.budget_ns)) return false;
+        const int4 inf = read_info(&sm.info[s]);
+        mbar_arrive(smem_u32(&sm.item_empty[s]));
+        if (inf.x == kDone) return true;
+        const int role = inf.x, n = inf.w;
+        for (int t = 0; t < n; ++t, ++P) {
+            if (!mbar_wait(smem_u32(&sm.e_full), P & 1, abortf, p.budget_ns)) return false;
+            tc_fence_after();
+            const int r = (int)(P % kRing);
+            if (role == 0) mma_sb(tb0 + kColA0, smem_u32(sm.e[0]), smem_u32(sm.x[r]), t > 0);  // dQ += dS K
+            mma_commit(smem_u32(&sm.bar_a));
+            mma_commit(smem_u32(&sm.tile_empty[r]));
+        }
+    }
+}
+
 __device__ bool issue(const BwdParams& p, WsSmem& sm, const int which)
 {
     volatile int* abortf = &sm.abort_flag;
@@ -403,13 +429,13 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_bwd_ws_kernel(const __grid_c
             mbar_init(smem_u32(&sm.item_full[i]), 1);
             mbar_init(smem_u32(&sm.item_empty[i]), kCompute / 32 + kIssuers);
             mbar_init(smem_u32(&sm.ab_full[i]), 1);
-            mbar_init(smem_u32(&sm.ab_empty[i]), kIssuers);
+            mbar_init(smem_u32(&sm.ab_empty[i]), kSdpIssuers);
         }
         for (int i = 0; i < kRing; ++i) {
             mbar_init(smem_u32(&sm.tile_full[i]), 1);
             mbar_init(smem_u32(&sm.tile_empty[i]), kIssuers);
         }
-        mbar_init(smem_u32(&sm.bar_s), kIssuers);
+        mbar_init(smem_u32(&sm.bar_s), kSdpIssuers);
         mbar_init(smem_u32(&sm.s_free), kCompute / 32);
         mbar_init(smem_u32(&sm.e_full), kCompute / 32);
         mbar_init(smem_u32(&sm.bar_a), kIssuers);
@@ -437,6 +463,8 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_bwd_ws_kernel(const __grid_c
         ok = compute(p, sm);
     else if (threadIdx.x == kIssuer0 || threadIdx.x == kIssuer1)
         ok = issue(p, sm, threadIdx.x == kIssuer1 ? 1 : 0);
+    else if (threadIdx.x == kIssuer2)
+        ok = issue_dq(p, sm);
     else if (warp == kProducer)
         ok = produce(maps, p, sm, nk, P, kab);
     const bool dead = __syncthreads_or(!ok);
@@ -456,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, 2) ssba_bwd_ws_kernel(const __grid_c
                 settle(smem_u32(&sm.tile_full[q % kRing]), (q / kRing) & 1);
             }
         }
-        if (threadIdx.x == kIssuer0 || threadIdx.x == kIssuer1) {  // both commit: the barrier counts two
+        if (threadIdx.x == kIssuer0 || threadIdx.x == kIssuer1 || threadIdx.x == kIssuer2) {  // drain counts 3
             mma_commit(smem_u32(&sm.drain));
             const uint64_t t0 = globaltimer_ns();
             while (!mbar_try_wait(smem_u32(&sm.drain), 0) && globaltimer_ns() - t0 < p.budget_ns) {
