@@ -123,7 +123,9 @@ SSBA_API int ssba_build_mask(const ssba_desc* desc, const void* Q, const void* K
  *               persistent kernel gives its pipelines equal shares of key blocks and
  *               cuts at most one query block per share boundary in two, merging the
  *               parts' partial softmax sums; otherwise shares are whole query blocks
- *               (up to one query block's work of imbalance).
+ *               (up to one query block's work of imbalance). The part that finishes
+ *               second does the merge, so the rows of a cut query block may differ in
+ *               their last bit from one call to the next (within the usual rounding).
  *               Rules: zero-fill it once before its first use. Every call that
  *               returns SSBA_OK and runs to completion leaves it zero-filled again,
  *               so later calls ordered after it on the GPU reuse it as is. Calls that
