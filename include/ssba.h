@@ -176,10 +176,11 @@ SSBA_API int ssba_forward_dense(const ssba_desc* desc, const void* Q, const void
  *   D_n = dO_n . O_n,  dV_m = sum_n p_nm dO_n,  ds_nm = p_nm (dO_n . v_m - D_n),
  *   dQ_n = scale sum_m ds_nm k_m,  dK_m = scale sum_n ds_nm q_n.
  *   Q, K, V, O, dO  device, [B][heads][N][head_dim] of desc->dtype (O and lse as
- *                   ssba_forward wrote them).
- *   lse             device, fp32 [B][heads][N].
- *   kv_idx, kv_cnt  the lists of the forward.
- *   dQ, dK, dV      device out, fp32 [B][heads][N][head_dim], every element written.
+ *                   ssba_forward wrote them), 16-byte aligned.
+ *   lse             device, fp32 [B][heads][N], 4-byte aligned.
+ *   kv_idx, kv_cnt  the lists of the forward, 4-byte aligned.
+ *   dQ, dK, dV      device out, fp32 [B][heads][N][head_dim], 16-byte aligned, every element
+ *                   written.
  *   workspace       device scratch of at least ssba_backward_workspace_bytes(desc) bytes
  *                   (the D_n values and the key blocks' transposed lists), 16-byte aligned,
  *                   one per stream (a call's kernels read what its own first kernel wrote).

@@ -539,11 +539,11 @@ int ssba_backward(const ssba_desc* desc, const void* Q, const void* K, const voi
         set_error("ssba_backward: every pointer must be non-null");
         return SSBA_ERR_INVALID;
     }
-    const size_t es = elem_size(desc);
-    if (!aligned(Q, es) || !aligned(K, es) || !aligned(V, es) || !aligned(O, es) || !aligned(dO, es) ||
-        !aligned(lse, 4) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) || !aligned(dQ, 4) || !aligned(dK, 4) ||
-        !aligned(dV, 4)) {
-        set_error("ssba_backward: pointers must be aligned to their element size");
+    // the kernels copy 16-byte chunks of the rows and store the gradients as float4
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(O, 16) || !aligned(dO, 16) ||
+        !aligned(lse, 4) || !aligned(kv_idx, 4) || !aligned(kv_cnt, 4) || !aligned(dQ, 16) || !aligned(dK, 16) ||
+        !aligned(dV, 16)) {
+        set_error("ssba_backward: tensors must be 16-byte aligned; lse, kv_idx, kv_cnt 4-byte aligned");
         return SSBA_ERR_INVALID;
     }
     const size_t need = ssba_backward_workspace_bytes(desc);

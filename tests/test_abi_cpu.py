@@ -147,6 +147,11 @@ def test_backward_validation(lib):
     assert lib.ssba_backward(*args, None, need, None) == api.SSBA_ERR_WORKSPACE
     bad = [ctypes.byref(d)] + [FAKE] * 5 + [None] + [FAKE] * 5
     assert lib.ssba_backward(*bad, FAKE, need, None) == api.SSBA_ERR_INVALID
+    for i in (1, 2, 3, 4, 6, 9, 10, 11):  # Q, K, V, O, dO, dQ, dK, dV: 16-byte aligned or rejected
+        mis = list(args)
+        mis[i] = FAKE + 4
+        assert lib.ssba_backward(*mis, FAKE, need, None) == api.SSBA_ERR_INVALID, i
+    assert b"16-byte" in lib.ssba_last_error()
     assert lib.ssba_backward_workspace_bytes(ctypes.byref(desc(H_tok=12))) == 0
 
 
