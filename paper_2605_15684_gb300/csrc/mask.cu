@@ -14,7 +14,8 @@
 //   ssba_mask_fused_kernel  both steps in one launch for head_dim 64, 8x8 blocks and at
 //                       most 256 blocks: a cluster of 8 CTAs per (batch, head) pools its
 //                       blocks into shared memory, reads the head's k_b from the other CTAs
-//                       of the cluster (distributed shared memory), and selects its rows. No
+//                       of the cluster (distributed shared memory), and selects its rows
+//                       (keys in registers, the radix walk of sel::ballot_select). No
 //                       q_b/k_b round trip through global memory and no second launch.
 #include <cooperative_groups.h>
 #include <cstdio>
@@ -263,16 +264,44 @@ constexpr int kFuseCluster = 8;    // CTAs per (batch, head)
 constexpr int kFuseWarps = 8;
 constexpr int kFuseMaxTb = 256;
 
+// Affinity row of one query block (S_j = q_b . k_b[j], four interleaved partial sums over d
+// combined in a fixed order, as ssba_select_kernel) with the keys kept in registers (lane l:
+// labels l + 32 m), then the radix walk of sel::ballot_select, which keeps the same labels as
+// sel::rank_select. kbT: the head's k_b transposed, row stride ld.
+template <int kPer>
+__device__ __forceinline__ void affinity_select(const float* q, const float* kbT, int ld, int Tb, int keep, int lane,
+                                                float* srow, int32_t* dst)
+{
+    constexpr int kD = 64;
+    uint32_t key[kPer];
+#pragma unroll
+    for (int m = 0; m < kPer; ++m) {
+        const int j = lane + 32 * m;
+        key[m] = 0u;
+        if (j < Tb) {
+            float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int c = 0; c < kD; c += 4)
+#pragma unroll
+                for (int u = 0; u < 4; ++u) a[u] = fmaf(q[c + u], kbT[(c + u) * ld + j], a[u]);
+            const float acc = (a[0] + a[1]) + (a[2] + a[3]);
+            if (srow) srow[j] = acc;
+            key[m] = sel::order_key(acc);
+        }
+    }
+    sel::ballot_select<kPer>(key, Tb, keep, lane, dst);
+}
+
 // One cluster of kFuseCluster CTAs per (batch*head); CTA r of the cluster owns the blocks
 // [r * bpc, (r + 1) * bpc) ∩ [0, Tb).
-// smem: qown [bpc][64] | kown [bpc][64] | kbT [64][Tb + 1] | S keys [kFuseWarps][Tb]
+// smem: qown [bpc][64] | kown [bpc][64] | kbT [64][Tb + 1]
 //   1. pool: warp w takes (block, tensor) units w, w + 8, ... of its CTA; lane l covers
 //      16-byte chunk l % CPR of rows l / CPR + RPI * i, summed in row order, then across
 //      lanes by shuffles (fixed order); the mean goes to qown / kown.
 //   2. cluster barrier; every CTA copies the head's k_b (transposed) from the owners'
 //      kown into its kbT; cluster barrier again (no CTA leaves while another reads it).
-//   3. one warp per owned query block: S row by four interleaved partial sums over d,
-//      then the exact rank selection of ssba_select_kernel.
+//   3. one warp per owned query block: S row by four interleaved partial sums over d, its
+//      keys in registers, then the radix walk (affinity_select).
 template <typename T>
 __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const T* __restrict__ Q,
                                                                           const T* __restrict__ K, Grid g,
@@ -301,7 +330,6 @@ __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const 
     float* kown = qown + bpc * kD;
     const int ld = Tb + 1;
     float* kbT = kown + bpc * kD;
-    uint32_t* Skey = reinterpret_cast<uint32_t*>(kbT + kD * ld);
 
     // Q and K may come from the grid launched just before this one
     ptx::grid_dep_wait();
@@ -379,28 +407,16 @@ __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const 
     cluster.sync();
 
     // 3. affinity rows and selection
-    uint32_t* S = Skey + (size_t)warp * Tb;
     for (int k = warp; k < nb; k += kFuseWarps) {
         const size_t rowoff = (size_t)bh * Tb + b0 + k;
         const float* q = qown + k * kD;
-        for (int j = lane; j < Tb; j += 32) {
-            float a[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int c = 0; c < kD; c += 4)
-#pragma unroll
-                for (int u = 0; u < 4; ++u) a[u] = fmaf(q[c + u], kbT[(c + u) * ld + j], a[u]);
-            const float acc = (a[0] + a[1]) + (a[2] + a[3]);
-            if (scores) scores[rowoff * Tb + j] = acc;
-            S[j] = sel::order_key(acc);
-        }
-        __syncwarp();
+        float* srow = scores ? scores + rowoff * Tb : nullptr;
         int32_t* dst = idx + rowoff * keep;
-        if (Tb <= 32) sel::rank_select<1>(S, Tb, keep, lane, dst);
-        else if (Tb <= 64) sel::rank_select<2>(S, Tb, keep, lane, dst);
-        else if (Tb <= 128) sel::rank_select<4>(S, Tb, keep, lane, dst);
-        else sel::rank_select<8>(S, Tb, keep, lane, dst);
+        if (Tb <= 32) affinity_select<1>(q, kbT, ld, Tb, keep, lane, srow, dst);
+        else if (Tb <= 64) affinity_select<2>(q, kbT, ld, Tb, keep, lane, srow, dst);
+        else if (Tb <= 128) affinity_select<4>(q, kbT, ld, Tb, keep, lane, srow, dst);
+        else affinity_select<8>(q, kbT, ld, Tb, keep, lane, srow, dst);
         if (lane == 0) cnt[rowoff] = keep;
-        __syncwarp();
     }
 }
 
@@ -575,7 +591,7 @@ int launch_mask_fused(const ssba_desc& d, const Grid& g, int keep, const void* Q
     const int Tb = g.Tb();
     if (d.head_dim != 64 || g.blk != 8 || Tb > kFuseMaxTb) return SSBA_ERR_UNSUPPORTED;
     const int bpc = (Tb + kFuseCluster - 1) / kFuseCluster;
-    const size_t smem = ((size_t)2 * bpc * 64 + (size_t)64 * (Tb + 1) + (size_t)kFuseWarps * Tb) * sizeof(float);
+    const size_t smem = ((size_t)2 * bpc * 64 + (size_t)64 * (Tb + 1)) * sizeof(float);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(kFuseCluster, d.B * d.heads, 1);
     cfg.blockDim = dim3(kFuseWarps * 32, 1, 1);
