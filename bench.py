@@ -851,6 +851,33 @@ def run_ours(args, rank, world):
         except Exception as exc:  # reported, not fatal
             mask_split = f"failed: {exc}"
 
+    # ---- the mask kernel against the HBM roofline: ssba_build_mask (one ssba_mask_fused_kernel
+    #      launch) over the step's layers, each with its own Q and K (larger than L2 together),
+    #      captured in a CUDA graph; algorithmic bytes = Q + K read once
+    mask_roofline = None
+    try:
+        midx = torch.empty((w.B, w.heads, Tb, keep), dtype=torch.int32, device=dev)
+        mcnt = torch.empty((w.B, w.heads, Tb), dtype=torch.int32, device=dev)
+        api.build_mask(descs[0], Qs[0], Ks[0], midx, mcnt, workspace=ws)
+        torch.cuda.synchronize()
+        mgraph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(mgraph):
+            for l in range(L):
+                api.build_mask(descs[l], Qs[l], Ks[l], midx, mcnt, workspace=ws)
+        mgraph.replay()
+        torch.cuda.synchronize()
+        m_us = events_ms(mgraph.replay, 5) / L * 1e3
+        m_bytes = 2 * w.B * w.heads * w.N * w.head_dim * 2
+        m_ach = m_bytes / (m_us * 1e-6) / 1e9
+        mask_roofline = {"kernel": "ssba_mask_fused_kernel (ssba_build_mask)", "bound": "hbm",
+                         "achieved": m_ach, "peak": hbm_gbs, "unit": "GB/s", "frac": m_ach / hbm_gbs,
+                         "us_per_layer": m_us, "algorithmic_bytes": m_bytes,
+                         "how": "one launch per layer over the step's layers (distinct Q, K: larger than "
+                                "L2), captured in a CUDA graph, 5 replays; Q + K read once per launch"}
+        assert api.get_status() == api.SSBA_OK
+    except Exception as exc:  # reported, not fatal
+        mask_roofline = f"failed: {exc}"
+
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": K,
@@ -870,6 +897,7 @@ def run_ours(args, rank, world):
             "configs_sweep": sweep,
             "qkv_fused": qkv,
             "mask_after_fused_pooling": mask_split,
+            "roofline_mask": mask_roofline,
             "speedup_vs_dense": (dense_ms / layer_ms) if isinstance(dense_ms, float) else None,
             "speedup_vs_dense_how": "per layer, both back to back over the step's layers: "
                                     "ssba_forward_dense against the fused sparse launch",

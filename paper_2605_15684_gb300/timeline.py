@@ -2,11 +2,11 @@
 its pipelines, from the time stamps of the timeline build (build.py variant "timeline",
 -DSSBA_TIMELINE; the default library records nothing).
 
-    python -m paper_2605_15684_gb300.timeline [--layers 24] [--isolated] [--phases-only]
+    python -m paper_2605_15684_gb300.timeline [--layers 24] [--isolated] [--phases-only] [--px 1024]
 
 Runs the benchmark's 1024 px step (64 x 64 grid, B = 1, 24 heads x 64, rho = 0.8416, layer l
-with seed l and shift (0,0) / (4,4) alternating, one ssba_forward_fused launch per layer) a few
-times, then reads the stamps of the last launch (layer 23 in the stream, or, with --isolated,
+with seed l and shift (0,0) / (4,4) alternating, one ssba_forward_fused launch per layer; with
+--px 512 or 2048 the 32 x 32 or 128 x 128 grid of those workloads) a few times, then reads the stamps of the last launch (layer 23 in the stream, or, with --isolated,
 one more launch of layer 1 alone) and prints:
   * per phase, the min / median / max over the CTAs of globaltimer microseconds since the first
     CTA's entry (pooling copies landed, means stored, grid barrier, staging, selection,
@@ -92,12 +92,13 @@ def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--layers", type=int, default=24)
     ap.add_argument("--isolated", action="store_true")
+    ap.add_argument("--px", type=int, default=1024, choices=(512, 1024, 2048))
     ap.add_argument("--phases-only", action="store_true",
                     help="the build that records the phase stamps only (per-tile stamps cost time)")
     args = ap.parse_args()
     lib = api.load_library(build.build(variant="phases" if args.phases_only else "timeline"))
     dev = torch.device("cuda", 0)
-    w = synthetic.PX1024
+    w = {512: synthetic.PX512, 1024: synthetic.PX1024, 2048: synthetic.PX2048}[args.px]
     L = args.layers
     descs = [api.SsbaDesc(w.B, w.heads, w.H_tok, w.W_tok, shift_r=4 * (l % 2), shift_c=4 * (l % 2), rho=w.rho,
                           dtype=w.dtype) for l in range(L)]
