@@ -267,9 +267,10 @@ constexpr int kFuseMaxTb = 256;
 // Affinity row of one query block (S_j = q_b . k_b[j], four interleaved partial sums over d
 // combined in a fixed order, as ssba_select_kernel) with the keys kept in registers (lane l:
 // labels l + 32 m), then the radix walk of sel::ballot_select, which keeps the same labels as
-// sel::rank_select. kbT: the head's k_b transposed, row stride ld.
+// sel::rank_select. kbs: the head's k_b by rows, the 16-byte chunk c4 of row j at chunk
+// c4 ^ (j & 15) (so the 32 lanes reading one chunk of 32 rows hit distinct banks pairwise).
 template <int kPer>
-__device__ __forceinline__ void affinity_select(const float* q, const float* kbT, int ld, int Tb, int keep, int lane,
+__device__ __forceinline__ void affinity_select(const float* q, const float* kbs, int Tb, int keep, int lane,
                                                 float* srow, int32_t* dst)
 {
     constexpr int kD = 64;
@@ -279,11 +280,18 @@ __device__ __forceinline__ void affinity_select(const float* q, const float* kbT
         const int j = lane + 32 * m;
         key[m] = 0u;
         if (j < Tb) {
+            const float* row = kbs + j * kD;
+            const int sw = j & 15;
             float a[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int c = 0; c < kD; c += 4)
-#pragma unroll
-                for (int u = 0; u < 4; ++u) a[u] = fmaf(q[c + u], kbT[(c + u) * ld + j], a[u]);
+            for (int c = 0; c < kD; c += 4) {
+                const float4 qv = *reinterpret_cast<const float4*>(q + c);
+                const float4 kv = *reinterpret_cast<const float4*>(row + 4 * ((c >> 2) ^ sw));
+                a[0] = fmaf(qv.x, kv.x, a[0]);
+                a[1] = fmaf(qv.y, kv.y, a[1]);
+                a[2] = fmaf(qv.z, kv.z, a[2]);
+                a[3] = fmaf(qv.w, kv.w, a[3]);
+            }
             const float acc = (a[0] + a[1]) + (a[2] + a[3]);
             if (srow) srow[j] = acc;
             key[m] = sel::order_key(acc);
@@ -294,12 +302,13 @@ __device__ __forceinline__ void affinity_select(const float* q, const float* kbT
 
 // One cluster of kFuseCluster CTAs per (batch*head); CTA r of the cluster owns the blocks
 // [r * bpc, (r + 1) * bpc) ∩ [0, Tb).
-// smem: qown [bpc][64] | kown [bpc][64] | kbT [64][Tb + 1]
+// smem: qown [bpc][64] | kbs [Tb][64] (the head's k_b, 16-byte chunks swizzled by row)
 //   1. pool: warp w takes (block, tensor) units w, w + 8, ... of its CTA; lane l covers
 //      16-byte chunk l % CPR of rows l / CPR + RPI * i, summed in row order, then across
-//      lanes by shuffles (fixed order); the mean goes to qown / kown.
-//   2. cluster barrier; every CTA copies the head's k_b (transposed) from the owners'
-//      kown into its kbT; cluster barrier again (no CTA leaves while another reads it).
+//      lanes by shuffles (fixed order); a q_b mean goes to qown, a k_b mean into kbs of every
+//      CTA of the cluster (distributed shared memory stores, one per CTA and chunk).
+//   2. one cluster barrier (release / acquire: every CTA's stores into kbs are visible after
+//      it, and none follow it, so a CTA may leave once it is done).
 //   3. one warp per owned query block: S row by four interleaved partial sums over d, its
 //      keys in registers, then the radix walk (affinity_select).
 template <typename T>
@@ -327,9 +336,12 @@ __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int N = g.H * g.W;
     float* qown = smf;
-    float* kown = qown + bpc * kD;
-    const int ld = Tb + 1;
-    float* kbT = kown + bpc * kD;
+    float* kbs = qown + bpc * kD;
+
+    // the k_b stores go into the other CTAs' shared memory, which is only valid once every CTA
+    // of the cluster runs: arrive here, wait before the first store (after the first loads)
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    bool started = false;
 
     // Q and K may come from the grid launched just before this one
     ptx::grid_dep_wait();
@@ -370,40 +382,33 @@ __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const 
         for (int o = CPR; o < 32; o <<= 1)
 #pragma unroll
             for (int e = 0; e < VE; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+        if (!started) {  // warp-uniform
+            asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+            started = true;
+        }
         if (r0 == 0) {
-            float* dst = (which ? kown : qown) + k * kD + col * VE;
 #pragma unroll
-            for (int e = 0; e < VE; ++e) dst[e] = acc[e] * (1.0f / 64.0f);
-        }
-    }
-    cluster.sync();
-
-    // 2. gather the head's k_b, transposed: kbT[c][j] = k_b[j][c] (four remote loads in
-    //    flight per thread and round)
-    constexpr int kG = 4;
-    for (int base = 0; base < Tb * (kD / 4); base += kG * kFuseWarps * 32) {
-        float4 v[kG];
+            for (int e = 0; e < VE; ++e) acc[e] *= 1.0f / 64.0f;
+            if (!which) {
+                float* dst = qown + k * kD + col * VE;
 #pragma unroll
-        for (int r = 0; r < kG; ++r) {
-            const int e4 = base + r * kFuseWarps * 32 + threadIdx.x;
-            if (e4 < Tb * (kD / 4)) {
-                const int j = e4 / (kD / 4), c = (e4 - j * (kD / 4)) * 4;
-                const int owner = j / bpc, jl = j - owner * bpc;
-                v[r] = *reinterpret_cast<const float4*>(cluster.map_shared_rank(kown, owner) + jl * kD + c);
-            }
-        }
+                for (int e = 0; e < VE; ++e) dst[e] = acc[e];
+            } else {
+                // chunks col * VE / 4 .. of row `label`, into the k_b of every CTA of the cluster
 #pragma unroll
-        for (int r = 0; r < kG; ++r) {
-            const int e4 = base + r * kFuseWarps * 32 + threadIdx.x;
-            if (e4 < Tb * (kD / 4)) {
-                const int j = e4 / (kD / 4), c = (e4 - j * (kD / 4)) * 4;
-                kbT[(c + 0) * ld + j] = v[r].x;
-                kbT[(c + 1) * ld + j] = v[r].y;
-                kbT[(c + 2) * ld + j] = v[r].z;
-                kbT[(c + 3) * ld + j] = v[r].w;
+                for (int r = 0; r < kFuseCluster; ++r) {
+                    float* rk = cluster.map_shared_rank(kbs, r) + label * kD;
+#pragma unroll
+                    for (int h = 0; h < VE / 4; ++h) {
+                        const int c4 = col * (VE / 4) + h;
+                        *reinterpret_cast<float4*>(rk + 4 * (c4 ^ (label & 15))) =
+                            make_float4(acc[4 * h], acc[4 * h + 1], acc[4 * h + 2], acc[4 * h + 3]);
+                    }
+                }
             }
         }
     }
+    if (!started) asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
     cluster.sync();
 
     // 3. affinity rows and selection
@@ -412,10 +417,10 @@ __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const 
         const float* q = qown + k * kD;
         float* srow = scores ? scores + rowoff * Tb : nullptr;
         int32_t* dst = idx + rowoff * keep;
-        if (Tb <= 32) affinity_select<1>(q, kbT, ld, Tb, keep, lane, srow, dst);
-        else if (Tb <= 64) affinity_select<2>(q, kbT, ld, Tb, keep, lane, srow, dst);
-        else if (Tb <= 128) affinity_select<4>(q, kbT, ld, Tb, keep, lane, srow, dst);
-        else affinity_select<8>(q, kbT, ld, Tb, keep, lane, srow, dst);
+        if (Tb <= 32) affinity_select<1>(q, kbs, Tb, keep, lane, srow, dst);
+        else if (Tb <= 64) affinity_select<2>(q, kbs, Tb, keep, lane, srow, dst);
+        else if (Tb <= 128) affinity_select<4>(q, kbs, Tb, keep, lane, srow, dst);
+        else affinity_select<8>(q, kbs, Tb, keep, lane, srow, dst);
         if (lane == 0) cnt[rowoff] = keep;
     }
 }
@@ -591,7 +596,7 @@ int launch_mask_fused(const ssba_desc& d, const Grid& g, int keep, const void* Q
     const int Tb = g.Tb();
     if (d.head_dim != 64 || g.blk != 8 || Tb > kFuseMaxTb) return SSBA_ERR_UNSUPPORTED;
     const int bpc = (Tb + kFuseCluster - 1) / kFuseCluster;
-    const size_t smem = ((size_t)2 * bpc * 64 + (size_t)64 * (Tb + 1)) * sizeof(float);
+    const size_t smem = ((size_t)bpc * 64 + (size_t)Tb * 64) * sizeof(float);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(kFuseCluster, d.B * d.heads, 1);
     cfg.blockDim = dim3(kFuseWarps * 32, 1, 1);
