@@ -37,6 +37,9 @@ METRIC = "SSBA fwd latency (ms) and effective TFLOP/s @4096 tok, 84% sparse, bf1
 ATTN_SOURCES = ("paper_2605_15684_gb300/csrc/attn_tc.cu", "paper_2605_15684_gb300/csrc/ptx.cuh",
                 "paper_2605_15684_gb300/csrc/window.cuh")
 ATTN_PROFILE = os.path.join(ROOT, "profiles", "ssba_attn_tc_kernel_1024px.md")
+MASK_SOURCES = ("paper_2605_15684_gb300/csrc/mask.cu", "paper_2605_15684_gb300/csrc/select.cuh",
+                "paper_2605_15684_gb300/csrc/ptx.cuh")
+MASK_PROFILE = os.path.join(ROOT, "profiles", "ssba_mask_fused_kernel_1024px.md")
 
 
 def parse_args():
@@ -197,18 +200,18 @@ def measured_peaks():
     return 6800.0, 1900.0, "fallback"
 
 
-def profiled_traffic():
-    """DRAM bytes per launch of the attention kernel from the committed ncu summary, if
-    the kernel source is unchanged since the capture (else None)."""
-    if not os.path.exists(ATTN_PROFILE):
+def profiled_traffic(profile=ATTN_PROFILE, sources=ATTN_SOURCES):
+    """DRAM bytes per launch of a kernel from its committed ncu summary, if the kernel's
+    sources are unchanged since the capture (else None)."""
+    if not os.path.exists(profile):
         return None
-    text = open(ATTN_PROFILE).read()
+    text = open(profile).read()
     m_b = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
     m_h = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
     if not m_b or not m_h:
         return None
     h = hashlib.sha256()
-    for rel in ATTN_SOURCES:
+    for rel in sources:
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
     return int(m_b.group(1)) if h.hexdigest() == m_h.group(1) else None
@@ -871,6 +874,7 @@ def run_ours(args, rank, world):
         m_ach = m_bytes / (m_us * 1e-6) / 1e9
         mask_roofline = {"kernel": "ssba_mask_fused_kernel (ssba_build_mask)", "bound": "hbm",
                          "achieved": m_ach, "peak": hbm_gbs, "unit": "GB/s", "frac": m_ach / hbm_gbs,
+                         "traffic": profiled_traffic(MASK_PROFILE, MASK_SOURCES),
                          "us_per_layer": m_us, "algorithmic_bytes": m_bytes,
                          "how": "one launch per layer over the step's layers (distinct Q, K: larger than "
                                 "L2), captured in a CUDA graph, 5 replays; Q + K read once per launch"}
