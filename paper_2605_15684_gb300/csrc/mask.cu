@@ -268,7 +268,8 @@ constexpr int kFuseMaxTb = 256;
 // combined in a fixed order, as ssba_select_kernel) with the keys kept in registers (lane l:
 // labels l + 32 m), then the radix walk of sel::ballot_select, which keeps the same labels as
 // sel::rank_select. kbs: the head's k_b by rows, the 16-byte chunk c4 of row j at chunk
-// c4 ^ (j & 15) (so the 32 lanes reading one chunk of 32 rows hit distinct banks pairwise).
+// c4 ^ (j & 15) (the 32 lanes reading one chunk of 32 rows cover all 32 banks: four wavefronts,
+// the least for 512 bytes).
 template <int kPer>
 __device__ __forceinline__ void affinity_select(const float* q, const float* kbs, int Tb, int keep, int lane,
                                                 float* srow, int32_t* dst)
@@ -409,6 +410,7 @@ __global__ void __launch_bounds__(kFuseWarps * 32) ssba_mask_fused_kernel(const 
         }
     }
     if (!started) asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+    // 2. every k_b row of the head is in this CTA's kbs after the barrier
     cluster.sync();
 
     // 3. affinity rows and selection
