@@ -12,7 +12,12 @@ layer has its own seeded synthetic Q/K/V (906 MB in all), so every layer's input
 cold in L2 when it runs.
 
 Prints one JSON line. value = effective TFLOP/s counting only the kept blocks
-(4 * B * heads * Tb * keep * 64 * 64 * head_dim per layer) over the whole step.
+(4 * B * heads * Tb * keep * 64 * 64 * head_dim per layer) over the whole step. Beside it:
+`roofline` (the fused launch against the bf16 peak), `roofline_mask` (the mask kernel of
+ssba_build_mask against the HBM peak), `roofline_pool`, `configs_sweep` (the paper's other
+workloads, each on the fused launch and, as `two_call_ms_per_layer`, through
+ssba_build_mask + ssba_forward), the same-build dense kernel, the backward, the NEXT rows'
+kernels, `e2e`, `cpu_baseline` and the clocks sampled during the timed region.
 ``--impl reference`` times the CPU oracle on the host cores instead.
 """
 from __future__ import annotations
